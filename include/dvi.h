@@ -1,0 +1,231 @@
+/*
+ * dvi.h -- C-ABI of the GB300 (sm_103a) DVI library.
+ *
+ * DVI (Draft, Verify & Improve, arxiv 2510.05421) splits one decoder at layer
+ * k (Sec. 3.1): layers 1..k plus a LoRA drafter head greedily propose k_spec
+ * tokens; the frozen layers k+1..L plus the LM head verify the whole block in
+ * one multi-query pass; the longest agreeing prefix is committed and the KV
+ * cache rolled back past it (Sec. 3.3); the logged accept/reject tuples drive
+ * an online KL->RL update of the drafter head (Sec. 3.4).
+ *
+ * Conventions shared by every call
+ *  - Memory.  The caller owns all device memory: weights, the workspace and
+ *    every input/output buffer.  The library never allocates or frees device
+ *    memory.  A context keeps raw pointers to the weights and the workspace;
+ *    both must outlive it.
+ *  - Asynchrony.  Every call only enqueues work on the context's stream and
+ *    returns.  Argument errors are reported synchronously through the return
+ *    value.  Errors found on the device (non-finite logits or loss, KV or
+ *    buffer capacity, a bounded wait that ran out) set bits of a device
+ *    status word that dvi_get_stats() reads.
+ *  - Threads.  A context is used by one host thread at a time.  No C++
+ *    exception crosses this interface.
+ *  - Layout.  Matrices are row-major with the output feature as the row
+ *    (torch nn.Linear layout): W[out][in].  Token ids are int32.
+ */
+#ifndef DVI_H_
+#define DVI_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct dvi_ctx dvi_ctx;           /* opaque, host-side */
+typedef struct CUstream_st* dvi_stream;   /* a cudaStream_t */
+
+typedef enum {
+  DVI_OK = 0,
+  DVI_ERR_INVALID_ARG = -1,
+  DVI_ERR_CAPACITY = -2,
+  DVI_ERR_NONFINITE = -3,
+  DVI_ERR_CUDA = -4,
+  DVI_ERR_UNIMPLEMENTED = -5,
+  DVI_ERR_TIMEOUT = -6
+} dvi_status;
+
+/* bits of dvi_stats.device_status */
+enum {
+  DVI_DEV_NONFINITE = 1,   /* a NaN/Inf logit, or a non-finite update loss (update skipped) */
+  DVI_DEV_TIMEOUT = 2,     /* a bounded device wait gave up */
+  DVI_DEV_KV_FULL = 4,     /* a KV row fell past max_seq_len (row not written) */
+  DVI_DEV_BAD_TOKEN = 8,   /* a token id outside [0, vocab) */
+  DVI_DEV_LOG_FULL = 16    /* the replay buffer was full; tuples of a step were dropped */
+};
+
+typedef enum { DVI_F32 = 0, DVI_BF16 = 1 } dvi_dtype;
+
+/* The decoder (Sec. 3.1; the backbone is Llama-style: pre-norm RMSNorm,
+ * RoPE rotate-half, SwiGLU, GQA).  dtype applies to the weight matrices,
+ * the KV cache and the activations fed to matrix products.  Norm gains and
+ * the LoRA factors are always float32. */
+typedef struct {
+  int n_layers;       /* L */
+  int d_model;        /* d, a multiple of 128 */
+  int n_heads;        /* H_q */
+  int n_kv_heads;     /* H_kv, divides H_q */
+  int head_dim;       /* 64 or 128 */
+  int d_ffn;          /* F */
+  int vocab;          /* V */
+  int split_k;        /* k: draft path = layers 1..k, verify path = k+1..L; 1 <= k <= L */
+  int lora_rank;      /* r of A_s [V][r], B_s [r][d]; 0 = no LoRA */
+  float lora_gamma;   /* gamma_s */
+  float rms_eps;      /* 1e-5 */
+  float rope_theta;   /* 10000 */
+  int dtype;          /* dvi_dtype */
+} dvi_model_config;
+
+typedef struct {
+  int batch;            /* B sequences decoded together */
+  int k_spec;           /* K: drafted tokens per step, 1 <= K <= 16 / (H_q / H_kv) */
+  int max_seq_len;      /* KV rows per sequence: prompt + generated + K */
+  int log_steps;        /* decode steps the replay buffer holds between updates (U) */
+  int head_mode;        /* 0: train LoRA A_s, B_s on the frozen W^(S); 1: train W^(S) itself */
+  int max_prefill_chunk;/* rows per prefill pass, 16..128 (multiple of 16); 0 = 128 */
+  int use_graphs;       /* capture the decode step in a CUDA graph on first use */
+} dvi_runtime_config;
+
+typedef struct {
+  const void* attn_norm;   /* [d] f32 */
+  const void* wq;          /* [H_q*hd][d] */
+  const void* wk;          /* [H_kv*hd][d] */
+  const void* wv;          /* [H_kv*hd][d] */
+  const void* wo;          /* [d][H_q*hd] */
+  const void* ffn_norm;    /* [d] f32 */
+  const void* w_gate;      /* [F][d] */
+  const void* w_up;        /* [F][d] */
+  const void* w_down;      /* [d][F] */
+} dvi_layer_weights;
+
+/* Device pointers, caller-owned, read for the whole life of the context.
+ * draft_head (W^(S)) may alias lm_head (W^(V)) only when head_mode == 0.
+ * lora_a / lora_b are updated in place by dvi_update_drafter (head_mode 0);
+ * draft_head is updated in place in head_mode 1. */
+typedef struct {
+  const void* embed;              /* [V][d] */
+  const dvi_layer_weights* layers;/* host array of L entries */
+  const void* final_norm;         /* [d] f32 */
+  const void* lm_head;            /* W^(V) [V][d], frozen */
+  void* draft_head;               /* W^(S) [V][d] */
+  float* lora_a;                  /* A_s [V][r] f32 */
+  float* lora_b;                  /* B_s [r][d] f32 */
+} dvi_weights;
+
+/* Drafter-update hyper-parameters (Sec. 3.4).  objective: 0 = the KL->RL
+ * schedule (L_fast, plus L_policy once t >= t_warmup), 1 = KL only, 2 = PG
+ * only (REINFORCE), 3 = reward-masked CE only (the ablations of Sec. 4.3).
+ * optimizer: 0 = bias-corrected Adam, 1 = SGD. */
+typedef struct {
+  int objective;
+  int optimizer;
+  float lr, beta1, beta2, adam_eps;
+  float tau;                                  /* KD temperature */
+  float lambda0, lambda_kl_min, lambda_pg_max;
+  int t_warmup, t_ramp;
+  float w_ce, w_ent, w_rl_max;
+  float beta0, beta_min, t_beta;              /* beta(t) of L_policy */
+  float baseline_rho;                         /* EMA constant of the reward baseline b */
+} dvi_update_config;
+
+typedef struct {
+  int64_t steps;          /* draft_verify_commit calls */
+  int64_t drafted;        /* sum over sequences of K per step */
+  int64_t accepted;       /* sum of m (mean accepted length = accepted / (steps * B)) */
+  int64_t committed;      /* tokens committed by decode steps */
+  int64_t updates;        /* drafter updates applied */
+  int64_t kernel_launches;/* kernels this context enqueued (graph replays count their nodes) */
+  float last_loss;        /* objective of the last update */
+  float last_kl, last_pg, last_ce, last_ent, last_rl, last_kl1;
+  float last_accept_rate; /* accepted / logged rows of the last update's buffer */
+  float baseline_b;       /* EMA reward baseline after the last update */
+  int update_t;           /* completed updates t (the schedule's clock) */
+  int device_status;      /* DVI_DEV_* bits */
+} dvi_stats;
+
+/* Bytes of device workspace a context needs (KV caches, residual streams,
+ * replay buffer, optimizer state, scratch).  0 for an invalid config. */
+size_t dvi_workspace_bytes(const dvi_model_config* cfg, const dvi_runtime_config* rt);
+
+/* "Load split model" (Sec. 3.1): validate the config, keep the weight
+ * pointers, carve `workspace` (>= dvi_workspace_bytes, 256-byte aligned,
+ * contents arbitrary) and enqueue its initialisation on `stream`.  Builds
+ * the TMA descriptors of every weight matrix. */
+dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
+                      const dvi_weights* weights, void* workspace,
+                      size_t workspace_bytes, dvi_stream stream, dvi_ctx** out);
+
+/* Reset sequence `seq` and run its prompt (device int32 [n_tokens]) through
+ * all L layers, filling the KV cache; the greedy next token (the first
+ * generated token, committed) becomes the pending token of the sequence and
+ * is written to d_first_token (device int32 [1]) when non-null. */
+dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tokens,
+                       int32_t* d_first_token);
+
+/* One DVI step for all B sequences (Sec. 3.3): K greedy draft passes through
+ * layers 1..k and the drafter head, one verify pass of the K rows through
+ * layers k+1..L and the LM head, accept length m, commit and rollback, and
+ * (when logging is on) the replay-buffer tuples of positions 1..min(m+1, K).
+ * Outputs (device, may be null): d_out_ids [B][K] committed ids (the first
+ * d_n_committed[b] = min(m+1, K) entries of row b are valid), d_n_accepted
+ * [B] = m. */
+dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids,
+                                   int32_t* d_n_committed, int32_t* d_n_accepted);
+
+/* Replay-buffer logging on (1, the default) or off (0) for later steps. */
+dvi_status dvi_log(dvi_ctx* ctx, int enable);
+
+/* One drafter-head update on every tuple logged since the last update
+ * (Sec. 3.4), then clear the buffer and advance t.  A non-finite loss skips
+ * the parameter step and sets DVI_DEV_NONFINITE. */
+dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* ucfg);
+
+/* Baseline: one greedy autoregressive step of the full model for every
+ * sequence (the speedup denominator of Sec. 4.1); commits one token each.
+ * d_out_ids: device int32 [B] or null. */
+dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids);
+
+/* Synchronise the context's stream and copy the counters to *out. */
+dvi_status dvi_get_stats(dvi_ctx* ctx, dvi_stats* out);
+
+/* Message of the last synchronous error on this context ("" if none). */
+const char* dvi_last_error(const dvi_ctx* ctx);
+
+/* Free the host-side context (never the caller's device memory). */
+dvi_status dvi_destroy(dvi_ctx* ctx);
+
+/* Inspection of internal device buffers for tests and tools: sets *dptr and
+ * *bytes for buffer `which` (DVI_BUF_*).  The memory stays owned by the
+ * workspace. */
+enum {
+  DVI_BUF_LENS = 0,        /* int32 [B] committed KV length n per sequence */
+  DVI_BUF_PENDING = 1,     /* int32 [B] pending (last committed) token */
+  DVI_BUF_DRAFT_IDS = 2,   /* int32 [B][K+1]: pending, t~_1..t~_K of the last step */
+  DVI_BUF_LOG_U = 3,       /* dtype [cap][d] logged head inputs u = RMSNorm_final(h_k) */
+  DVI_BUF_LOG_LOGITS = 4,  /* f32 [cap][V] logged verifier logits */
+  DVI_BUF_LOG_META = 5,    /* int32 [cap][6]: valid, a, r, i, prev_id, y* */
+  DVI_BUF_GRAD_A = 6,      /* f32 [V][r] last dL/dA */
+  DVI_BUF_GRAD_B = 7,      /* f32 [r][d] last dL/dB */
+  DVI_BUF_X_DRAFT = 8,     /* f32 [B][d] residual stream of the draft pass */
+  DVI_BUF_X_VERIFY = 9,    /* f32 [B*K][d] h_k rows, then h_L after verify */
+  DVI_BUF_K_CACHE = 10,    /* dtype [L][B][H_kv][max_seq_len][hd] */
+  DVI_BUF_V_CACHE = 11,
+  DVI_BUF_STATUS = 12,     /* int32 device status word */
+  DVI_BUF_GRAD_W = 13,     /* f32 [V][d] last dL/dW^(S) (head_mode 1) */
+  DVI_BUF_Z = 14,          /* f32 [cap][V] drafter logits of the last update */
+  DVI_BUF_COUNT
+};
+dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes);
+
+/* Y[M][n_out] = X[M][K] . W[n_out][K]^T through the library's projection
+ * kernel (tcgen05 for bf16, FP32 FMA for f32), with X float32 (rounded to the
+ * weight dtype first) and Y float32, on the context's stream.  M <= 256.
+ * A building block exposed for tests of the projection kernel itself. */
+dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in,
+                      const float* d_x, int m_rows, float* d_y);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DVI_H_ */

@@ -1,0 +1,903 @@
+// C-ABI of the DVI library (include/dvi.h): context, workspace layout and the
+// order in which the kernels of each call are enqueued.
+//
+//  prefill              chunks of the prompt through layers 1..L, verifier head
+//                       on the last row -> first committed token (Sec. 3.1)
+//  draft_verify_commit  K draft passes (layers 1..k + drafter head), one verify
+//                       pass (layers k+1..L on the K rows + LM head), accept /
+//                       commit / rollback / log (Sec. 3.3); captured once into
+//                       a CUDA graph and replayed (all state is device-side)
+//  update_drafter       the KL->RL update of the drafter head (Sec. 3.4)
+//  ar_step              greedy AR step of the full model (Sec. 4.1 baseline)
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace dvi;
+
+namespace {
+
+struct LayerMaps {
+  ProjMaps qkv, o, gu, down;
+};
+
+struct Pass {
+  float* x;
+  float* ss;
+  int ss_ld;
+  int M;
+  int rows_per_seq;
+  int seq0;
+  int n_seqs;
+  int pos_off;
+};
+
+struct Plan {
+  int n_tiles, n_splits, kb_total, kb_per_split;
+};
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+struct dvi_ctx {
+  dvi_model_config cfg;
+  dvi_runtime_config rt;
+  dvi_weights w;
+  std::vector<dvi_layer_weights> layers;
+  cudaStream_t stream = nullptr;
+  int n_sms = 152;
+  bool tc = false;
+  size_t esz = 4;
+  int L, d, Hq, Hkv, hd, F, V, k, r, B, K, max_len, cap_steps, cap_rows, chunk, M_max, nq, nkv;
+  // device state
+  int *lens, *pending, *draft_ids, *status, *log_step, *log_meta;
+  long long* counters;
+  float* dev_state;
+  float *x_dr, *ss_dr, *x_ver, *ss_ver, *x_pf, *ss_pf, *q, *bu;
+  void *attn_o, *ffn_h, *u_buf;
+  unsigned long long* amax;
+  void *kcache, *vcache;
+  float2* rope;
+  float* part;
+  size_t part_floats;
+  int* proj_counters;
+  int n_proj_counters;
+  float* attn_part;
+  size_t attn_part_floats;
+  int* attn_ctr;
+  int n_attn_ctr;
+  int attn_split_len, attn_nsplits;
+  void* log_u;
+  float* log_logits;
+  float *Z, *rowstat, *coef, *ub, *ga, *ga_part;
+  float *m_a, *v_a, *m_b, *v_b, *grad_a, *grad_b;
+  int *out_ids, *n_committed, *n_accepted, *ar_out;
+  size_t ws_bytes;
+  void* ws;
+  // plans and TMA descriptors
+  Plan p_qkv, p_o, p_gu, p_down, p_head;
+  std::vector<LayerMaps> maps;
+  ProjMaps head_v, head_s;
+  int log_enabled = 1;
+  // graph of one decode step
+  cudaGraphExec_t step_exec = nullptr;
+  int step_calls = 0;
+  long long step_launches = 0;
+  long long launches = 0;
+  std::string err;
+};
+
+namespace {
+
+dvi_status fail(dvi_ctx* c, dvi_status s, const char* msg) {
+  if (c) c->err = msg;
+  return s;
+}
+
+#define DVI_CUDA(call)                                                                 \
+  do {                                                                                 \
+    cudaError_t e_ = (call);                                                           \
+    if (e_ != cudaSuccess) {                                                           \
+      ctx->err = std::string(#call) + ": " + cudaGetErrorString(e_);                   \
+      return DVI_ERR_CUDA;                                                             \
+    }                                                                                  \
+  } while (0)
+
+bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::string* why) {
+  auto bad = [&](const char* m) { if (why) *why = m; return false; };
+  if (!c || !rt) return bad("null config");
+  if (c->dtype != DVI_F32 && c->dtype != DVI_BF16) return bad("dtype must be DVI_F32 or DVI_BF16");
+  if (c->n_layers < 1 || c->d_model < 128 || c->d_model % 128) return bad("d_model must be a positive multiple of 128");
+  if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads) return bad("n_kv_heads must divide n_heads");
+  if (c->head_dim != 64 && c->head_dim != 128) return bad("head_dim must be 64 or 128");
+  if ((c->n_heads * c->head_dim) % 128 || (c->n_kv_heads * c->head_dim) % 128)
+    return bad("H*head_dim must be multiples of 128");
+  if (c->n_heads / c->n_kv_heads > kAttnQ) return bad("GQA group larger than 16");
+  if (c->d_ffn < 1 || c->vocab < 2) return bad("bad d_ffn / vocab");
+  if (c->dtype == DVI_BF16 && c->d_ffn % 8) return bad("bf16 needs d_ffn % 8 == 0");
+  if (c->split_k < 1 || c->split_k > c->n_layers) return bad("split_k must be in [1, n_layers]");
+  if (c->lora_rank < 0 || c->lora_rank > 64) return bad("lora_rank must be in [0, 64]");
+  if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f)) return bad("bad rms_eps / rope_theta");
+  if (rt->batch < 1 || rt->batch > 64) return bad("batch must be in [1, 64]");
+  if (rt->k_spec < 1 || rt->k_spec > 16) return bad("k_spec must be in [1, 16]");
+  if (rt->max_seq_len < rt->k_spec + 2) return bad("max_seq_len too small");
+  if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
+    return bad("log_steps * batch * k_spec must be in [1, 256]");
+  if (rt->head_mode != 0) return bad("head_mode 1 (full W^S training) is not available");
+  if (rt->max_prefill_chunk && (rt->max_prefill_chunk < 16 || rt->max_prefill_chunk > 128 || rt->max_prefill_chunk % 16))
+    return bad("max_prefill_chunk must be 16..128, a multiple of 16");
+  if (rt->batch * rt->k_spec > kMaxTokens) return bad("batch * k_spec > 256");
+  return true;
+}
+
+// The one place the workspace layout is defined: walks the buffers in order,
+// either measuring (base == nullptr) or assigning pointers.
+size_t layout(dvi_ctx* c, char* base) {
+  size_t off = 0;
+  auto take = [&](size_t bytes) -> char* {
+    off = align_up(off, 256);
+    char* p = base ? base + off : nullptr;
+    off += bytes;
+    return p;
+  };
+  const size_t e = c->esz;
+  const int B = c->B, K = c->K, d = c->d, V = c->V, r = c->r;
+  const int st = d / kTileRows;
+  c->lens = reinterpret_cast<int*>(take(sizeof(int) * B));
+  c->pending = reinterpret_cast<int*>(take(sizeof(int) * B));
+  c->draft_ids = reinterpret_cast<int*>(take(sizeof(int) * B * (K + 1)));
+  c->status = reinterpret_cast<int*>(take(sizeof(int) * 4));
+  c->log_step = reinterpret_cast<int*>(take(sizeof(int) * 4));
+  c->log_meta = reinterpret_cast<int*>(take(sizeof(int) * 6 * c->cap_rows));
+  c->counters = reinterpret_cast<long long*>(take(sizeof(long long) * 8));
+  c->dev_state = reinterpret_cast<float*>(take(sizeof(float) * 16));
+  c->x_dr = reinterpret_cast<float*>(take(sizeof(float) * B * d));
+  c->ss_dr = reinterpret_cast<float*>(take(sizeof(float) * st * B));
+  c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * K * d));
+  c->ss_ver = reinterpret_cast<float*>(take(sizeof(float) * st * B * K));
+  c->x_pf = reinterpret_cast<float*>(take(sizeof(float) * c->chunk * d));
+  c->ss_pf = reinterpret_cast<float*>(take(sizeof(float) * st * c->chunk));
+  c->q = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * c->nq));
+  c->bu = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * (r > 0 ? r : 1)));
+  c->attn_o = take(e * c->M_max * c->nq);
+  c->ffn_h = take(e * c->M_max * c->F);
+  c->u_buf = take(e * c->M_max * d);
+  c->amax = reinterpret_cast<unsigned long long*>(take(sizeof(unsigned long long) * c->M_max));
+  const size_t kv = static_cast<size_t>(c->L) * B * c->Hkv * c->max_len * c->hd;
+  c->kcache = take(e * kv);
+  c->vcache = take(e * kv);
+  c->rope = reinterpret_cast<float2*>(take(sizeof(float2) * static_cast<size_t>(c->max_len) * (c->hd / 2)));
+  c->part = reinterpret_cast<float*>(take(sizeof(float) * c->part_floats));
+  c->proj_counters = reinterpret_cast<int*>(take(sizeof(int) * c->n_proj_counters));
+  c->attn_part = reinterpret_cast<float*>(take(sizeof(float) * c->attn_part_floats));
+  c->attn_ctr = reinterpret_cast<int*>(take(sizeof(int) * c->n_attn_ctr));
+  c->log_u = take(e * c->cap_rows * d);
+  c->log_logits = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
+  c->Z = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
+  c->rowstat = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * 8));
+  c->coef = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * 8));
+  const int rr = r > 0 ? r : 1;
+  c->ub = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * rr));
+  c->ga = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * rr));
+  const int nvt = (V + 127) / 128;
+  c->ga_part = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(nvt) * c->cap_rows * rr));
+  c->m_a = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(V) * rr));
+  c->v_a = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(V) * rr));
+  c->grad_a = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(V) * rr));
+  c->m_b = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(rr) * d));
+  c->v_b = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(rr) * d));
+  c->grad_b = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(rr) * d));
+  c->out_ids = reinterpret_cast<int*>(take(sizeof(int) * B * K));
+  c->n_committed = reinterpret_cast<int*>(take(sizeof(int) * B));
+  c->n_accepted = reinterpret_cast<int*>(take(sizeof(int) * B));
+  c->ar_out = reinterpret_cast<int*>(take(sizeof(int) * B));
+  return align_up(off, 256);
+}
+
+Plan plan_for(dvi_ctx* c, int flavor, int n_out, int K, int rq, int rk, int rv) {
+  ProjArgs a{};
+  a.flavor = flavor;
+  a.n_out = n_out;
+  a.K = K;
+  a.rows_q = rq;
+  a.rows_k = rk;
+  a.rows_v = rv;
+  plan_splits(a, c->n_sms, c->tc);
+  return Plan{a.n_tiles, a.n_splits, a.kb_total, a.kb_per_split};
+}
+
+void size_scratch(dvi_ctx* c) {
+  const int Ms[2] = {c->M_max, 1};
+  size_t part = 0;
+  int ctr = 0;
+  const Plan* plans[5] = {&c->p_qkv, &c->p_o, &c->p_gu, &c->p_down, &c->p_head};
+  const int flav[5] = {EPI_QKV, EPI_RESID, EPI_GATEUP, EPI_RESID, EPI_HEAD};
+  for (int i = 0; i < 5; ++i) {
+    for (int M : Ms) {
+      ProjArgs a{};
+      a.flavor = flav[i];
+      a.M = M;
+      a.n_pad = (M + 15) / 16 * 16;
+      a.n_tiles = plans[i]->n_tiles;
+      a.n_splits = plans[i]->n_splits;
+      part = std::max(part, proj_partial_floats(a, c->tc));
+      const int ntt = c->tc ? 1 : (M + kChunk - 1) / kChunk;
+      ctr = std::max(ctr, a.n_tiles * ntt);
+    }
+  }
+  // room for dvi_linear on modest shapes: 8 Mi floats of partials
+  c->part_floats = std::max(part, static_cast<size_t>(8) << 20);
+  c->n_proj_counters = std::max(ctr, 4096);
+  // attention: fixed split length from the capacity so row results do not
+  // depend on the number of rows; about 3 CTAs per SM at full length.
+  const int target = 3 * c->n_sms;
+  int splits = std::max(1, target / std::max(1, c->B * c->Hkv));
+  int sl = (c->max_len + splits - 1) / splits;
+  sl = std::max(kAttnBlk, (sl + kAttnBlk - 1) / kAttnBlk * kAttnBlk);
+  c->attn_split_len = sl;
+  c->attn_nsplits = (c->max_len + sl - 1) / sl;
+  AttnArgs at{};
+  at.n_heads = c->Hq;
+  at.n_kv_heads = c->Hkv;
+  at.head_dim = c->hd;
+  at.n_splits_max = c->attn_nsplits;
+  size_t ap = 0;
+  int ac = 0;
+  const int rps[3] = {c->K, 1, c->chunk};
+  const int nse[3] = {c->B, c->B, 1};
+  for (int i = 0; i < 3; ++i) {
+    at.rows_per_seq = rps[i];
+    at.n_seqs = nse[i];
+    ap = std::max(ap, attn_partial_floats(at));
+    ac = std::max(ac, attn_counters(at));
+  }
+  c->attn_part_floats = ap;
+  c->n_attn_ctr = ac;
+}
+
+bool init_dims(dvi_ctx* c, const dvi_model_config* cfg, const dvi_runtime_config* rt) {
+  c->cfg = *cfg;
+  c->rt = *rt;
+  c->L = cfg->n_layers;
+  c->d = cfg->d_model;
+  c->Hq = cfg->n_heads;
+  c->Hkv = cfg->n_kv_heads;
+  c->hd = cfg->head_dim;
+  c->F = cfg->d_ffn;
+  c->V = cfg->vocab;
+  c->k = cfg->split_k;
+  c->r = cfg->lora_rank;
+  c->B = rt->batch;
+  c->K = rt->k_spec;
+  c->max_len = rt->max_seq_len;
+  c->cap_steps = rt->log_steps;
+  c->cap_rows = rt->log_steps * rt->batch * rt->k_spec;
+  c->chunk = rt->max_prefill_chunk ? rt->max_prefill_chunk : 128;
+  c->M_max = std::max(std::max(c->B * c->K, c->chunk), std::max(c->cap_rows, c->B));
+  c->nq = c->Hq * c->hd;
+  c->nkv = c->Hkv * c->hd;
+  c->tc = cfg->dtype == DVI_BF16;
+  c->esz = c->tc ? 2 : 4;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0) c->n_sms = n;
+  }
+  c->p_qkv = plan_for(c, EPI_QKV, 0, c->d, c->nq, c->nkv, c->nkv);
+  c->p_o = plan_for(c, EPI_RESID, c->d, c->nq, 0, 0, 0);
+  c->p_gu = plan_for(c, EPI_GATEUP, c->F, c->d, 0, 0, 0);
+  c->p_down = plan_for(c, EPI_RESID, c->d, c->F, 0, 0, 0);
+  c->p_head = plan_for(c, EPI_HEAD, c->V, c->d, 0, 0, 0);
+  size_scratch(c);
+  return true;
+}
+
+ProjArgs base_args(dvi_ctx* c, int flavor, const Plan& pl, const Pass& ps) {
+  ProjArgs a{};
+  a.flavor = flavor;
+  a.dtype = c->cfg.dtype;
+  a.M = ps.M;
+  a.n_pad = (ps.M + 15) / 16 * 16;
+  a.n_tiles = pl.n_tiles;
+  a.n_splits = pl.n_splits;
+  a.kb_total = pl.kb_total;
+  a.kb_per_split = pl.kb_per_split;
+  a.n_ttiles = 1;
+  a.lens = c->lens;
+  a.rows_per_seq = ps.rows_per_seq;
+  a.seq0 = ps.seq0;
+  a.pos_off = ps.pos_off;
+  a.part = c->part;
+  a.counters = c->proj_counters;
+  a.status = c->status;
+  a.eps = c->cfg.rms_eps;
+  a.d_norm = c->d;
+  a.ss_tiles = c->d / kTileRows;
+  return a;
+}
+
+size_t layer_kv_offset(dvi_ctx* c, int l) {
+  return static_cast<size_t>(l) * c->B * c->Hkv * c->max_len * c->hd * c->esz;
+}
+
+dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps) {
+  const dvi_layer_weights& lw = ctx->layers[l];
+  const LayerMaps* mp = ctx->tc ? &ctx->maps[l] : nullptr;
+  cudaStream_t s = ctx->stream;
+  // q, k, v with RoPE; k, v rows into the cache
+  ProjArgs a = base_args(ctx, EPI_QKV, ctx->p_qkv, ps);
+  a.b_mode = B_NORM;
+  a.x = ps.x;
+  a.ldx = ctx->d;
+  a.ss = ps.ss;
+  a.ss_ld = ps.ss_ld;
+  a.gain = static_cast<const float*>(lw.attn_norm);
+  a.K = ctx->d;
+  a.rows_q = ctx->nq;
+  a.rows_k = ctx->nkv;
+  a.rows_v = ctx->nkv;
+  a.n_out = ctx->nq;
+  a.w0 = lw.wq;
+  a.w1 = lw.wk;
+  a.w2 = lw.wv;
+  a.q_out = ctx->q;
+  a.ld_q = ctx->nq;
+  a.kc = static_cast<char*>(ctx->kcache) + layer_kv_offset(ctx, l);
+  a.vc = static_cast<char*>(ctx->vcache) + layer_kv_offset(ctx, l);
+  a.max_len = ctx->max_len;
+  a.head_dim = ctx->hd;
+  a.n_kv_heads = ctx->Hkv;
+  a.rope = ctx->rope;
+  DVI_CUDA(launch_proj(a, mp ? &mp->qkv : nullptr, s));
+  // block-causal multi-query attention
+  AttnArgs t{};
+  t.q = ctx->q;
+  t.ld_q = ctx->nq;
+  t.kc = a.kc;
+  t.vc = a.vc;
+  t.o = ctx->attn_o;
+  t.ld_o = ctx->nq;
+  t.o_dtype = ctx->cfg.dtype;
+  t.dtype = ctx->cfg.dtype;
+  t.n_heads = ctx->Hq;
+  t.n_kv_heads = ctx->Hkv;
+  t.head_dim = ctx->hd;
+  t.max_len = ctx->max_len;
+  t.lens = ctx->lens;
+  t.rows_per_seq = ps.rows_per_seq;
+  t.seq0 = ps.seq0;
+  t.n_seqs = ps.n_seqs;
+  t.pos_off = ps.pos_off;
+  t.split_len = ctx->attn_split_len;
+  t.n_splits_max = ctx->attn_nsplits;
+  t.part = ctx->attn_part;
+  t.counters = ctx->attn_ctr;
+  t.status = ctx->status;
+  t.scale = 1.f / sqrtf(static_cast<float>(ctx->hd));
+  DVI_CUDA(launch_attn(t, s));
+  // x += W_o . attn
+  a = base_args(ctx, EPI_RESID, ctx->p_o, ps);
+  a.b_mode = B_COPY;
+  a.act = ctx->attn_o;
+  a.ld_act = ctx->nq;
+  a.K = ctx->nq;
+  a.n_out = ctx->d;
+  a.w0 = lw.wo;
+  a.x_res = ps.x;
+  a.ld_res = ctx->d;
+  a.ss_out = ps.ss;
+  a.ss_out_ld = ps.ss_ld;
+  DVI_CUDA(launch_proj(a, mp ? &mp->o : nullptr, s));
+  // h = SiLU(W_gate n) * (W_up n)
+  a = base_args(ctx, EPI_GATEUP, ctx->p_gu, ps);
+  a.b_mode = B_NORM;
+  a.x = ps.x;
+  a.ldx = ctx->d;
+  a.ss = ps.ss;
+  a.ss_ld = ps.ss_ld;
+  a.gain = static_cast<const float*>(lw.ffn_norm);
+  a.K = ctx->d;
+  a.n_out = ctx->F;
+  a.w0 = lw.w_gate;
+  a.w1 = lw.w_up;
+  a.h_out = ctx->ffn_h;
+  a.ld_h = ctx->F;
+  DVI_CUDA(launch_proj(a, mp ? &mp->gu : nullptr, s));
+  // x += W_down . h
+  a = base_args(ctx, EPI_RESID, ctx->p_down, ps);
+  a.b_mode = B_COPY;
+  a.act = ctx->ffn_h;
+  a.ld_act = ctx->F;
+  a.K = ctx->F;
+  a.n_out = ctx->d;
+  a.w0 = lw.w_down;
+  a.x_res = ps.x;
+  a.ld_res = ctx->d;
+  a.ss_out = ps.ss;
+  a.ss_out_ld = ps.ss_ld;
+  DVI_CUDA(launch_proj(a, mp ? &mp->down : nullptr, s));
+  ctx->launches += 5;
+  return DVI_OK;
+}
+
+dvi_status enqueue_layers(dvi_ctx* ctx, int lo, int hi, const Pass& ps) {
+  for (int l = lo; l < hi; ++l) {
+    dvi_status st = enqueue_layer(ctx, l, ps);
+    if (st != DVI_OK) return st;
+  }
+  return DVI_OK;
+}
+
+StepState step_state(dvi_ctx* c) {
+  StepState st{};
+  st.B = c->B;
+  st.K = c->K;
+  st.d = c->d;
+  st.vocab = c->V;
+  st.max_len = c->max_len;
+  st.dtype = c->cfg.dtype;
+  st.lens = c->lens;
+  st.pending = c->pending;
+  st.draft_ids = c->draft_ids;
+  st.x_dr = c->x_dr;
+  st.ss_dr = c->ss_dr;
+  st.ss_dr_ld = c->B;
+  st.embed = c->w.embed;
+  st.amax = c->amax;
+  st.out_ids = c->out_ids;
+  st.n_committed = c->n_committed;
+  st.n_accepted = c->n_accepted;
+  st.log_meta = c->log_meta;
+  st.log_step = c->log_step;
+  st.log_cap_steps = c->cap_steps;
+  st.log_enabled = c->log_enabled;
+  st.counters = c->counters;
+  st.status = c->status;
+  return st;
+}
+
+HeadPrepArgs head_prep_args(dvi_ctx* c, const float* x, int rows) {
+  HeadPrepArgs h{};
+  h.x = x;
+  h.ldx = c->d;
+  h.gain = static_cast<const float*>(c->w.final_norm);
+  h.eps = c->cfg.rms_eps;
+  h.d = c->d;
+  h.dtype = c->cfg.dtype;
+  h.u_out = c->u_buf;
+  h.ld_u = c->d;
+  h.rows = rows;
+  return h;
+}
+
+// Head projection over `rows` rows of u_buf; W^S (+LoRA) when `draft`.
+dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode) {
+  Pass ps{nullptr, nullptr, 0, rows, 1, 0, 1, 0};
+  ProjArgs a = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
+  a.b_mode = B_COPY;
+  a.act = ctx->u_buf;
+  a.ld_act = ctx->d;
+  a.K = ctx->d;
+  a.n_out = ctx->V;
+  a.w0 = draft ? ctx->w.draft_head : ctx->w.lm_head;
+  a.amax = ctx->amax;
+  if (draft && ctx->r > 0) {
+    a.lora_a = ctx->w.lora_a;
+    a.lora_bu = ctx->bu;
+    a.lora_r = ctx->r;
+    a.gamma = ctx->cfg.lora_gamma;
+  }
+  if (logits_mode == 2) {
+    a.logits_mode = 2;
+    a.logits_out = ctx->log_logits;
+    a.ld_logits = ctx->V;
+    a.log_step = ctx->log_step;
+    a.log_cap_steps = ctx->cap_steps;
+    a.log_rows_per_step = ctx->B * ctx->K;
+  }
+  DVI_CUDA(launch_proj(a, ctx->tc ? (draft ? &ctx->head_s : &ctx->head_v) : nullptr, ctx->stream));
+  ctx->launches += 1;
+  return DVI_OK;
+}
+
+dvi_status enqueue_step(dvi_ctx* ctx) {
+  cudaStream_t s = ctx->stream;
+  const StepState st = step_state(ctx);
+  dvi_status rc;
+  for (int j = 0; j < ctx->K; ++j) {
+    Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, j};
+    if ((rc = enqueue_layers(ctx, 0, ctx->k, ps)) != DVI_OK) return rc;
+    HeadPrepArgs h = head_prep_args(ctx, ctx->x_dr, ctx->B);
+    h.x_copy = ctx->x_ver;
+    h.ld_copy = ctx->d;
+    h.copy_row_stride = ctx->K;
+    h.copy_row_off = j;
+    h.ss_copy = ctx->ss_ver;
+    h.ss_copy_ld = ctx->B * ctx->K;
+    h.log_u = ctx->log_u;
+    h.log_step = ctx->log_step;
+    h.log_cap_steps = ctx->cap_steps;
+    h.log_rows_per_step = ctx->B * ctx->K;
+    h.log_row_stride = ctx->K;
+    h.log_row_off = j;
+    h.log_enabled = ctx->log_enabled;
+    if (ctx->r > 0) {
+      h.lora_b = ctx->w.lora_b;
+      h.bu = ctx->bu;
+      h.r = ctx->r;
+    }
+    DVI_CUDA(launch_head_prep(h, s));
+    if ((rc = enqueue_head(ctx, true, ctx->B, 0)) != DVI_OK) return rc;
+    DVI_CUDA(launch_finalize_draft(st, j, s));
+    ctx->launches += 2;
+  }
+  Pass pv{ctx->x_ver, ctx->ss_ver, ctx->B * ctx->K, ctx->B * ctx->K, ctx->K, 0, ctx->B, 0};
+  if ((rc = enqueue_layers(ctx, ctx->k, ctx->L, pv)) != DVI_OK) return rc;
+  HeadPrepArgs h = head_prep_args(ctx, ctx->x_ver, ctx->B * ctx->K);
+  DVI_CUDA(launch_head_prep(h, s));
+  if ((rc = enqueue_head(ctx, false, ctx->B * ctx->K, ctx->log_enabled ? 2 : 0)) != DVI_OK) return rc;
+  DVI_CUDA(launch_finalize_verify(st, s));
+  ctx->launches += 2;
+  return DVI_OK;
+}
+
+void fill_rope_host(int max_len, int hd, float theta, std::vector<float2>& out) {
+  const int half = hd / 2;
+  out.resize(static_cast<size_t>(max_len) * half);
+  for (int p = 0; p < max_len; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double inv = std::pow(static_cast<double>(theta), -2.0 * i / hd);
+      const double ang = static_cast<double>(p) * inv;
+      out[static_cast<size_t>(p) * half + i] = make_float2(static_cast<float>(std::cos(ang)),
+                                                           static_cast<float>(std::sin(ang)));
+    }
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" {
+
+size_t dvi_workspace_bytes(const dvi_model_config* cfg, const dvi_runtime_config* rt) {
+  if (!valid_config(cfg, rt, nullptr)) return 0;
+  dvi_ctx c;
+  init_dims(&c, cfg, rt);
+  return layout(&c, nullptr);
+}
+
+dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt, const dvi_weights* weights,
+                      void* workspace, size_t workspace_bytes, dvi_stream stream, dvi_ctx** out) {
+  if (!out) return DVI_ERR_INVALID_ARG;
+  *out = nullptr;
+  std::string why;
+  if (!valid_config(cfg, rt, &why)) {
+    fprintf(stderr, "dvi_create: %s\n", why.c_str());
+    return DVI_ERR_INVALID_ARG;
+  }
+  if (!weights || !weights->layers || !weights->embed || !weights->final_norm || !weights->lm_head ||
+      !weights->draft_head || !workspace)
+    return DVI_ERR_INVALID_ARG;
+  if (cfg->lora_rank > 0 && (!weights->lora_a || !weights->lora_b)) return DVI_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return DVI_ERR_INVALID_ARG;
+  dvi_ctx* ctx = new dvi_ctx();
+  init_dims(ctx, cfg, rt);
+  ctx->ws_bytes = layout(ctx, nullptr);
+  if (workspace_bytes < ctx->ws_bytes) {
+    delete ctx;
+    return DVI_ERR_CAPACITY;
+  }
+  ctx->ws = workspace;
+  layout(ctx, static_cast<char*>(workspace));
+  ctx->w = *weights;
+  ctx->layers.assign(weights->layers, weights->layers + cfg->n_layers);
+  ctx->w.layers = ctx->layers.data();
+  ctx->stream = reinterpret_cast<cudaStream_t>(stream);
+  if (ctx->tc) {
+    auto mk = [&](CUtensorMap* m, const void* p, int rows, int cols) {
+      return aligned16(p) && make_weight_map(m, p, rows, cols);
+    };
+    bool ok = true;
+    ctx->maps.resize(ctx->L);
+    for (int l = 0; l < ctx->L && ok; ++l) {
+      const dvi_layer_weights& lw = ctx->layers[l];
+      LayerMaps& m = ctx->maps[l];
+      ok = mk(&m.qkv.m0, lw.wq, ctx->nq, ctx->d) && mk(&m.qkv.m1, lw.wk, ctx->nkv, ctx->d) &&
+           mk(&m.qkv.m2, lw.wv, ctx->nkv, ctx->d) && mk(&m.o.m0, lw.wo, ctx->d, ctx->nq) &&
+           mk(&m.gu.m0, lw.w_gate, ctx->F, ctx->d) && mk(&m.gu.m1, lw.w_up, ctx->F, ctx->d) &&
+           mk(&m.down.m0, lw.w_down, ctx->d, ctx->F);
+    }
+    ok = ok && mk(&ctx->head_v.m0, weights->lm_head, ctx->V, ctx->d) &&
+         mk(&ctx->head_s.m0, weights->draft_head, ctx->V, ctx->d);
+    if (!ok) {
+      fprintf(stderr, "dvi_create: TMA descriptor creation failed (weights must be 16-byte aligned)\n");
+      delete ctx;
+      return DVI_ERR_INVALID_ARG;
+    }
+  }
+  std::vector<float2> rope;
+  fill_rope_host(ctx->max_len, ctx->hd, cfg->rope_theta, rope);
+  if (cudaMemsetAsync(workspace, 0, ctx->ws_bytes, ctx->stream) != cudaSuccess ||
+      cudaMemcpyAsync(ctx->rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice, ctx->stream) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(ctx->stream) != cudaSuccess) {
+    delete ctx;
+    return DVI_ERR_CUDA;
+  }
+  *out = ctx;
+  return DVI_OK;
+}
+
+dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tokens, int32_t* d_first_token) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  if (seq < 0 || seq >= ctx->B || !d_tokens || n_tokens < 1)
+    return fail(ctx, DVI_ERR_INVALID_ARG, "prefill: bad sequence, tokens or length");
+  if (n_tokens + ctx->K + 1 > ctx->max_len) return fail(ctx, DVI_ERR_CAPACITY, "prefill: prompt exceeds max_seq_len");
+  cudaStream_t s = ctx->stream;
+  const StepState st = step_state(ctx);
+  DVI_CUDA(launch_reset_seq(st, seq, s));
+  ctx->launches += 1;
+  int last_rows = 0;
+  for (int c0 = 0; c0 < n_tokens; c0 += ctx->chunk) {
+    const int rows = std::min(ctx->chunk, n_tokens - c0);
+    EmbedArgs e{};
+    e.table = ctx->w.embed;
+    e.dtype = ctx->cfg.dtype;
+    e.d = ctx->d;
+    e.vocab = ctx->V;
+    e.tokens = d_tokens + c0;
+    e.x = ctx->x_pf;
+    e.ldx = ctx->d;
+    e.ss = ctx->ss_pf;
+    e.ss_ld = ctx->chunk;
+    e.rows = rows;
+    e.status = ctx->status;
+    DVI_CUDA(launch_embed(e, s));
+    ctx->launches += 1;
+    Pass ps{ctx->x_pf, ctx->ss_pf, ctx->chunk, rows, rows, seq, 1, c0};
+    dvi_status rc = enqueue_layers(ctx, 0, ctx->L, ps);
+    if (rc != DVI_OK) return rc;
+    last_rows = rows;
+  }
+  HeadPrepArgs h = head_prep_args(ctx, ctx->x_pf + static_cast<size_t>(last_rows - 1) * ctx->d, 1);
+  DVI_CUDA(launch_head_prep(h, s));
+  dvi_status rc = enqueue_head(ctx, false, 1, 0);
+  if (rc != DVI_OK) return rc;
+  DVI_CUDA(launch_finalize_prefill(st, seq, n_tokens, d_first_token, s));
+  ctx->launches += 2;
+  return DVI_OK;
+}
+
+dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids, int32_t* d_n_committed,
+                                   int32_t* d_n_accepted) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  cudaStream_t s = ctx->stream;
+  ctx->step_calls += 1;
+  if (ctx->rt.use_graphs && ctx->step_calls > 1) {
+    if (!ctx->step_exec) {
+      const long long before = ctx->launches;
+      cudaGraph_t g = nullptr;
+      DVI_CUDA(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
+      dvi_status rc = enqueue_step(ctx);
+      cudaError_t ce = cudaStreamEndCapture(s, &g);
+      if (rc != DVI_OK) return rc;
+      if (ce != cudaSuccess) return fail(ctx, DVI_ERR_CUDA, cudaGetErrorString(ce));
+      ce = cudaGraphInstantiate(&ctx->step_exec, g, 0);
+      cudaGraphDestroy(g);
+      if (ce != cudaSuccess) {
+        ctx->step_exec = nullptr;
+        return fail(ctx, DVI_ERR_CUDA, cudaGetErrorString(ce));
+      }
+      ctx->step_launches = ctx->launches - before;
+      ctx->launches = before;
+    }
+    DVI_CUDA(cudaGraphLaunch(ctx->step_exec, s));
+    ctx->launches += ctx->step_launches;
+  } else {
+    dvi_status rc = enqueue_step(ctx);
+    if (rc != DVI_OK) return rc;
+  }
+  if (d_out_ids)
+    DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->out_ids, sizeof(int) * ctx->B * ctx->K, cudaMemcpyDeviceToDevice, s));
+  if (d_n_committed)
+    DVI_CUDA(cudaMemcpyAsync(d_n_committed, ctx->n_committed, sizeof(int) * ctx->B, cudaMemcpyDeviceToDevice, s));
+  if (d_n_accepted)
+    DVI_CUDA(cudaMemcpyAsync(d_n_accepted, ctx->n_accepted, sizeof(int) * ctx->B, cudaMemcpyDeviceToDevice, s));
+  return DVI_OK;
+}
+
+dvi_status dvi_log(dvi_ctx* ctx, int enable) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  const int e = enable ? 1 : 0;
+  if (e != ctx->log_enabled && ctx->step_exec) {
+    cudaGraphExecDestroy(ctx->step_exec);
+    ctx->step_exec = nullptr;
+  }
+  ctx->log_enabled = e;
+  return DVI_OK;
+}
+
+dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
+  if (!ctx || !u) return DVI_ERR_INVALID_ARG;
+  if (!(u->tau > 0.f) || u->t_ramp < 0 || u->t_warmup < 0 || u->objective < 0 || u->objective > 3 ||
+      u->optimizer < 0 || u->optimizer > 1 || !(u->t_beta > 0.f))
+    return fail(ctx, DVI_ERR_INVALID_ARG, "update: bad hyper-parameters");
+  if (ctx->r == 0) return fail(ctx, DVI_ERR_UNIMPLEMENTED, "update: no LoRA factors (lora_rank 0)");
+  cudaStream_t s = ctx->stream;
+  UpdateArgs a{};
+  a.cap = ctx->cap_rows;
+  a.V = ctx->V;
+  a.d = ctx->d;
+  a.r = ctx->r;
+  a.dtype = ctx->cfg.dtype;
+  a.B = ctx->B;
+  a.K = ctx->K;
+  a.log_u = ctx->log_u;
+  a.log_logits = ctx->log_logits;
+  a.log_meta = ctx->log_meta;
+  a.log_step = ctx->log_step;
+  a.Z = ctx->Z;
+  a.rowstat = ctx->rowstat;
+  a.coef = ctx->coef;
+  a.ub = ctx->ub;
+  a.ga = ctx->ga;
+  a.ga_part = ctx->ga_part;
+  a.n_vtiles = (ctx->V + 127) / 128;
+  a.lora_a = ctx->w.lora_a;
+  a.lora_b = ctx->w.lora_b;
+  a.gamma = ctx->cfg.lora_gamma;
+  a.m_a = ctx->m_a;
+  a.v_a = ctx->v_a;
+  a.m_b = ctx->m_b;
+  a.v_b = ctx->v_b;
+  a.grad_a = ctx->grad_a;
+  a.grad_b = ctx->grad_b;
+  a.dev_state = ctx->dev_state;
+  a.counters = ctx->counters;
+  a.status = ctx->status;
+  a.cfg = *u;
+  DVI_CUDA(launch_update_prep(a, s));
+  // drafter logits of every buffer row: Z = U W^S^T + gamma (U B^T) A^T
+  Pass ps{nullptr, nullptr, 0, ctx->cap_rows, 1, 0, 1, 0};
+  ProjArgs p = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
+  p.b_mode = B_COPY;
+  p.act = ctx->log_u;
+  p.ld_act = ctx->d;
+  p.K = ctx->d;
+  p.n_out = ctx->V;
+  p.w0 = ctx->w.draft_head;
+  p.logits_mode = 1;
+  p.logits_out = ctx->Z;
+  p.ld_logits = ctx->V;
+  p.lora_a = ctx->w.lora_a;
+  p.lora_bu = ctx->ub;
+  p.lora_r = ctx->r;
+  p.gamma = ctx->cfg.lora_gamma;
+  DVI_CUDA(launch_proj(p, ctx->tc ? &ctx->head_s : nullptr, s));
+  DVI_CUDA(launch_update_rowstats(a, s));
+  DVI_CUDA(launch_update_coef(a, s));
+  DVI_CUDA(launch_update_grad_a(a, s));
+  DVI_CUDA(launch_update_grad_b(a, s));
+  DVI_CUDA(launch_update_finish(a, s));
+  ctx->launches += 8;
+  return DVI_OK;
+}
+
+dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  cudaStream_t s = ctx->stream;
+  StepState st = step_state(ctx);
+  st.out_ids = ctx->ar_out;
+  Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0};
+  dvi_status rc = enqueue_layers(ctx, 0, ctx->L, ps);
+  if (rc != DVI_OK) return rc;
+  HeadPrepArgs h = head_prep_args(ctx, ctx->x_dr, ctx->B);
+  DVI_CUDA(launch_head_prep(h, s));
+  if ((rc = enqueue_head(ctx, false, ctx->B, 0)) != DVI_OK) return rc;
+  DVI_CUDA(launch_finalize_ar(st, s));
+  ctx->launches += 2;
+  if (d_out_ids) DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->ar_out, sizeof(int) * ctx->B, cudaMemcpyDeviceToDevice, s));
+  return DVI_OK;
+}
+
+dvi_status dvi_get_stats(dvi_ctx* ctx, dvi_stats* out) {
+  if (!ctx || !out) return DVI_ERR_INVALID_ARG;
+  DVI_CUDA(cudaStreamSynchronize(ctx->stream));
+  long long c[8];
+  float ds[16];
+  int status = 0;
+  DVI_CUDA(cudaMemcpy(c, ctx->counters, sizeof(c), cudaMemcpyDeviceToHost));
+  DVI_CUDA(cudaMemcpy(ds, ctx->dev_state, sizeof(ds), cudaMemcpyDeviceToHost));
+  DVI_CUDA(cudaMemcpy(&status, ctx->status, sizeof(int), cudaMemcpyDeviceToHost));
+  memset(out, 0, sizeof(*out));
+  out->steps = c[0];
+  out->drafted = c[1];
+  out->accepted = c[2];
+  out->committed = c[3];
+  out->updates = c[4];
+  out->kernel_launches = ctx->launches;
+  out->update_t = static_cast<int>(ds[0]);
+  out->baseline_b = ds[1];
+  out->last_loss = ds[2];
+  out->last_kl = ds[3];
+  out->last_pg = ds[4];
+  out->last_ce = ds[5];
+  out->last_ent = ds[6];
+  out->last_rl = ds[7];
+  out->last_kl1 = ds[8];
+  out->last_accept_rate = ds[9];
+  out->device_status = status;
+  return DVI_OK;
+}
+
+const char* dvi_last_error(const dvi_ctx* ctx) { return ctx ? ctx->err.c_str() : "null context"; }
+
+dvi_status dvi_destroy(dvi_ctx* ctx) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  if (ctx->step_exec) cudaGraphExecDestroy(ctx->step_exec);
+  delete ctx;
+  return DVI_OK;
+}
+
+dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes) {
+  if (!ctx || !dptr || !bytes) return DVI_ERR_INVALID_ARG;
+  const size_t e = ctx->esz;
+  const size_t kv = static_cast<size_t>(ctx->L) * ctx->B * ctx->Hkv * ctx->max_len * ctx->hd * e;
+  const int rr = ctx->r > 0 ? ctx->r : 1;
+  switch (which) {
+    case DVI_BUF_LENS: *dptr = ctx->lens; *bytes = sizeof(int) * ctx->B; break;
+    case DVI_BUF_PENDING: *dptr = ctx->pending; *bytes = sizeof(int) * ctx->B; break;
+    case DVI_BUF_DRAFT_IDS: *dptr = ctx->draft_ids; *bytes = sizeof(int) * ctx->B * (ctx->K + 1); break;
+    case DVI_BUF_LOG_U: *dptr = ctx->log_u; *bytes = e * ctx->cap_rows * ctx->d; break;
+    case DVI_BUF_LOG_LOGITS: *dptr = ctx->log_logits; *bytes = sizeof(float) * ctx->cap_rows * static_cast<size_t>(ctx->V); break;
+    case DVI_BUF_LOG_META: *dptr = ctx->log_meta; *bytes = sizeof(int) * 6 * ctx->cap_rows; break;
+    case DVI_BUF_GRAD_A: *dptr = ctx->grad_a; *bytes = sizeof(float) * static_cast<size_t>(ctx->V) * rr; break;
+    case DVI_BUF_GRAD_B: *dptr = ctx->grad_b; *bytes = sizeof(float) * static_cast<size_t>(rr) * ctx->d; break;
+    case DVI_BUF_X_DRAFT: *dptr = ctx->x_dr; *bytes = sizeof(float) * ctx->B * ctx->d; break;
+    case DVI_BUF_X_VERIFY: *dptr = ctx->x_ver; *bytes = sizeof(float) * ctx->B * ctx->K * ctx->d; break;
+    case DVI_BUF_K_CACHE: *dptr = ctx->kcache; *bytes = kv; break;
+    case DVI_BUF_V_CACHE: *dptr = ctx->vcache; *bytes = kv; break;
+    case DVI_BUF_STATUS: *dptr = ctx->status; *bytes = sizeof(int); break;
+    case DVI_BUF_Z: *dptr = ctx->Z; *bytes = sizeof(float) * ctx->cap_rows * static_cast<size_t>(ctx->V); break;
+    default: return fail(ctx, DVI_ERR_INVALID_ARG, "debug_buffer: unknown buffer");
+  }
+  return DVI_OK;
+}
+
+dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in, const float* d_x, int m_rows,
+                      float* d_y) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  if (!d_w || !d_x || !d_y || n_out < 1 || k_in < 1 || m_rows < 1 || m_rows > kMaxTokens)
+    return fail(ctx, DVI_ERR_INVALID_ARG, "linear: bad arguments");
+  if (ctx->tc && (k_in % 8 || !aligned16(d_w) || !aligned16(d_x)))
+    return fail(ctx, DVI_ERR_INVALID_ARG, "linear: bf16 needs k_in % 8 == 0 and 16-byte aligned pointers");
+  Plan pl = plan_for(ctx, EPI_HEAD, n_out, k_in, 0, 0, 0);
+  Pass ps{nullptr, nullptr, 0, m_rows, 1, 0, 1, 0};
+  ProjArgs a = base_args(ctx, EPI_HEAD, pl, ps);
+  a.b_mode = B_COPY_F32;
+  a.act = d_x;
+  a.ld_act = k_in;
+  a.K = k_in;
+  a.n_out = n_out;
+  a.w0 = d_w;
+  a.logits_mode = 1;
+  a.logits_out = d_y;
+  a.ld_logits = n_out;
+  const int ntt = ctx->tc ? 1 : (m_rows + kChunk - 1) / kChunk;
+  if (proj_partial_floats(a, ctx->tc) > ctx->part_floats || a.n_tiles * ntt > ctx->n_proj_counters)
+    return fail(ctx, DVI_ERR_CAPACITY, "linear: shape needs more split-K scratch than the workspace has");
+  ProjMaps m{};
+  if (ctx->tc && !make_weight_map(&m.m0, d_w, n_out, k_in))
+    return fail(ctx, DVI_ERR_INVALID_ARG, "linear: TMA descriptor creation failed");
+  DVI_CUDA(launch_proj(a, ctx->tc ? &m : nullptr, ctx->stream));
+  ctx->launches += 1;
+  return DVI_OK;
+}
+
+}  // extern "C"

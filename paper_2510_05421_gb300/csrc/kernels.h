@@ -1,0 +1,165 @@
+// Internal interface between the C-ABI layer (dvi_api.cu) and the kernel
+// translation units.  Host-side launchers only; no torch types anywhere.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/dvi.h"
+
+namespace dvi {
+
+enum Flavor : int {
+  EPI_QKV = 0,     // RoPE on q/k, q -> q_out (f32), k/v -> KV cache rows
+  EPI_RESID = 1,   // x += W.act, plus per-tile sums of squares for the next RMSNorm
+  EPI_GATEUP = 2,  // h = SiLU(W_gate.n) * (W_up.n), two accumulators per tile
+  EPI_HEAD = 3     // vocabulary logits (+ gamma A (B u)), stored and/or argmax
+};
+
+enum BMode : int {
+  B_NORM = 0,      // B[n][k] = x[n][k] * rstd[n] * gain[k], rstd from sum-of-squares partials
+  B_COPY = 1,      // B[n][k] = act[n][k] in the model dtype
+  B_COPY_F32 = 2   // B[n][k] = act[n][k] given as float32
+};
+
+struct ProjArgs {
+  int flavor, b_mode, dtype;
+  int M;              // token rows
+  int n_pad;          // tcgen05 N: multiple of 16, >= M
+  int n_out;          // rows of one weight (GATEUP: F); QKV uses rows_q/k/v
+  int K;              // input features
+  int n_tiles, n_splits, kb_total, kb_per_split, n_ttiles;
+  const void* w0;     // f32 path: weight pointers (QKV: wq, wk, wv; GATEUP: gate, up)
+  const void* w1;
+  const void* w2;
+  int rows_q, rows_k, rows_v;
+  // B source
+  const float* x; int ldx;
+  const float* ss; int ss_ld; int ss_tiles;
+  const float* gain; float eps; int d_norm;
+  const void* act; int ld_act;
+  // token row -> (sequence, position)
+  const int* lens; int rows_per_seq; int seq0; int pos_off;
+  // split-K scratch: partial tiles and arrival counters (counters start at 0
+  // and are reset to 0 by the CTA that reduces a tile)
+  float* part; int* counters;
+  int* status;
+  // EPI_QKV
+  float* q_out; int ld_q;
+  void* kc; void* vc; int max_len; int head_dim;
+  int n_kv_heads;
+  const float2* rope;
+  // EPI_RESID
+  float* x_res; int ld_res; float* ss_out; int ss_out_ld;
+  // EPI_GATEUP
+  void* h_out; int ld_h;
+  // EPI_HEAD
+  float* logits_out; int ld_logits;
+  int logits_mode;            // 0 none, 1 row n -> logits_out[n], 2 replay-buffer slot
+  const int* log_step; int log_cap_steps; int log_rows_per_step;
+  const float* lora_a; const float* lora_bu; int lora_r; float gamma;
+  unsigned long long* amax;   // [M] argmax keys, or null
+};
+
+struct ProjMaps {
+  CUtensorMap m0, m1, m2;     // bf16 path: TMA descriptors of w0, w1, w2
+};
+
+// Picks n_splits / kb_per_split from the weight shape only (never from M),
+// so a row's result does not depend on how many rows share the launch.
+void plan_splits(ProjArgs& a, int n_sms, bool tc);
+size_t proj_partial_floats(const ProjArgs& a, bool tc);
+cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s);
+bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
+
+struct AttnArgs {
+  const float* q; int ld_q;          // rotated queries [M][H_q*hd]
+  const void* kc; const void* vc;    // layer base of the caches [B][H_kv][max_len][hd]
+  void* o; int ld_o;                 // output [M][H_q*hd] in `o_dtype`
+  int o_dtype;
+  int dtype;                         // cache dtype
+  int n_heads, n_kv_heads, head_dim, max_len;
+  const int* lens; int rows_per_seq; int seq0; int n_seqs; int pos_off;
+  int split_len;                     // positions per split (multiple of 64)
+  int n_splits_max;
+  float* part; int* counters;        // combine scratch
+  int* status;
+  float scale;
+};
+size_t attn_partial_floats(const AttnArgs& a);
+int attn_counters(const AttnArgs& a);
+cudaError_t launch_attn(const AttnArgs& a, cudaStream_t s);
+
+// ---- small kernels (misc.cu)
+struct EmbedArgs {
+  const void* table; int dtype; int d; int vocab;
+  const int* tokens;                 // device ids, or null -> use `tok_src` indirection
+  float* x; int ldx;                 // destination rows
+  float* ss; int ss_ld;              // per-128-feature sums of squares
+  int rows;
+  int* status;
+};
+cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s);
+
+struct HeadPrepArgs {
+  const float* x; int ldx;           // rows to normalise
+  const float* gain; float eps; int d;
+  int dtype;
+  void* u_out; int ld_u;             // normalised rows in dtype (B operand of the head)
+  int rows;
+  // optional: copy x rows into another residual stream (+ its ss)
+  float* x_copy; int ld_copy; int copy_row_stride; int copy_row_off;
+  float* ss_copy; int ss_copy_ld;
+  // optional: log u into the replay buffer at slot (log_step*rows_per_step + row*K + j)
+  void* log_u; const int* log_step; int log_cap_steps; int log_rows_per_step; int log_row_stride;
+  int log_row_off; int log_enabled;
+  // optional LoRA down-projection: bu[row][j] = sum_c B[j][c] u[c]
+  const float* lora_b; float* bu; int r;
+};
+cudaError_t launch_head_prep(const HeadPrepArgs& a, cudaStream_t s);
+
+struct StepState {
+  int B, K, d, vocab, max_len, dtype;
+  int* lens; int* pending; int* draft_ids;      // [B][K+1]
+  float* x_dr; float* ss_dr; int ss_dr_ld;
+  const void* embed;
+  unsigned long long* amax;
+  int* out_ids; int* n_committed; int* n_accepted;
+  int* log_meta; int* log_step; int log_cap_steps; int log_enabled;
+  long long* counters;                          // steps, drafted, accepted, committed
+  int* status;
+};
+cudaError_t launch_finalize_draft(const StepState& st, int j, cudaStream_t s);
+cudaError_t launch_finalize_verify(const StepState& st, cudaStream_t s);
+cudaError_t launch_finalize_ar(const StepState& st, cudaStream_t s);
+cudaError_t launch_finalize_prefill(const StepState& st, int seq, int n_tokens, int32_t* first_out,
+                                    cudaStream_t s);
+cudaError_t launch_reset_seq(const StepState& st, int seq, cudaStream_t s);
+
+// ---- drafter update (update.cu)
+struct UpdateArgs {
+  int cap, V, d, r, dtype, B, K;
+  const void* log_u; const float* log_logits; int* log_meta; int* log_step;
+  float* Z;                                     // [cap][V] drafter logits
+  float* rowstat;                               // [cap][8]
+  float* coef;                                  // [cap][4] + globals
+  float* ub;                                    // [cap][r]  U B^T
+  float* ga;                                    // [cap][r]  G A
+  float* ga_part; int* ga_counter; int n_vtiles;
+  float* lora_a; float* lora_b; float gamma;
+  float* m_a; float* v_a; float* m_b; float* v_b;
+  float* grad_a; float* grad_b;
+  float* dev_state;                             // [0]=t, [1]=b, [2..] loss parts
+  long long* counters;
+  int* status;
+  dvi_update_config cfg;
+};
+cudaError_t launch_update_prep(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_update_rowstats(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_update_coef(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_update_finish(const UpdateArgs& a, cudaStream_t s);
+
+}  // namespace dvi

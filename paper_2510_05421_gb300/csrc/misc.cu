@@ -1,0 +1,268 @@
+// Small kernels around the projections: embedding rows, head preparation
+// (final RMSNorm, LoRA down-projection B u, logging u, handing h_k to the
+// verify stream), and the single-CTA finalize kernels that turn argmax keys
+// into drafted / committed tokens.
+//
+// finalize_verify is the accept/commit/rollback step of Sec. 3.3: with
+// y*_{n+i} the verifier's argmax at block row i-1 and t~_i the drafts,
+// m = max{i <= K : t~_j = y*_{n+j} for all j <= i}; the step commits
+// t~_1..t~_m and, when m < K, the correction y*_{n+m+1} -- min(m+1, K)
+// tokens -- and the cache length advances by the same count, which discards
+// the KV rows of rejected drafts (they are overwritten later; no data moves).
+// The replay-buffer tuples of rows 1..min(m+1, K) get r = 1 up to m and r = 0
+// at the first reject (Sec. 3.3); later rows stay invalid (counterfactual).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace dvi {
+
+template <typename T>
+__device__ void embed_row_block(const T* table, int tok, int d, float* x, float* ss, int ss_ld, int row,
+                                float* red) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  for (int t = 0; t < d / kTileRows; ++t) {
+    const int c = t * kTileRows + tid;
+    const float v = DT<T>::ld(table + static_cast<size_t>(tok) * d + c);
+    x[c] = v;
+    const float s = warp_sum(v * v);
+    if (lane == 0) red[warp] = s;
+    __syncthreads();
+    if (tid == 0) ss[static_cast<size_t>(t) * ss_ld + row] = (red[0] + red[1]) + (red[2] + red[3]);
+    __syncthreads();
+  }
+}
+
+// ---------------------------------------------------------------- embed
+template <typename T>
+__global__ void __launch_bounds__(128) embed_kernel(const EmbedArgs a) {
+  __shared__ float red[4];
+  const int row = blockIdx.x;
+  int tok = a.tokens[row];
+  if (tok < 0 || tok >= a.vocab) {
+    if (threadIdx.x == 0) flag_status(a.status, DVI_DEV_BAD_TOKEN);
+    tok = 0;
+  }
+  embed_row_block<T>(static_cast<const T*>(a.table), tok, a.d, a.x + static_cast<size_t>(row) * a.ldx, a.ss,
+                     a.ss_ld, row, red);
+}
+
+cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s) {
+  if (a.dtype == DVI_BF16) embed_kernel<__nv_bfloat16><<<a.rows, 128, 0, s>>>(a);
+  else embed_kernel<float><<<a.rows, 128, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- head prep
+// grid (rows, ceil(r/4) or 1); block 128.  Every CTA recomputes the row's
+// RMSNorm; CTA y == 0 writes u, logs it and copies x; each CTA computes four
+// entries of B u (one warp each).
+template <typename T>
+__global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
+  __shared__ float red[4];
+  __shared__ float rstd_s;
+  const int row = blockIdx.x, grp = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const float* x = a.x + static_cast<size_t>(row) * a.ldx;
+  float s = 0.f;
+  for (int c = tid; c < a.d; c += 128) s = fmaf(x[c], x[c], s);
+  s = warp_sum(s);
+  if (lane == 0) red[warp] = s;
+  __syncthreads();
+  if (tid == 0) rstd_s = rsqrtf(((red[0] + red[1]) + (red[2] + red[3])) / static_cast<float>(a.d) + a.eps);
+  __syncthreads();
+  const float rstd = rstd_s;
+  if (grp == 0) {
+    T* u = static_cast<T*>(a.u_out) + static_cast<size_t>(row) * a.ld_u;
+    T* lu = nullptr;
+    if (a.log_u && a.log_enabled) {
+      const int ls = *a.log_step;
+      if (ls < a.log_cap_steps)
+        lu = static_cast<T*>(a.log_u) +
+             (static_cast<size_t>(ls) * a.log_rows_per_step + static_cast<size_t>(row) * a.log_row_stride +
+              a.log_row_off) * a.d;
+    }
+    for (int c = tid; c < a.d; c += 128) {
+      const float v = x[c] * rstd * a.gain[c];
+      DT<T>::st(u + c, v);
+      if (lu) DT<T>::st(lu + c, v);
+    }
+    if (a.x_copy) {
+      const int crow = row * a.copy_row_stride + a.copy_row_off;
+      float* xc = a.x_copy + static_cast<size_t>(crow) * a.ld_copy;
+      for (int t = 0; t < a.d / kTileRows; ++t) {
+        const float v = x[t * kTileRows + tid];
+        xc[t * kTileRows + tid] = v;
+        const float q = warp_sum(v * v);
+        __syncthreads();
+        if (lane == 0) red[warp] = q;
+        __syncthreads();
+        if (tid == 0) a.ss_copy[static_cast<size_t>(t) * a.ss_copy_ld + crow] = (red[0] + red[1]) + (red[2] + red[3]);
+      }
+    }
+  }
+  if (a.r > 0 && a.bu) {
+    const int j = grp * 4 + warp;
+    if (j < a.r) {
+      const float* br = a.lora_b + static_cast<size_t>(j) * a.d;
+      float acc = 0.f;
+      for (int c = lane; c < a.d; c += 32) acc = fmaf(br[c], x[c] * rstd * a.gain[c], acc);
+      acc = warp_sum(acc);
+      if (lane == 0) a.bu[static_cast<size_t>(row) * a.r + j] = acc;
+    }
+  }
+}
+
+cudaError_t launch_head_prep(const HeadPrepArgs& a, cudaStream_t s) {
+  dim3 grid(a.rows, (a.r > 0 && a.bu) ? (a.r + 3) / 4 : 1);
+  if (a.dtype == DVI_BF16) head_prep_kernel<__nv_bfloat16><<<grid, 128, 0, s>>>(a);
+  else head_prep_kernel<float><<<grid, 128, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- finalize
+__device__ __forceinline__ int take_argmax(unsigned long long* slot, int* status) {
+  const unsigned long long k = *slot;
+  *slot = 0ull;
+  if (k == 0ull) {
+    flag_status(status, DVI_DEV_NONFINITE);
+    return 0;
+  }
+  return argmax_idx(k);
+}
+
+template <typename T>
+__device__ void embed_rows(const StepState& st, const int* toks, float* red) {
+  for (int b = 0; b < st.B; ++b)
+    embed_row_block<T>(static_cast<const T*>(st.embed), toks[b], st.d, st.x_dr + static_cast<size_t>(b) * st.d,
+                       st.ss_dr, st.ss_dr_ld, b, red);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st, int j) {
+  __shared__ int tok_s[64];
+  __shared__ float red[4];
+  for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
+    const int t = take_argmax(st.amax + b, st.status);
+    st.draft_ids[b * (st.K + 1) + j + 1] = t;
+    tok_s[b] = t;
+  }
+  __syncthreads();
+  if (j + 1 < st.K) embed_rows<T>(st, tok_s, red);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) finalize_verify_kernel(const StepState st) {
+  __shared__ int tok_s[64];
+  __shared__ float red[4];
+  const int K = st.K;
+  const int ls = *st.log_step;
+  const bool log_ok = st.log_enabled && ls < st.log_cap_steps;
+  for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
+    int y[16];
+    for (int i = 0; i < K; ++i) y[i] = take_argmax(st.amax + b * K + i, st.status);
+    int* dr = st.draft_ids + b * (K + 1);
+    int m = 0;
+    while (m < K && dr[m + 1] == y[m]) ++m;
+    const int c = m < K ? m + 1 : K;
+    for (int i = 0; i < K; ++i) {
+      const int id = i < m ? dr[i + 1] : (i == m ? y[m] : -1);
+      st.out_ids[b * K + i] = id;
+    }
+    st.n_committed[b] = c;
+    st.n_accepted[b] = m;
+    if (log_ok) {
+      for (int i = 0; i < K; ++i) {
+        int* meta = st.log_meta + (static_cast<size_t>(ls) * st.B * K + b * K + i) * 6;
+        meta[0] = i < c;
+        meta[1] = dr[i + 1];
+        meta[2] = i < m ? 1 : 0;
+        meta[3] = i + 1;
+        meta[4] = dr[i];
+        meta[5] = y[i];
+      }
+    }
+    const int newtok = st.out_ids[b * K + c - 1];
+    st.lens[b] += c;
+    st.pending[b] = newtok;
+    dr[0] = newtok;
+    tok_s[b] = newtok;
+    atomicAdd(reinterpret_cast<unsigned long long*>(st.counters + 2), static_cast<unsigned long long>(m));
+    atomicAdd(reinterpret_cast<unsigned long long*>(st.counters + 3), static_cast<unsigned long long>(c));
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    st.counters[0] += 1;
+    st.counters[1] += static_cast<long long>(st.B) * K;
+    if (st.log_enabled) {
+      if (ls < st.log_cap_steps) *st.log_step = ls + 1;
+      else flag_status(st.status, DVI_DEV_LOG_FULL);
+    }
+  }
+  embed_rows<T>(st, tok_s, red);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) finalize_ar_kernel(const StepState st) {
+  __shared__ int tok_s[64];
+  __shared__ float red[4];
+  for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
+    const int y = take_argmax(st.amax + b, st.status);
+    st.out_ids[b] = y;
+    st.lens[b] += 1;
+    st.pending[b] = y;
+    st.draft_ids[b * (st.K + 1)] = y;
+    tok_s[b] = y;
+  }
+  __syncthreads();
+  embed_rows<T>(st, tok_s, red);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) finalize_prefill_kernel(const StepState st, int seq, int n_tokens,
+                                                               int32_t* first_out) {
+  __shared__ float red[4];
+  __shared__ int tok;
+  if (threadIdx.x == 0) {
+    const int y = take_argmax(st.amax, st.status);
+    st.lens[seq] = n_tokens;
+    st.pending[seq] = y;
+    st.draft_ids[seq * (st.K + 1)] = y;
+    if (first_out) *first_out = y;
+    tok = y;
+  }
+  __syncthreads();
+  embed_row_block<T>(static_cast<const T*>(st.embed), tok, st.d, st.x_dr + static_cast<size_t>(seq) * st.d,
+                     st.ss_dr, st.ss_dr_ld, seq, red);
+}
+
+__global__ void reset_seq_kernel(const StepState st, int seq) {
+  st.lens[seq] = 0;
+}
+
+cudaError_t launch_finalize_draft(const StepState& st, int j, cudaStream_t s) {
+  if (st.dtype == DVI_BF16) finalize_draft_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st, j);
+  else finalize_draft_kernel<float><<<1, 128, 0, s>>>(st, j);
+  return cudaGetLastError();
+}
+cudaError_t launch_finalize_verify(const StepState& st, cudaStream_t s) {
+  if (st.dtype == DVI_BF16) finalize_verify_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st);
+  else finalize_verify_kernel<float><<<1, 128, 0, s>>>(st);
+  return cudaGetLastError();
+}
+cudaError_t launch_finalize_ar(const StepState& st, cudaStream_t s) {
+  if (st.dtype == DVI_BF16) finalize_ar_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st);
+  else finalize_ar_kernel<float><<<1, 128, 0, s>>>(st);
+  return cudaGetLastError();
+}
+cudaError_t launch_finalize_prefill(const StepState& st, int seq, int n_tokens, int32_t* first_out,
+                                    cudaStream_t s) {
+  if (st.dtype == DVI_BF16) finalize_prefill_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st, seq, n_tokens, first_out);
+  else finalize_prefill_kernel<float><<<1, 128, 0, s>>>(st, seq, n_tokens, first_out);
+  return cudaGetLastError();
+}
+cudaError_t launch_reset_seq(const StepState& st, int seq, cudaStream_t s) {
+  reset_seq_kernel<<<1, 1, 0, s>>>(st, seq);
+  return cudaGetLastError();
+}
+
+}  // namespace dvi

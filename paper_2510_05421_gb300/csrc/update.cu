@@ -1,0 +1,354 @@
+// Drafter-head update (Sec. 3.4) on the replay buffer of Sec. 3.3.
+//
+// Rows are the buffer slots (step, sequence, block position); only rows with
+// the valid flag (positions up to and including the first reject) count.
+// With u = RMSNorm_final(h_k), l = logits^phi, p = softmax(z),
+// z = (W^S + gamma A B) u, q = softmax(l / tau), q1 = softmax(l):
+//
+//  update_prep      UB[n] = B u_n                               (LoRA down)
+//  (projection)     Z = U W^S^T + gamma UB A^T                  (EPI_HEAD)
+//  update_rowstats  per row: log-normalisers of z, l/tau, l; KL(p||q),
+//                   KL(p||q1), H[p], -log p(a), -log p(y*)
+//  update_coef      the schedule's term weights at update t, the means that
+//                   form the loss, per-row gradient coefficients; the EMA
+//                   baseline b moves after the loss is formed
+//  update_grad_a    per vocabulary entry v, dL/dz_{n,v} from the closed forms
+//                     KL:  p (log p - log q - KL)     CE to a: p - [v=a]
+//                     -H:  p (log p + H)
+//                   then dA[v] = gamma sum_n G[n][v] UB[n] and the optimizer
+//                   step on A[v]; partial sums of G A for dB (old A)
+//  update_ga_reduce GA[n] = sum over vocabulary tiles (fixed order)
+//  update_grad_b    dB[j][c] = gamma sum_n GA[n][j] u_n[c], optimizer step
+//  update_finish    t += 1, empty the buffer
+#include <cmath>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace dvi {
+
+constexpr int kMaxRank = 64;
+
+enum { RS_LSEZ = 0, RS_LSEQ, RS_LSEQ1, RS_KL, RS_KL1, RS_ENT, RS_NLLA, RS_NLLY, RS_N };
+enum { CF_KL = 0, CF_KL1, CF_ENT, CF_A, CF_Y, CF_N };
+// dev_state floats: 0 t, 1 b, 2 loss, 3 kl, 4 pg, 5 ce, 6 ent, 7 rl, 8 kl1, 9 accept rate,
+// 10 skip flag, 11 adam steps
+enum { DS_T = 0, DS_B, DS_LOSS, DS_KL, DS_PG, DS_CE, DS_ENT, DS_RL, DS_KL1, DS_ACC, DS_SKIP, DS_ADAM };
+
+__device__ __forceinline__ bool row_valid(const UpdateArgs& a, int n) { return a.log_meta[n * 6] != 0; }
+
+template <typename T>
+__global__ void __launch_bounds__(128) update_prep_kernel(const UpdateArgs a) {
+  const int n = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (!row_valid(a, n)) {
+    for (int j = threadIdx.x; j < a.r; j += 128) a.ub[n * a.r + j] = 0.f;
+    return;
+  }
+  const T* u = static_cast<const T*>(a.log_u) + static_cast<size_t>(n) * a.d;
+  for (int j = warp; j < a.r; j += 4) {
+    const float* br = a.lora_b + static_cast<size_t>(j) * a.d;
+    float acc = 0.f;
+    for (int c = lane; c < a.d; c += 32) acc = fmaf(br[c], DT<T>::ld(u + c), acc);
+    acc = warp_sum(acc);
+    if (lane == 0) a.ub[n * a.r + j] = acc;
+  }
+}
+
+__device__ float block_reduce(float v, float* red, bool is_max) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  v = is_max ? warp_max(v) : warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float r = red[0];
+  for (int w = 1; w < nw; ++w) r = is_max ? fmaxf(r, red[w]) : r + red[w];
+  return r;
+}
+
+__global__ void __launch_bounds__(256) update_rowstats_kernel(const UpdateArgs a) {
+  __shared__ float red[8];
+  const int n = blockIdx.x;
+  float* rs = a.rowstat + n * RS_N;
+  if (!row_valid(a, n)) {
+    if (threadIdx.x < RS_N) rs[threadIdx.x] = 0.f;
+    return;
+  }
+  const float* z = a.Z + static_cast<size_t>(n) * a.V;
+  const float* l = a.log_logits + static_cast<size_t>(n) * a.V;
+  const float it = 1.f / a.cfg.tau;
+  float mz = -INFINITY, mq = -INFINITY, mq1 = -INFINITY;
+  for (int v = threadIdx.x; v < a.V; v += blockDim.x) {
+    mz = fmaxf(mz, z[v]);
+    mq = fmaxf(mq, l[v] * it);
+    mq1 = fmaxf(mq1, l[v]);
+  }
+  mz = block_reduce(mz, red, true);
+  mq = block_reduce(mq, red, true);
+  mq1 = block_reduce(mq1, red, true);
+  float sz = 0.f, sq = 0.f, sq1 = 0.f;
+  for (int v = threadIdx.x; v < a.V; v += blockDim.x) {
+    sz += expf(z[v] - mz);
+    sq += expf(l[v] * it - mq);
+    sq1 += expf(l[v] - mq1);
+  }
+  sz = block_reduce(sz, red, false);
+  sq = block_reduce(sq, red, false);
+  sq1 = block_reduce(sq1, red, false);
+  const float lz = mz + logf(sz), lq = mq + logf(sq), lq1 = mq1 + logf(sq1);
+  float kl = 0.f, kl1 = 0.f, ent = 0.f;
+  for (int v = threadIdx.x; v < a.V; v += blockDim.x) {
+    const float lp = z[v] - lz;
+    const float p = expf(lp);
+    kl = fmaf(p, lp - (l[v] * it - lq), kl);
+    kl1 = fmaf(p, lp - (l[v] - lq1), kl1);
+    ent = fmaf(-p, lp, ent);
+  }
+  kl = block_reduce(kl, red, false);
+  kl1 = block_reduce(kl1, red, false);
+  ent = block_reduce(ent, red, false);
+  if (threadIdx.x == 0) {
+    const int* meta = a.log_meta + n * 6;
+    rs[RS_LSEZ] = lz;
+    rs[RS_LSEQ] = lq;
+    rs[RS_LSEQ1] = lq1;
+    rs[RS_KL] = kl;
+    rs[RS_KL1] = kl1;
+    rs[RS_ENT] = ent;
+    rs[RS_NLLA] = -(z[meta[1]] - lz);
+    rs[RS_NLLY] = -(z[meta[5]] - lz);
+  }
+}
+
+// Weights of the terms at update t (Sec. 3.4's schedule; readings of the
+// unnamed constants are the config's).
+struct TermW { float kl, pg, ce, ent, rl, beta; };
+__device__ TermW term_weights(const dvi_update_config& c, int t) {
+  TermW w{0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (c.objective == 1) { w.kl = c.lambda0; return w; }
+  if (c.objective == 2) { w.rl = 1.f; return w; }
+  if (c.objective == 3) { w.pg = 1.f; return w; }
+  if (t < c.t_warmup) {
+    w.pg = 0.f;
+    w.kl = c.lambda0;
+  } else if (t < c.t_warmup + c.t_ramp) {
+    const float f = static_cast<float>(t - c.t_warmup) / static_cast<float>(c.t_ramp);
+    w.pg = f * c.lambda_pg_max;
+    w.kl = c.lambda0 - f * (c.lambda0 - c.lambda_kl_min);
+  } else {
+    w.pg = c.lambda_pg_max;
+    w.kl = c.lambda_kl_min;
+  }
+  w.ce = c.w_ce;
+  w.ent = c.w_ent;
+  if (t >= c.t_warmup) {
+    const float f = c.t_ramp > 0 ? fminf(1.f, static_cast<float>(t - c.t_warmup) / c.t_ramp) : 1.f;
+    w.rl = c.w_rl_max * f;
+    w.beta = c.beta_min + (c.beta0 - c.beta_min) * expf(-static_cast<float>(t - c.t_warmup) / c.t_beta);
+  }
+  return w;
+}
+
+__global__ void update_coef_kernel(const UpdateArgs a) {
+  if (threadIdx.x != 0) return;
+  const int t = static_cast<int>(a.dev_state[DS_T]);
+  const float b = a.dev_state[DS_B];
+  const TermW w = term_weights(a.cfg, t);
+  int N = 0, nP = 0;
+  float s_kl = 0.f, s_pg = 0.f, s_ce = 0.f, s_ent = 0.f, s_rl = 0.f, s_kl1 = 0.f, s_r = 0.f;
+  for (int n = 0; n < a.cap; ++n) {
+    if (!row_valid(a, n)) continue;
+    const float* rs = a.rowstat + n * RS_N;
+    const float r = static_cast<float>(a.log_meta[n * 6 + 2]);
+    ++N;
+    s_r += r;
+    s_kl += rs[RS_KL];
+    s_kl1 += rs[RS_KL1];
+    s_ce += rs[RS_NLLY];
+    s_ent += rs[RS_ENT];
+    s_rl += (r - b) * rs[RS_NLLA];
+    if (r == 1.f) { ++nP; s_pg += rs[RS_NLLA]; }
+  }
+  const float fN = N > 0 ? static_cast<float>(N) : 1.f;
+  const float kl = N ? s_kl / fN : 0.f, kl1 = N ? s_kl1 / fN : 0.f, ce = N ? s_ce / fN : 0.f;
+  const float ent = N ? s_ent / fN : 0.f, rl = N ? s_rl / fN : 0.f, pg = nP ? s_pg / nP : 0.f;
+  const float loss = w.kl * kl + w.pg * pg + w.ce * ce - w.ent * ent + w.rl * rl + w.beta * kl1;
+  const bool skip = (N == 0) || !isfinite(loss);
+  if (N > 0 && !isfinite(loss)) flag_status(a.status, DVI_DEV_NONFINITE);
+  a.dev_state[DS_LOSS] = loss;
+  a.dev_state[DS_KL] = kl;
+  a.dev_state[DS_PG] = pg;
+  a.dev_state[DS_CE] = ce;
+  a.dev_state[DS_ENT] = ent;
+  a.dev_state[DS_RL] = rl;
+  a.dev_state[DS_KL1] = kl1;
+  a.dev_state[DS_ACC] = N ? s_r / fN : 0.f;
+  a.dev_state[DS_SKIP] = skip ? 1.f : 0.f;
+  for (int n = 0; n < a.cap; ++n) {
+    float* cf = a.coef + n * CF_N;
+    if (skip || !row_valid(a, n)) {
+      for (int q = 0; q < CF_N; ++q) cf[q] = 0.f;
+      continue;
+    }
+    const float r = static_cast<float>(a.log_meta[n * 6 + 2]);
+    cf[CF_KL] = w.kl / fN;
+    cf[CF_KL1] = w.beta / fN;
+    cf[CF_ENT] = w.ent / fN;
+    cf[CF_A] = (r == 1.f && nP ? w.pg / nP : 0.f) + w.rl * (r - b) / fN;
+    cf[CF_Y] = w.ce / fN;
+  }
+  if (!skip) {
+    const float rho = a.cfg.baseline_rho;
+    a.dev_state[DS_B] = rho * b + (1.f - rho) * (s_r / fN);
+    a.dev_state[DS_ADAM] += 1.f;
+  }
+}
+
+__device__ __forceinline__ void opt_step(const dvi_update_config& c, float step, float g, float* p, float* m,
+                                         float* v) {
+  if (c.optimizer == 1) {
+    *p -= c.lr * g;
+    return;
+  }
+  const float mn = c.beta1 * *m + (1.f - c.beta1) * g;
+  const float vn = c.beta2 * *v + (1.f - c.beta2) * g * g;
+  *m = mn;
+  *v = vn;
+  const float mh = mn / (1.f - powf(c.beta1, step));
+  const float vh = vn / (1.f - powf(c.beta2, step));
+  *p -= c.lr * mh / (sqrtf(vh) + c.adam_eps);
+}
+
+// grid = ceil(V/128); dynamic smem: G tile [cap][128] + A tile [128][r]
+__global__ void __launch_bounds__(128) update_grad_a_kernel(const UpdateArgs a) {
+  extern __shared__ float sm[];
+  if (a.dev_state[DS_SKIP] != 0.f) return;
+  float* Gs = sm;                              // [cap][128]
+  float* As = Gs + static_cast<size_t>(a.cap) * 128;   // [128][r]
+  const int tid = threadIdx.x;
+  const int v = blockIdx.x * 128 + tid;
+  const bool ok = v < a.V;
+  const float it = 1.f / a.cfg.tau;
+  float dA[kMaxRank];
+  float Av[kMaxRank];
+  for (int j = 0; j < a.r; ++j) {
+    dA[j] = 0.f;
+    Av[j] = ok ? a.lora_a[static_cast<size_t>(v) * a.r + j] : 0.f;
+    As[tid * a.r + j] = Av[j];
+  }
+  for (int n = 0; n < a.cap; ++n) {
+    float G = 0.f;
+    if (ok && row_valid(a, n)) {
+      const float* rs = a.rowstat + n * RS_N;
+      const float* cf = a.coef + n * CF_N;
+      const float z = a.Z[static_cast<size_t>(n) * a.V + v];
+      const float l = a.log_logits[static_cast<size_t>(n) * a.V + v];
+      const float lp = z - rs[RS_LSEZ];
+      const float p = expf(lp);
+      const float lq = l * it - rs[RS_LSEQ];
+      const float lq1 = l - rs[RS_LSEQ1];
+      const int* meta = a.log_meta + n * 6;
+      G = cf[CF_KL] * p * (lp - lq - rs[RS_KL]) + cf[CF_KL1] * p * (lp - lq1 - rs[RS_KL1]) +
+          cf[CF_ENT] * p * (lp + rs[RS_ENT]) + cf[CF_A] * (p - (v == meta[1] ? 1.f : 0.f)) +
+          cf[CF_Y] * (p - (v == meta[5] ? 1.f : 0.f));
+      const float* ub = a.ub + n * a.r;
+      for (int j = 0; j < a.r; ++j) dA[j] = fmaf(G, ub[j], dA[j]);
+    }
+    Gs[static_cast<size_t>(n) * 128 + tid] = G;
+  }
+  __syncthreads();
+  // partial G A over this vocabulary tile: pairs (n, j)
+  float* part = a.ga_part + static_cast<size_t>(blockIdx.x) * a.cap * a.r;
+  for (int idx = tid; idx < a.cap * a.r; idx += 128) {
+    const int n = idx / a.r, j = idx % a.r;
+    const float* g = Gs + static_cast<size_t>(n) * 128;
+    float acc = 0.f;
+    for (int q = 0; q < 128; ++q) acc = fmaf(g[q], As[q * a.r + j], acc);
+    part[idx] = acc;
+  }
+  if (!ok) return;
+  const float step = a.dev_state[DS_ADAM];
+  for (int j = 0; j < a.r; ++j) {
+    const float g = a.gamma * dA[j];
+    const size_t i = static_cast<size_t>(v) * a.r + j;
+    a.grad_a[i] = g;
+    opt_step(a.cfg, step, g, a.lora_a + i, a.m_a + i, a.v_a + i);
+  }
+}
+
+__global__ void update_ga_reduce_kernel(const UpdateArgs a) {
+  if (a.dev_state[DS_SKIP] != 0.f) return;
+  const int n = blockIdx.x, j = threadIdx.x;
+  if (j >= a.r) return;
+  float acc = 0.f;
+  for (int t = 0; t < a.n_vtiles; ++t) acc += a.ga_part[(static_cast<size_t>(t) * a.cap + n) * a.r + j];
+  a.ga[n * a.r + j] = acc;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) update_grad_b_kernel(const UpdateArgs a) {
+  if (a.dev_state[DS_SKIP] != 0.f) return;
+  const int c = blockIdx.x * 128 + threadIdx.x;
+  if (c >= a.d) return;
+  const float step = a.dev_state[DS_ADAM];
+  for (int j = 0; j < a.r; ++j) {
+    float acc = 0.f;
+    for (int n = 0; n < a.cap; ++n) {
+      if (!row_valid(a, n)) continue;
+      acc = fmaf(a.ga[n * a.r + j], DT<T>::ld(static_cast<const T*>(a.log_u) + static_cast<size_t>(n) * a.d + c),
+                 acc);
+    }
+    const float g = a.gamma * acc;
+    const size_t i = static_cast<size_t>(j) * a.d + c;
+    a.grad_b[i] = g;
+    opt_step(a.cfg, step, g, a.lora_b + i, a.m_b + i, a.v_b + i);
+  }
+}
+
+__global__ void update_finish_kernel(const UpdateArgs a) {
+  for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < a.cap; n += gridDim.x * blockDim.x) a.log_meta[n * 6] = 0;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    a.dev_state[DS_T] += 1.f;
+    *a.log_step = 0;
+    if (a.dev_state[DS_SKIP] == 0.f) a.counters[4] += 1;
+  }
+}
+
+cudaError_t launch_update_prep(const UpdateArgs& a, cudaStream_t s) {
+  if (a.r == 0) return cudaSuccess;
+  if (a.dtype == DVI_BF16) update_prep_kernel<__nv_bfloat16><<<a.cap, 128, 0, s>>>(a);
+  else update_prep_kernel<float><<<a.cap, 128, 0, s>>>(a);
+  return cudaGetLastError();
+}
+cudaError_t launch_update_rowstats(const UpdateArgs& a, cudaStream_t s) {
+  update_rowstats_kernel<<<a.cap, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+cudaError_t launch_update_coef(const UpdateArgs& a, cudaStream_t s) {
+  update_coef_kernel<<<1, 32, 0, s>>>(a);
+  return cudaGetLastError();
+}
+cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s) {
+  if (a.r == 0) return cudaSuccess;
+  const size_t smem = sizeof(float) * (static_cast<size_t>(a.cap) * 128 + 128 * a.r);
+  static size_t attr = 0;
+  if (smem > 48 * 1024 && smem > attr) {
+    cudaFuncSetAttribute(update_grad_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    attr = smem;
+  }
+  update_grad_a_kernel<<<a.n_vtiles, 128, smem, s>>>(a);
+  return cudaGetLastError();
+}
+cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s) {
+  if (a.r == 0) return cudaSuccess;
+  update_ga_reduce_kernel<<<a.cap, 64, 0, s>>>(a);
+  if (a.dtype == DVI_BF16) update_grad_b_kernel<__nv_bfloat16><<<(a.d + 127) / 128, 128, 0, s>>>(a);
+  else update_grad_b_kernel<float><<<(a.d + 127) / 128, 128, 0, s>>>(a);
+  return cudaGetLastError();
+}
+cudaError_t launch_update_finish(const UpdateArgs& a, cudaStream_t s) {
+  update_finish_kernel<<<(a.cap + 255) / 256, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace dvi

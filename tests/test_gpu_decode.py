@@ -1,0 +1,182 @@
+"""DVI decode and update through the C-ABI on the GPU, against the CPU oracle.
+
+* fp32 (tiny workload): committed tokens bit-exact to the oracle and to greedy
+  AR, the same accept lengths, logged verifier logits within 1e-4, drafter
+  gradients within 1e-3 relative (Sec. 3.3, Sec. 3.4).
+* bf16: the GPU's DVI stream equals the GPU's own greedy AR stream bit for
+  bit (lossless), and the logged verifier logits are within 3e-2 of the
+  oracle's teacher-forced logits on the bf16-rounded weights.
+* Batch of ragged prompts, CUDA-graph vs eager launch, and the full-acceptance
+  case (drafter = the whole model).
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import OracleModel, greedy_ar, dvi_generate, DrafterUpdater
+from oracle.update import head_logits, grad_logits, param_grads, objective_weights, total_loss
+from workloads import workload, make_weights, make_prompts, tiny_shape, UpdateHyper
+from gpu_helpers import engine_for, rounded_weights, teacher_forced_logits
+
+pytestmark = pytest.mark.gpu
+GOLD = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "tiny_dvi.json")))
+
+
+def test_tiny_f32_dvi_matches_oracle_golden():
+    w = workload("tiny")
+    eng, W, _ = engine_for(w)
+    P = make_prompts(w)
+    toks, mats, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
+    st = eng.stats()
+    assert st["device_status"] == 0, st["device_flags"]
+    assert toks[0] == GOLD["dvi_tokens"]
+    assert list(mats[:, 0]) == GOLD["accept_lengths"]
+    assert st["updates"] == len(GOLD["update_losses"])
+    eng.close()
+
+
+def test_tiny_f32_ar_matches_oracle_golden():
+    w = workload("tiny")
+    eng, _, _ = engine_for(w)
+    ar = eng.generate_ar(make_prompts(w), w.gen_tokens)
+    assert list(ar[0]) == GOLD["ar_tokens"]
+    eng.close()
+
+
+class Recorder(DrafterUpdater):
+    def __init__(self, *a, **k):
+        super().__init__(*a, **k)
+        self.buffers = []
+
+    def update(self, tuples):
+        self.buffers.append(list(tuples))
+        return super().update(tuples)
+
+
+@pytest.mark.parametrize("objective", ["kl", "dvi_all_terms", "ce", "pg"])
+def test_tiny_f32_logged_tuples_and_gradients(objective):
+    """One update period: logged logits/u, then dA, dB against the oracle."""
+    w = workload("tiny")
+    if objective == "dvi_all_terms":
+        # past warmup and ramp at t = 0: KL, reward-masked CE, REINFORCE, KL(p||q1), CE, entropy
+        hyper = UpdateHyper(objective="dvi", lr=1e-3, t_warmup=0, t_ramp=0, w_ent=0.01, w_ce=0.05)
+    else:
+        hyper = UpdateHyper(objective=objective, lr=1e-3)
+    W = make_weights(w)
+    W.lora_a[:] = np.random.default_rng(11).standard_normal(W.lora_a.shape).astype(np.float32) * 0.05
+    eng, _, dw = engine_for(w, W=W)
+    P = make_prompts(w)
+    U = w.update_every
+    toks, mats, _, _ = eng.generate(P, 10 ** 6, max_steps=U)
+    eng.sync()
+    meta = eng.buffer("LOG_META", torch.int32).view(-1, 6).cpu().numpy()
+    lg = eng.buffer("LOG_LOGITS", torch.float32).view(-1, w.shape.vocab).cpu().numpy()
+    lu = eng.buffer("LOG_U", torch.float32).view(-1, w.shape.d_model).cpu().numpy()
+    eng.update(hyper)
+    eng.sync()
+    ga = eng.buffer("GRAD_A", torch.float32).view(w.shape.vocab, -1).cpu().numpy()
+    gb = eng.buffer("GRAD_B", torch.float32).view(w.lora_rank, -1).cpu().numpy()
+    st = eng.stats()
+    eng.close()
+
+    m = OracleModel(W, w.shape, w.lora_gamma)
+    rec = Recorder(m, hyper)
+    res = dvi_generate(m, P, 10 ** 6, w.split_k, w.k_spec, U, rec, max_steps=U)
+    assert [s.m for s in res.steps] == list(mats[:, 0])
+    tup = rec.buffers[0]
+    valid = np.nonzero(meta[:, 0])[0]
+    assert len(valid) == len(tup)
+    for row, t in zip(valid, tup):
+        assert meta[row, 1] == t.a and meta[row, 2] == t.r and meta[row, 3] == t.i
+        assert meta[row, 4] == t.prev_id and meta[row, 5] == t.ystar
+        np.testing.assert_allclose(lg[row], t.logits, atol=1e-4, rtol=0)
+        np.testing.assert_allclose(lu[row], t.u, atol=1e-5, rtol=0)
+    info = res.updates[0]
+    np.testing.assert_allclose(st["last_loss"], info["loss"], rtol=1e-4, atol=1e-6)
+    for name, got in (("A", ga), ("B", gb)):
+        ref = info["grads"][name]
+        rel = np.abs(got - ref).max() / np.abs(ref).max()
+        assert rel < 1e-3, (name, rel)
+
+
+def _bf16_case(seed=0, L=4, k=2, K=5):
+    shape = tiny_shape(n_layers=L, d_model=512, n_heads=4, n_kv_heads=2, head_dim=128, d_ffn=1408, vocab=4000)
+    return workload("tiny").with_(shape=shape, dtype="bf16", weight_seed=seed, split_k=k, k_spec=K,
+                                  lora_rank=16, update_every=4, gen_tokens=48,
+                                  update=UpdateHyper(objective="dvi", t_warmup=2, t_ramp=2, lr=1e-3))
+
+
+@pytest.mark.parametrize("graphs", [True, False])
+def test_bf16_dvi_equals_gpu_ar_and_oracle_teacher_forced(graphs):
+    w = _bf16_case()
+    P = make_prompts(w)
+    eng, W, _ = engine_for(w, use_graphs=graphs)
+    ar = eng.generate_ar(P, w.gen_tokens)[0]
+    eng.close()
+    eng, W, _ = engine_for(w, W=W, use_graphs=graphs)
+    toks, mats, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
+    st = eng.stats()
+    assert st["device_status"] == 0, st["device_flags"]
+    assert toks[0] == list(ar)
+    assert st["updates"] >= 2
+    assert all(0 <= x <= w.k_spec for x in mats[:, 0])
+    eng.close()
+    # teacher-forced verifier logits of the oracle on the bf16-rounded weights
+    model = OracleModel(rounded_weights(W), w.shape, w.lora_gamma)
+    seq = np.concatenate([P[0], np.array(toks[0], dtype=np.int32)])
+    ref = teacher_forced_logits(model, seq)
+    plen = len(P[0])
+    # AR logits at each generated position (recomputed on GPU via a fresh run)
+    eng, _, _ = engine_for(w, W=W, use_graphs=graphs)
+    eng.generate(P, 10 ** 6, max_steps=1)
+    eng.sync()
+    meta = eng.buffer("LOG_META", torch.int32).view(-1, 6).cpu().numpy()
+    lg = eng.buffer("LOG_LOGITS", torch.float32).view(-1, w.shape.vocab).cpu().numpy()
+    eng.close()
+    n0 = plen          # position of the pending token at step 0
+    for i in range(w.k_spec):
+        if meta[i, 0]:
+            err = np.abs(lg[i] - ref[n0 + i]).max()
+            assert err < 3e-2, (i, err)
+
+
+def test_batch_ragged_each_sequence_lossless():
+    w = workload("tiny").with_(batch=3, prompt_len=(9, 40), gen_tokens=40)
+    P = make_prompts(w)
+    assert len({len(p) for p in P}) == 3
+    eng, W, _ = engine_for(w)
+    toks, _, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
+    st = eng.stats()
+    eng.close()
+    assert st["device_status"] == 0
+    m = OracleModel(W, w.shape, w.lora_gamma)
+    for b in range(3):
+        assert toks[b] == list(greedy_ar(m, P[b], w.gen_tokens)), b
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_full_acceptance_when_drafter_is_whole_model(dtype):
+    w = workload("tiny").with_(dtype=dtype, split_k=4, gen_tokens=40, scaled_layers=(), scale=1.0)
+    W = make_weights(w)
+    W.lora_a[:] = 0.0
+    eng, _, _ = engine_for(w, W=W)
+    _, mats, _, _ = eng.generate(make_prompts(w), w.gen_tokens)
+    eng.close()
+    assert (mats[:, 0] == w.k_spec).all()
+
+
+def test_prefill_chunks_do_not_change_results():
+    w = workload("tiny").with_(prompt_len=(70, 70), gen_tokens=20)
+    P = make_prompts(w)
+    outs = []
+    for chunk in (16, 128):
+        eng, W, _ = engine_for(w, prefill_chunk=chunk)
+        outs.append(eng.generate_ar(P, w.gen_tokens)[0])
+        eng.close()
+    m = OracleModel(W, w.shape, w.lora_gamma)
+    ref = greedy_ar(m, P[0], w.gen_tokens)
+    np.testing.assert_array_equal(outs[0], ref)
+    np.testing.assert_array_equal(outs[1], ref)

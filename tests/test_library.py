@@ -1,0 +1,84 @@
+"""The C-ABI library builds, loads and exports every function include/dvi.h
+declares; host-side validation rejects bad configurations without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2510_05421_gb300 import build as build_mod
+from paper_2510_05421_gb300 import dvi as D
+from workloads import WORKLOADS
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "dvi.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    if not os.path.exists(D.LIB_PATH):
+        build_mod.build()
+    return D.lib()
+
+
+def declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dvi_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_function(L):
+    names = declared()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(L, n), n
+    assert sorted(D.EXPORTS) == names
+
+
+def _cfgs(w, **rt):
+    s = w.shape
+    cfg = D.ModelConfig(s.n_layers, s.d_model, s.n_heads, s.n_kv_heads, s.head_dim, s.d_ffn, s.vocab, w.split_k,
+                        w.lora_rank, 1.0, s.rms_eps, s.rope_theta, D.DVI_BF16 if w.dtype == "bf16" else D.DVI_F32)
+    base = dict(batch=w.batch, k_spec=w.k_spec, max_seq_len=w.prompt_len[1] + w.gen_tokens + 64,
+                log_steps=w.update_every, head_mode=0, max_prefill_chunk=128, use_graphs=1)
+    base.update(rt)
+    return cfg, D.RuntimeConfig(**base)
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_workspace_sizes(L, name):
+    cfg, rt = _cfgs(WORKLOADS[name])
+    n = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt))
+    assert n > 0 and n % 256 == 0
+    s = WORKLOADS[name].shape
+    esz = 2 if WORKLOADS[name].dtype == "bf16" else 4
+    kv = 2 * s.n_layers * rt.batch * s.n_kv_heads * rt.max_seq_len * s.head_dim * esz
+    assert kv <= n < kv + (1 << 31)
+
+
+@pytest.mark.parametrize("bad", [dict(k_spec=0), dict(k_spec=17), dict(batch=0), dict(max_seq_len=3),
+                                 dict(log_steps=100), dict(max_prefill_chunk=24), dict(head_mode=1)])
+def test_invalid_runtime_rejected(L, bad):
+    cfg, rt = _cfgs(WORKLOADS["tiny"], **bad)
+    assert L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt)) == 0
+    ctx = ctypes.c_void_p()
+    w = D.WeightsC()
+    rc = L.dvi_create(ctypes.byref(cfg), ctypes.byref(rt), ctypes.byref(w), ctypes.c_void_p(256), 1 << 30, None,
+                      ctypes.byref(ctx))
+    assert rc == -1 and not ctx.value
+
+
+def test_invalid_model_rejected(L):
+    cfg, rt = _cfgs(WORKLOADS["tiny"])
+    for field, val in (("split_k", 0), ("split_k", 5), ("head_dim", 96), ("d_model", 200), ("n_kv_heads", 3),
+                       ("lora_rank", 65), ("dtype", 7)):
+        c = D.ModelConfig.from_buffer_copy(cfg)
+        setattr(c, field, val)
+        assert L.dvi_workspace_bytes(ctypes.byref(c), ctypes.byref(rt)) == 0, field
+
+
+def test_null_context_calls_fail_cleanly(L):
+    assert L.dvi_draft_verify_commit(None, None, None, None) == -1
+    assert L.dvi_update_drafter(None, None) == -1
+    assert L.dvi_ar_step(None, None) == -1
+    assert L.dvi_destroy(None) == -1
+    assert L.dvi_last_error(None) == b"null context"
