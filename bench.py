@@ -1,0 +1,332 @@
+#!/usr/bin/env python
+"""Throughput of the DVI decode step + online drafter update on GB300.
+
+One bench step = `update_every` draft_verify_commit calls (K draft passes
+through layers 1..k and the drafter head, one verify pass of the K rows
+through layers k+1..L and the LM head, accept / commit / rollback / log)
+plus one drafter update on the logged buffer -- every row of the hot path.
+Default workload: Llama-2-7B-shaped decoder in bf16, batch 1, split k=2
+(the paper's split), k_spec 5, 1024-token Zipf(1.1) prompt, update every 4
+steps under the KL->RL schedule; random-init weights (synthetic, seeded).
+
+    python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+Multi-GPU runs are independent replicas (one process per GPU, no
+collective on the data path); value = tokens committed by all ranks / the
+slowest rank's time.  `--impl reference` times the CPU oracle instead (rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from workloads import workload, make_weights, make_prompts  # noqa: E402
+
+METRIC = "committed tokens/s at batch 1"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+# ---------------------------------------------------------------- byte model
+def layer_bytes(s, esz):
+    nq, nkv = s.n_heads * s.head_dim, s.n_kv_heads * s.head_dim
+    return (nq * s.d_model + 2 * nkv * s.d_model + s.d_model * nq + 3 * s.d_model * s.d_ffn) * esz
+
+
+def kv_row_bytes(s, esz):
+    return 2 * s.n_kv_heads * s.head_dim * esz
+
+
+def step_bytes(w, n_ctx):
+    """Algorithmic HBM bytes of one decode step at committed lengths n_ctx[b].
+
+    Weights are streamed once per pass; every KV row a pass attends to is
+    read once for all its queries.  Returns (draft bytes, verify bytes).
+    """
+    s, esz, k, K = w.shape, (2 if w.dtype == "bf16" else 4), w.split_k, w.k_spec
+    lb, kvb, head = layer_bytes(s, esz), kv_row_bytes(s, esz), s.vocab * s.d_model * esz
+    lora = (s.vocab + s.d_model) * w.lora_rank * 4
+    draft = K * (k * lb + head + lora)
+    verify = (s.n_layers - k) * lb + head
+    for n in n_ctx:
+        draft += sum(k * (n + j + 1) * kvb for j in range(K))
+        verify += (s.n_layers - k) * (n + K) * kvb
+    return draft, verify
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    REASONS = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+    def __init__(self, gpu_index):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits",
+                                       "-i", str(gpu_index), "-lms", "100"], stdout=self.f,
+                                      stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        sm, mx, reasons = [], 0.0, set()
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = max(mx, float(r[2]))
+            except (ValueError, IndexError):
+                continue
+            for name, val in zip(self.REASONS, r[5:9]):
+                if val.strip().lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- CPU oracle
+def oracle_sample(w, W, budget_s, prompt_len=64, steps_cap=None, threads=None):
+    """Time the CPU oracle's DVI steps (float32) on a bounded sample.
+
+    Prefill of a truncated prompt is untimed; then DVI steps with an update
+    every `update_every` steps run until `budget_s` of wall time has passed.
+    """
+    from oracle import OracleModel, DrafterUpdater
+    from oracle.decode import prefill, dvi_step
+    m = OracleModel(W, w.shape, w.lora_gamma, dtype=np.float32)
+    upd = DrafterUpdater(m, w.update)
+    P = make_prompts(w)[0][:prompt_len]
+    cache = m.new_cache(prompt_len + 4096)
+    tok, _ = prefill(m, cache, P)
+    n, committed, steps, buf = len(P), 0, 0, []
+    t0 = time.perf_counter()
+    while True:
+        fields, tuples, n, tok = dvi_step(m, cache, n, tok, w.split_k, w.k_spec)
+        committed += len(fields[3])
+        buf.extend(tuples)
+        steps += 1
+        if steps % w.update_every == 0:
+            upd.update(buf)
+            buf = []
+            if time.perf_counter() - t0 >= budget_s or (steps_cap and steps >= steps_cap):
+                break
+    dt = time.perf_counter() - t0
+    return dict(committed=committed, steps=steps, seconds=dt, prompt=len(P))
+
+
+def cpu_baseline_dict(res, w, cores):
+    return {"value": res["committed"] / res["seconds"], "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": (f"{w.shape.n_layers}-layer d{w.shape.d_model} decoder in numpy float32, prompt truncated "
+                       f"to {res['prompt']} tokens (prefill untimed), {res['steps']} DVI steps with an update "
+                       f"every {w.update_every}, {res['seconds']:.1f} s")}
+
+
+# ---------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="dvi", choices=["dvi", "reference"])
+    ap.add_argument("--workload", default="7b")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    w = workload(args.workload)
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        cores = os.cpu_count() or 1
+        W = make_weights(w)
+        res_w = oracle_sample(w, W, 1e9, steps_cap=args.warmup * w.update_every)
+        per = max(1.0, args.cpu_seconds / max(1, args.steps))
+        tot_c, tot_s, tot_steps = 0, 0.0, 0
+        for _ in range(args.steps):
+            r = oracle_sample(w, W, per)
+            tot_c += r["committed"]
+            tot_s += r["seconds"]
+            tot_steps += r["steps"]
+        val = tot_c / tot_s
+        line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                "data": "synthetic", "config": {"workload": w.name},
+                "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                                 "sample": f"{args.steps} samples of ~{per:.1f} s: numpy float32 oracle, prompt "
+                                           f"truncated to 64 tokens, {tot_steps} DVI steps with updates"},
+                "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
+
+    import torch
+    import torch.distributed as dist
+    from paper_2510_05421_gb300 import DVIEngine, DeviceWeights, update_config
+
+    if world > 1:
+        dist.init_process_group("gloo", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    W = make_weights(w)
+    dw = DeviceWeights.from_host(W, w.dtype, device=dev)
+    P = make_prompts(w)
+    U, K = w.update_every, w.k_spec
+    gen_room = max(w.gen_tokens, (args.warmup + args.steps) * U * K)
+    max_len = max(len(p) for p in P) + gen_room + 2 * K + 64
+    eng = DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=K, split_k=w.split_k, lora_rank=w.lora_rank,
+                    lora_gamma=w.lora_gamma, max_seq_len=max_len, log_steps=U, device=local)
+    hyper = update_config(w.update)
+    for b, p in enumerate(P):
+        eng.prefill(b, torch.from_numpy(p).to(dev))
+    eng.log(True)
+
+    def one_step():
+        for _ in range(U):
+            eng.step()
+        eng.update(hyper)
+
+    for _ in range(args.warmup):
+        one_step()
+    eng.sync()
+    lens0 = eng.buffer("LENS", torch.int32).clone()
+    st0 = eng.stats()
+    eng.get_timing()
+    eng.timing(True)
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(eng.stream)
+    for _ in range(args.steps):
+        one_step()
+    e1.record(eng.stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    phases = eng.get_timing()
+    eng.timing(False)
+    st1 = eng.stats()
+    lens1 = eng.buffer("LENS", torch.int32).cpu().numpy()
+    lens0 = lens0.cpu().numpy()
+    committed = st1["committed"] - st0["committed"]
+    dsteps = st1["steps"] - st0["steps"]
+    mat = (st1["accepted"] - st0["accepted"]) / max(1, dsteps * w.batch)
+    launches = st1["kernel_launches"] - st0["kernel_launches"]
+    if world > 1:
+        t = torch.tensor([ms, float(committed)], dtype=torch.float64)
+        tmax = t.clone()
+        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        ms_all, committed_all = float(tmax[0]), float(t[1])
+    else:
+        ms_all, committed_all = ms, float(committed)
+    value = committed_all / (ms_all / 1e3)
+
+    # roofline of the verify pass (and the draft pass), from the phase timing
+    pk, pk_src = peaks()
+    n_mid = (lens0 + lens1) / 2.0
+    draft_b, verify_b = step_bytes(w, n_mid)
+    v_ms = phases["verify"][0] / max(1, phases["verify"][1])
+    d_ms = phases["draft"][0] / max(1, phases["draft"][1])
+    u_ms = phases["update"][0] / max(1, phases["update"][1])
+    hbm = pk["hbm_gbs"]
+    v_gbs = verify_b / (v_ms / 1e3) / 1e9
+    d_gbs = draft_b / (d_ms / 1e3) / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        eng.close()
+        eng = DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=K, split_k=w.split_k, lora_rank=w.lora_rank,
+                        lora_gamma=w.lora_gamma, max_seq_len=max(len(p) for p in P) + w.gen_tokens * K + 64,
+                        log_steps=U, device=local)
+        eng.generate(P, 8, update_every=U, hyper=w.update, max_steps=2 * U)
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        toks, mats, h2d, d2h = eng.generate(P, w.gen_tokens, update_every=U, hyper=w.update)
+        torch.cuda.synchronize(dev)
+        dt = time.perf_counter() - t0
+        nsteps = max(1, len(mats))
+        ntok = sum(len(t) for t in toks)
+        e2e = {"value": ntok / dt, "unit": "tokens/s", "h2d_bytes_per_step": h2d / nsteps,
+               "d2h_bytes_per_step": d2h / nsteps,
+               "note": (f"DVIEngine.generate(): {w.gen_tokens} tokens per sequence from pinned host prompts "
+                        f"({len(P[0])} ids) to host token lists, prefill included, drafter updated every {U} "
+                        f"steps; {len(mats)} decode steps, MAT {float(np.mean(mats)):.3f}")}
+    eng.close()
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_all / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": w.name, "layers": w.shape.n_layers, "d_model": w.shape.d_model,
+                   "batch": w.batch, "split_k": w.split_k, "k_spec": K, "prompt": len(P[0]),
+                   "update_every": U, "lora_rank": w.lora_rank,
+                   "step": f"{U} draft_verify_commit calls + 1 update_drafter",
+                   "l2": "inputs larger than L2: ~13 GB of weights streamed per step",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "mean_accepted_length": mat,
+        "roofline": {"bound": "hbm", "achieved": v_gbs, "peak": hbm, "unit": "GB/s", "frac": v_gbs / hbm,
+                     "traffic": None, "kernel": "verify pass (layers k+1..L + LM head, CUDA-graph replay)",
+                     "bytes_per_launch": verify_b, "ms_per_launch": v_ms, "peak_source": pk_src},
+        "roofline_draft": {"bound": "hbm", "achieved": d_gbs, "peak": hbm, "unit": "GB/s", "frac": d_gbs / hbm,
+                           "bytes_per_launch": draft_b, "ms_per_launch": d_ms},
+        "update_ms": u_ms,
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cores = os.cpu_count() or 1
+        res = oracle_sample(w, W, args.cpu_seconds)
+        line["cpu_baseline"] = cpu_baseline_dict(res, w, cores)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -218,6 +218,15 @@ enum {
 };
 dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes);
 
+/* Device timing of the phases for measurement: while enabled, CUDA events
+ * are recorded on the context's stream around the draft phase (0), the
+ * verify phase (1) and the drafter update (2) of every call. */
+dvi_status dvi_timing(dvi_ctx* ctx, int enable);
+
+/* Synchronise the stream, then return per phase the summed milliseconds
+ * ms[3] and the number of timed calls counts[3] since the last read. */
+dvi_status dvi_get_timing(dvi_ctx* ctx, double* ms, int* counts);
+
 /* Y[M][n_out] = X[M][K] . W[n_out][K]^T through the library's projection
  * kernel (tcgen05 for bf16, FP32 FMA for f32), with X float32 (rounded to the
  * weight dtype first) and Y float32, on the context's stream.  M <= 256.

@@ -85,11 +85,15 @@ struct dvi_ctx {
   std::vector<LayerMaps> maps;
   ProjMaps head_v, head_s;
   int log_enabled = 1;
-  // graph of one decode step
-  cudaGraphExec_t step_exec = nullptr;
+  // graphs of one decode step: the K draft passes, then the verify pass
+  cudaGraphExec_t draft_exec = nullptr, verify_exec = nullptr;
   int step_calls = 0;
-  long long step_launches = 0;
+  long long draft_launches = 0, verify_launches = 0;
   long long launches = 0;
+  // optional per-phase timing (0 draft, 1 verify, 2 update): event pairs
+  int timing = 0;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> ev_marks;
   std::string err;
 };
 
@@ -506,7 +510,7 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode) {
   return DVI_OK;
 }
 
-dvi_status enqueue_step(dvi_ctx* ctx) {
+dvi_status enqueue_draft(dvi_ctx* ctx) {
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   dvi_status rc;
@@ -537,6 +541,13 @@ dvi_status enqueue_step(dvi_ctx* ctx) {
     DVI_CUDA(launch_finalize_draft(st, j, s));
     ctx->launches += 2;
   }
+  return DVI_OK;
+}
+
+dvi_status enqueue_verify(dvi_ctx* ctx) {
+  cudaStream_t s = ctx->stream;
+  const StepState st = step_state(ctx);
+  dvi_status rc;
   Pass pv{ctx->x_ver, ctx->ss_ver, ctx->B * ctx->K, ctx->B * ctx->K, ctx->K, 0, ctx->B, 0};
   if ((rc = enqueue_layers(ctx, ctx->k, ctx->L, pv)) != DVI_OK) return rc;
   HeadPrepArgs h = head_prep_args(ctx, ctx->x_ver, ctx->B * ctx->K);
@@ -560,6 +571,67 @@ void fill_rope_host(int max_len, int hd, float theta, std::vector<float2>& out) 
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+cudaEvent_t take_event(dvi_ctx* c) {
+  if (!c->ev_pool.empty()) {
+    cudaEvent_t e = c->ev_pool.back();
+    c->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Records the start of a timed phase; returns the event to close it with.
+cudaEvent_t mark_begin(dvi_ctx* c) {
+  if (!c->timing) return nullptr;
+  cudaEvent_t e = take_event(c);
+  cudaEventRecord(e, c->stream);
+  return e;
+}
+void mark_end(dvi_ctx* c, int phase, cudaEvent_t b) {
+  if (!c->timing || !b) return;
+  cudaEvent_t e = take_event(c);
+  cudaEventRecord(e, c->stream);
+  c->ev_marks.push_back({phase, {b, e}});
+}
+
+// Runs `fn` eagerly, or captures it once into `*exec` and replays it.
+template <typename Fn>
+dvi_status run_graph(dvi_ctx* ctx, cudaGraphExec_t* exec, long long* nlaunch, bool use_graph, Fn fn) {
+  cudaStream_t s = ctx->stream;
+  if (!use_graph) return fn();
+  if (!*exec) {
+    const long long before = ctx->launches;
+    cudaGraph_t g = nullptr;
+    DVI_CUDA(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
+    dvi_status rc = fn();
+    cudaError_t ce = cudaStreamEndCapture(s, &g);
+    if (rc != DVI_OK) {
+      if (g) cudaGraphDestroy(g);
+      return rc;
+    }
+    if (ce != cudaSuccess) return fail(ctx, DVI_ERR_CUDA, cudaGetErrorString(ce));
+    ce = cudaGraphInstantiate(exec, g, 0);
+    cudaGraphDestroy(g);
+    if (ce != cudaSuccess) {
+      *exec = nullptr;
+      return fail(ctx, DVI_ERR_CUDA, cudaGetErrorString(ce));
+    }
+    *nlaunch = ctx->launches - before;
+    ctx->launches = before;
+  }
+  DVI_CUDA(cudaGraphLaunch(*exec, s));
+  ctx->launches += *nlaunch;
+  return DVI_OK;
+}
+
+void drop_graphs(dvi_ctx* c) {
+  if (c->draft_exec) cudaGraphExecDestroy(c->draft_exec);
+  if (c->verify_exec) cudaGraphExecDestroy(c->verify_exec);
+  c->draft_exec = c->verify_exec = nullptr;
+}
 
 }  // namespace
 
@@ -679,30 +751,17 @@ dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids, int32_t* d_
   if (!ctx) return DVI_ERR_INVALID_ARG;
   cudaStream_t s = ctx->stream;
   ctx->step_calls += 1;
-  if (ctx->rt.use_graphs && ctx->step_calls > 1) {
-    if (!ctx->step_exec) {
-      const long long before = ctx->launches;
-      cudaGraph_t g = nullptr;
-      DVI_CUDA(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
-      dvi_status rc = enqueue_step(ctx);
-      cudaError_t ce = cudaStreamEndCapture(s, &g);
-      if (rc != DVI_OK) return rc;
-      if (ce != cudaSuccess) return fail(ctx, DVI_ERR_CUDA, cudaGetErrorString(ce));
-      ce = cudaGraphInstantiate(&ctx->step_exec, g, 0);
-      cudaGraphDestroy(g);
-      if (ce != cudaSuccess) {
-        ctx->step_exec = nullptr;
-        return fail(ctx, DVI_ERR_CUDA, cudaGetErrorString(ce));
-      }
-      ctx->step_launches = ctx->launches - before;
-      ctx->launches = before;
-    }
-    DVI_CUDA(cudaGraphLaunch(ctx->step_exec, s));
-    ctx->launches += ctx->step_launches;
-  } else {
-    dvi_status rc = enqueue_step(ctx);
-    if (rc != DVI_OK) return rc;
-  }
+  // the first step runs eagerly (it also sets kernel attributes); later
+  // steps replay the captured graphs
+  const bool g = ctx->rt.use_graphs && ctx->step_calls > 1;
+  cudaEvent_t t0 = mark_begin(ctx);
+  dvi_status rc = run_graph(ctx, &ctx->draft_exec, &ctx->draft_launches, g, [&] { return enqueue_draft(ctx); });
+  if (rc != DVI_OK) return rc;
+  mark_end(ctx, 0, t0);
+  cudaEvent_t t1 = mark_begin(ctx);
+  rc = run_graph(ctx, &ctx->verify_exec, &ctx->verify_launches, g, [&] { return enqueue_verify(ctx); });
+  if (rc != DVI_OK) return rc;
+  mark_end(ctx, 1, t1);
   if (d_out_ids)
     DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->out_ids, sizeof(int) * ctx->B * ctx->K, cudaMemcpyDeviceToDevice, s));
   if (d_n_committed)
@@ -715,10 +774,7 @@ dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids, int32_t* d_
 dvi_status dvi_log(dvi_ctx* ctx, int enable) {
   if (!ctx) return DVI_ERR_INVALID_ARG;
   const int e = enable ? 1 : 0;
-  if (e != ctx->log_enabled && ctx->step_exec) {
-    cudaGraphExecDestroy(ctx->step_exec);
-    ctx->step_exec = nullptr;
-  }
+  if (e != ctx->log_enabled) drop_graphs(ctx);
   ctx->log_enabled = e;
   return DVI_OK;
 }
@@ -762,6 +818,7 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   a.counters = ctx->counters;
   a.status = ctx->status;
   a.cfg = *u;
+  cudaEvent_t t0 = mark_begin(ctx);
   DVI_CUDA(launch_update_prep(a, s));
   // drafter logits of every buffer row: Z = U W^S^T + gamma (U B^T) A^T
   Pass ps{nullptr, nullptr, 0, ctx->cap_rows, 1, 0, 1, 0};
@@ -786,6 +843,7 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   DVI_CUDA(launch_update_grad_b(a, s));
   DVI_CUDA(launch_update_finish(a, s));
   ctx->launches += 8;
+  mark_end(ctx, 2, t0);
   return DVI_OK;
 }
 
@@ -840,7 +898,12 @@ const char* dvi_last_error(const dvi_ctx* ctx) { return ctx ? ctx->err.c_str() :
 
 dvi_status dvi_destroy(dvi_ctx* ctx) {
   if (!ctx) return DVI_ERR_INVALID_ARG;
-  if (ctx->step_exec) cudaGraphExecDestroy(ctx->step_exec);
+  drop_graphs(ctx);
+  for (auto& m : ctx->ev_marks) {
+    cudaEventDestroy(m.second.first);
+    cudaEventDestroy(m.second.second);
+  }
+  for (cudaEvent_t e : ctx->ev_pool) cudaEventDestroy(e);
   delete ctx;
   return DVI_OK;
 }
@@ -867,6 +930,32 @@ dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes)
     case DVI_BUF_Z: *dptr = ctx->Z; *bytes = sizeof(float) * ctx->cap_rows * static_cast<size_t>(ctx->V); break;
     default: return fail(ctx, DVI_ERR_INVALID_ARG, "debug_buffer: unknown buffer");
   }
+  return DVI_OK;
+}
+
+dvi_status dvi_timing(dvi_ctx* ctx, int enable) {
+  if (!ctx) return DVI_ERR_INVALID_ARG;
+  ctx->timing = enable ? 1 : 0;
+  return DVI_OK;
+}
+
+dvi_status dvi_get_timing(dvi_ctx* ctx, double* ms, int* counts) {
+  if (!ctx || !ms || !counts) return DVI_ERR_INVALID_ARG;
+  DVI_CUDA(cudaStreamSynchronize(ctx->stream));
+  for (int i = 0; i < 3; ++i) {
+    ms[i] = 0.0;
+    counts[i] = 0;
+  }
+  for (auto& m : ctx->ev_marks) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, m.second.first, m.second.second) == cudaSuccess && m.first >= 0 && m.first < 3) {
+      ms[m.first] += t;
+      counts[m.first] += 1;
+    }
+    ctx->ev_pool.push_back(m.second.first);
+    ctx->ev_pool.push_back(m.second.second);
+  }
+  ctx->ev_marks.clear();
   return DVI_OK;
 }
 

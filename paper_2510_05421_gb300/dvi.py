@@ -25,7 +25,7 @@ BUF = dict(LENS=0, PENDING=1, DRAFT_IDS=2, LOG_U=3, LOG_LOGITS=4, LOG_META=5, GR
            X_DRAFT=8, X_VERIFY=9, K_CACHE=10, V_CACHE=11, STATUS=12, GRAD_W=13, Z=14)
 EXPORTS = ["dvi_workspace_bytes", "dvi_create", "dvi_prefill", "dvi_draft_verify_commit", "dvi_log",
            "dvi_update_drafter", "dvi_ar_step", "dvi_get_stats", "dvi_last_error", "dvi_destroy",
-           "dvi_debug_buffer", "dvi_linear"]
+           "dvi_debug_buffer", "dvi_linear", "dvi_timing", "dvi_get_timing"]
 
 
 class ModelConfig(ctypes.Structure):
@@ -107,6 +107,10 @@ def lib() -> ctypes.CDLL:
         L.dvi_debug_buffer.argtypes = [vp, i, P(vp), P(ctypes.c_size_t)]
         L.dvi_linear.restype = i
         L.dvi_linear.argtypes = [vp, vp, i, i, vp, i, vp]
+        L.dvi_timing.restype = i
+        L.dvi_timing.argtypes = [vp, i]
+        L.dvi_get_timing.restype = i
+        L.dvi_get_timing.argtypes = [vp, P(ctypes.c_double), P(i)]
         _lib = L
     return _lib
 
@@ -256,6 +260,16 @@ class DVIEngine:
         off = p.value - self.ws_view.data_ptr()
         return self.ws_view[off:off + n.value].view(dtype)
 
+    def timing(self, enable: bool):
+        self._check(lib().dvi_timing(self.ctx, 1 if enable else 0), "dvi_timing")
+
+    def get_timing(self):
+        """{phase: (total ms, calls)} for 'draft', 'verify', 'update' since the last read."""
+        ms = (ctypes.c_double * 3)()
+        n = (ctypes.c_int * 3)()
+        self._check(lib().dvi_get_timing(self.ctx, ms, n), "dvi_get_timing")
+        return {k: (ms[i], n[i]) for i, k in enumerate(("draft", "verify", "update"))}
+
     def sync(self):
         self.stream.synchronize()
 
@@ -273,14 +287,16 @@ class DVIEngine:
 
     # -- public generation API -------------------------------------------
     def generate(self, prompts: Sequence[np.ndarray], n_gen: int, update_every: int = 0, hyper=None,
-                 max_steps: Optional[int] = None):
+                 max_steps: Optional[int] = None, log: Optional[bool] = None):
         """Self-speculative generation from host prompts to host token lists.
 
         Each prompt is copied from pinned host memory, prefilled, then steps
         run until every sequence has n_gen tokens; an update of the drafter
-        runs every `update_every` steps.  Returns (tokens per sequence,
-        per-step accept lengths [steps, B], bytes copied h2d, bytes d2h).
+        runs every `update_every` steps.  Replay-buffer logging is on when
+        updates are requested (or when `log` says so).  Returns (tokens per
+        sequence, per-step accept lengths [steps, B], bytes h2d, bytes d2h).
         """
+        self.log(bool(update_every and hyper is not None) if log is None else log)
         h2d = d2h = 0
         for b, p in enumerate(prompts):
             hp = torch.from_numpy(np.ascontiguousarray(p, dtype=np.int32)).pin_memory()
@@ -322,11 +338,13 @@ class DVIEngine:
 
     def generate_ar(self, prompts: Sequence[np.ndarray], n_gen: int):
         """Greedy AR baseline through dvi_ar_step (tokens to host at the end)."""
+        outs = torch.empty(self.B, n_gen, dtype=torch.int32, device=self.device)
         for b, p in enumerate(prompts):
             dp = torch.from_numpy(np.ascontiguousarray(p, dtype=np.int32)).to(self.device)
             self.prefill(b, dp)
-        outs = [self.first.clone()]
-        for _ in range(n_gen - 1):
-            outs.append(self.ar_step().clone())
+        with torch.cuda.stream(self.stream):
+            outs[:, 0].copy_(self.first)
+            for i in range(1, n_gen):
+                outs[:, i].copy_(self.ar_step())
         self.stream.synchronize()
-        return torch.stack(outs, 1).cpu().numpy()
+        return outs.cpu().numpy()
