@@ -234,6 +234,29 @@ dvi_status dvi_get_timing(dvi_ctx* ctx, double* ms, int* counts);
 dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in,
                       const float* d_x, int m_rows, float* d_y);
 
+/* Y[M][n_out] = X[M][K] . W[n_out][K]^T like dvi_linear, for callers that
+ * cannot allocate device memory (code inside another framework's memory
+ * pool or a fixed device-memory budget, plug-ins that are handed only their
+ * input and output buffers).  It needs no context and allocates nothing:
+ * the split-K scratch is a fixed array inside the library, 8 MiB of partial
+ * sums plus 4096 tile counters, which every GPU that loads the library
+ * holds until the process exits.  The paper has no counterpart to this
+ * call; it is a deployment convenience.
+ *  - dtype: DVI_BF16 (tcgen05 path; k_in % 8 == 0, 16-byte aligned d_w and
+ *    d_x) or DVI_F32 (FP32 FMA path).  d_w [n_out][k_in] in that dtype,
+ *    d_x [m_rows][k_in] f32 (rounded to the dtype), d_y [m_rows][n_out] f32,
+ *    all device pointers owned by the caller; 1 <= m_rows <= 256.
+ *  - Shapes whose split plan needs more scratch than the fixed array holds
+ *    return DVI_ERR_CAPACITY (with a message on stderr); for example a
+ *    4096 x 4096 weight fits for up to 32 rows.
+ *  - The first call on a device looks up the scratch address for that
+ *    device; make that first call before any stream capture.
+ *  - All calls on a device share the one scratch array, and it keeps the
+ *    last call's contents (the counters are cleared at the start of each
+ *    call): calls that overlap on the GPU, e.g. on two streams, race. */
+dvi_status dvi_linear_noalloc(int dtype, const void* d_w, int n_out, int k_in, const float* d_x,
+                              int m_rows, float* d_y, dvi_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

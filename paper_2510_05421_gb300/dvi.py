@@ -25,7 +25,7 @@ BUF = dict(LENS=0, PENDING=1, DRAFT_IDS=2, LOG_U=3, LOG_LOGITS=4, LOG_META=5, GR
            X_DRAFT=8, X_VERIFY=9, K_CACHE=10, V_CACHE=11, STATUS=12, GRAD_W=13, Z=14)
 EXPORTS = ["dvi_workspace_bytes", "dvi_create", "dvi_prefill", "dvi_draft_verify_commit", "dvi_log",
            "dvi_update_drafter", "dvi_ar_step", "dvi_get_stats", "dvi_last_error", "dvi_destroy",
-           "dvi_debug_buffer", "dvi_linear", "dvi_timing", "dvi_get_timing"]
+           "dvi_debug_buffer", "dvi_linear", "dvi_timing", "dvi_get_timing", "dvi_linear_noalloc"]
 
 
 class ModelConfig(ctypes.Structure):
@@ -111,6 +111,8 @@ def lib() -> ctypes.CDLL:
         L.dvi_timing.argtypes = [vp, i]
         L.dvi_get_timing.restype = i
         L.dvi_get_timing.argtypes = [vp, P(ctypes.c_double), P(i)]
+        L.dvi_linear_noalloc.restype = i
+        L.dvi_linear_noalloc.argtypes = [i, vp, i, i, vp, i, vp, vp]
         _lib = L
     return _lib
 
@@ -159,6 +161,19 @@ class DeviceWeights:
         lm = mat(w.lm_head)
         return DeviceWeights(embed=mat(w.embed), layers=layers, final_norm=f32(w.final_norm), lm_head=lm,
                              draft_head=lm.clone(), lora_a=f32(w.lora_a), lora_b=f32(w.lora_b))
+
+
+def linear_noalloc(w: torch.Tensor, x: torch.Tensor, y: torch.Tensor, stream=None) -> int:
+    """Y = X W^T through dvi_linear_noalloc (no context, no device allocation).
+
+    For callers that cannot allocate device memory: the caller provides w
+    ([N, K] bf16 or f32), x ([M, K] f32) and y ([M, N] f32); the library's
+    fixed scratch is used.  Returns the status code (0 on success).
+    """
+    dtype = DVI_BF16 if w.dtype == torch.bfloat16 else DVI_F32
+    s = stream if stream is not None else torch.cuda.current_stream(w.device)
+    return lib().dvi_linear_noalloc(dtype, _ptr(w), w.shape[0], w.shape[1], _ptr(x), x.shape[0], _ptr(y),
+                                    ctypes.c_void_p(s.cuda_stream))
 
 
 class DVIEngine:
