@@ -26,6 +26,9 @@ struct LayerMaps {
   ProjMaps qkv, o, gu, down;
 };
 
+// One pass of token rows through layers: the f32 residual stream x, its
+// per-tile sums of squares ss, and xg = x * g (the next projection's
+// activation rows in the model dtype) with its TMA descriptor.
 struct Pass {
   float* x;
   float* ss;
@@ -35,6 +38,8 @@ struct Pass {
   int seq0;
   int n_seqs;
   int pos_off;
+  void* xg;
+  const CUtensorMap* xg_map;
 };
 
 struct Plan {
@@ -60,7 +65,7 @@ struct dvi_ctx {
   long long* counters;
   float* dev_state;
   float *x_dr, *ss_dr, *x_ver, *ss_ver, *x_pf, *ss_pf, *q, *bu;
-  void *attn_o, *ffn_h, *u_buf;
+  void *xg_dr, *xg_ver, *xg_pf, *attn_o, *ffn_h;
   unsigned long long* amax;
   void *kcache, *vcache;
   float2* rope;
@@ -84,6 +89,8 @@ struct dvi_ctx {
   Plan p_qkv, p_o, p_gu, p_down, p_head;
   std::vector<LayerMaps> maps;
   ProjMaps head_v, head_s;
+  // TMA descriptors of the activation buffers (bf16 model)
+  CUtensorMap map_xg_dr, map_xg_ver, map_xg_pf, map_attn_o, map_ffn_h, map_log_u;
   int log_enabled = 1;
   // graphs of one decode step: the K draft passes, then the verify pass
   cudaGraphExec_t draft_exec = nullptr, verify_exec = nullptr;
@@ -167,11 +174,13 @@ size_t layout(dvi_ctx* c, char* base) {
   c->ss_ver = reinterpret_cast<float*>(take(sizeof(float) * st * B * K));
   c->x_pf = reinterpret_cast<float*>(take(sizeof(float) * c->chunk * d));
   c->ss_pf = reinterpret_cast<float*>(take(sizeof(float) * st * c->chunk));
+  c->xg_dr = take(e * B * d);
+  c->xg_ver = take(e * B * K * d);
+  c->xg_pf = take(e * c->chunk * d);
   c->q = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * c->nq));
   c->bu = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * (r > 0 ? r : 1)));
   c->attn_o = take(e * c->M_max * c->nq);
   c->ffn_h = take(e * c->M_max * c->F);
-  c->u_buf = take(e * c->M_max * d);
   c->amax = reinterpret_cast<unsigned long long*>(take(sizeof(unsigned long long) * c->M_max));
   const size_t kv = static_cast<size_t>(c->L) * B * c->Hkv * c->max_len * c->hd;
   c->kcache = take(e * kv);
@@ -323,6 +332,8 @@ ProjArgs base_args(dvi_ctx* c, int flavor, const Plan& pl, const Pass& ps) {
   a.eps = c->cfg.rms_eps;
   a.d_norm = c->d;
   a.ss_tiles = c->d / kTileRows;
+  a.prefetch_a = 1;
+  a.b_mode = B_ACT;
   return a;
 }
 
@@ -330,18 +341,27 @@ size_t layer_kv_offset(dvi_ctx* c, int l) {
   return static_cast<size_t>(l) * c->B * c->Hkv * c->max_len * c->hd * c->esz;
 }
 
-dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps) {
+ProjMaps with_act(const ProjMaps& w, const CUtensorMap* act) {
+  ProjMaps m = w;
+  if (act) m.mb = *act;
+  return m;
+}
+
+// One decoder layer on the pass's rows.  `g_last` is the gain of whatever
+// consumes the pass's residual after this layer (the next layer's attention
+// norm, or the final norm before a head).
+dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last) {
   const dvi_layer_weights& lw = ctx->layers[l];
-  const LayerMaps* mp = ctx->tc ? &ctx->maps[l] : nullptr;
+  const bool tc = ctx->tc;
   cudaStream_t s = ctx->stream;
-  // q, k, v with RoPE; k, v rows into the cache
+  ProjMaps pm{};
+  // q, k, v of RMSNorm(x) (gain folded into xg, 1/rms in the epilogue), RoPE,
+  // k/v rows into the cache
   ProjArgs a = base_args(ctx, EPI_QKV, ctx->p_qkv, ps);
-  a.b_mode = B_NORM;
-  a.x = ps.x;
-  a.ldx = ctx->d;
+  a.act = ps.xg;
+  a.ld_act = ctx->d;
   a.ss = ps.ss;
   a.ss_ld = ps.ss_ld;
-  a.gain = static_cast<const float*>(lw.attn_norm);
   a.K = ctx->d;
   a.rows_q = ctx->nq;
   a.rows_k = ctx->nkv;
@@ -358,7 +378,8 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps) {
   a.head_dim = ctx->hd;
   a.n_kv_heads = ctx->Hkv;
   a.rope = ctx->rope;
-  DVI_CUDA(launch_proj(a, mp ? &mp->qkv : nullptr, s));
+  if (tc) pm = with_act(ctx->maps[l].qkv, ps.xg_map);
+  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
   // block-causal multi-query attention
   AttnArgs t{};
   t.q = ctx->q;
@@ -385,9 +406,8 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps) {
   t.status = ctx->status;
   t.scale = 1.f / sqrtf(static_cast<float>(ctx->hd));
   DVI_CUDA(launch_attn(t, s));
-  // x += W_o . attn
+  // x += W_o . attn, then xg = x * ffn_norm for the FFN
   a = base_args(ctx, EPI_RESID, ctx->p_o, ps);
-  a.b_mode = B_COPY;
   a.act = ctx->attn_o;
   a.ld_act = ctx->nq;
   a.K = ctx->nq;
@@ -397,25 +417,27 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps) {
   a.ld_res = ctx->d;
   a.ss_out = ps.ss;
   a.ss_out_ld = ps.ss_ld;
-  DVI_CUDA(launch_proj(a, mp ? &mp->o : nullptr, s));
-  // h = SiLU(W_gate n) * (W_up n)
+  a.g_next = static_cast<const float*>(lw.ffn_norm);
+  a.xg_out = ps.xg;
+  a.ld_xg = ctx->d;
+  if (tc) pm = with_act(ctx->maps[l].o, &ctx->map_attn_o);
+  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
+  // h = SiLU(W_gate n) * (W_up n) with n = RMSNorm(x)
   a = base_args(ctx, EPI_GATEUP, ctx->p_gu, ps);
-  a.b_mode = B_NORM;
-  a.x = ps.x;
-  a.ldx = ctx->d;
+  a.act = ps.xg;
+  a.ld_act = ctx->d;
   a.ss = ps.ss;
   a.ss_ld = ps.ss_ld;
-  a.gain = static_cast<const float*>(lw.ffn_norm);
   a.K = ctx->d;
   a.n_out = ctx->F;
   a.w0 = lw.w_gate;
   a.w1 = lw.w_up;
   a.h_out = ctx->ffn_h;
   a.ld_h = ctx->F;
-  DVI_CUDA(launch_proj(a, mp ? &mp->gu : nullptr, s));
-  // x += W_down . h
+  if (tc) pm = with_act(ctx->maps[l].gu, ps.xg_map);
+  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
+  // x += W_down . h, then xg = x * (next norm's gain)
   a = base_args(ctx, EPI_RESID, ctx->p_down, ps);
-  a.b_mode = B_COPY;
   a.act = ctx->ffn_h;
   a.ld_act = ctx->F;
   a.K = ctx->F;
@@ -425,14 +447,27 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps) {
   a.ld_res = ctx->d;
   a.ss_out = ps.ss;
   a.ss_out_ld = ps.ss_ld;
-  DVI_CUDA(launch_proj(a, mp ? &mp->down : nullptr, s));
+  a.g_next = g_last;
+  a.xg_out = ps.xg;
+  a.ld_xg = ctx->d;
+  if (tc) pm = with_act(ctx->maps[l].down, &ctx->map_ffn_h);
+  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
   ctx->launches += 5;
   return DVI_OK;
 }
 
+// Gain of the RMSNorm that reads the residual after layer l-1: layer l's
+// attention norm, or the final norm after the last layer.
+const float* norm_gain_before(dvi_ctx* ctx, int l) {
+  return l < ctx->L ? static_cast<const float*>(ctx->layers[l].attn_norm)
+                    : static_cast<const float*>(ctx->w.final_norm);
+}
+
+// Layers lo..hi-1; after the last one xg holds x * final_norm for a head.
 dvi_status enqueue_layers(dvi_ctx* ctx, int lo, int hi, const Pass& ps) {
   for (int l = lo; l < hi; ++l) {
-    dvi_status st = enqueue_layer(ctx, l, ps);
+    const float* g_last = l + 1 < hi ? norm_gain_before(ctx, l + 1) : static_cast<const float*>(ctx->w.final_norm);
+    dvi_status st = enqueue_layer(ctx, l, ps, g_last);
     if (st != DVI_OK) return st;
   }
   return DVI_OK;
@@ -452,6 +487,8 @@ StepState step_state(dvi_ctx* c) {
   st.x_dr = c->x_dr;
   st.ss_dr = c->ss_dr;
   st.ss_dr_ld = c->B;
+  st.g0 = norm_gain_before(c, 0);
+  st.xg_dr = c->xg_dr;
   st.embed = c->w.embed;
   st.amax = c->amax;
   st.out_ids = c->out_ids;
@@ -466,27 +503,17 @@ StepState step_state(dvi_ctx* c) {
   return st;
 }
 
-HeadPrepArgs head_prep_args(dvi_ctx* c, const float* x, int rows) {
-  HeadPrepArgs h{};
-  h.x = x;
-  h.ldx = c->d;
-  h.gain = static_cast<const float*>(c->w.final_norm);
-  h.eps = c->cfg.rms_eps;
-  h.d = c->d;
-  h.dtype = c->cfg.dtype;
-  h.u_out = c->u_buf;
-  h.ld_u = c->d;
-  h.rows = rows;
-  return h;
-}
-
-// Head projection over `rows` rows of u_buf; W^S (+LoRA) when `draft`.
-dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode) {
-  Pass ps{nullptr, nullptr, 0, rows, 1, 0, 1, 0};
+// Head projection over `rows` activation rows xg (x * final_norm) starting
+// at row `row0` of `act`; 1/rms from `ss`.  W^S (+ LoRA) when `draft`.
+dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, const void* act,
+                        const CUtensorMap* act_map, int row0, const float* ss, int ss_ld) {
+  Pass ps{nullptr, nullptr, 0, rows, 1, 0, 1, 0, nullptr, nullptr};
   ProjArgs a = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
-  a.b_mode = B_COPY;
-  a.act = ctx->u_buf;
+  a.act = act;
   a.ld_act = ctx->d;
+  a.act_row0 = row0;
+  a.ss = ss;
+  a.ss_ld = ss_ld;
   a.K = ctx->d;
   a.n_out = ctx->V;
   a.w0 = draft ? ctx->w.draft_head : ctx->w.lm_head;
@@ -505,7 +532,9 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode) {
     a.log_cap_steps = ctx->cap_steps;
     a.log_rows_per_step = ctx->B * ctx->K;
   }
-  DVI_CUDA(launch_proj(a, ctx->tc ? (draft ? &ctx->head_s : &ctx->head_v) : nullptr, ctx->stream));
+  ProjMaps pm{};
+  if (ctx->tc) pm = with_act(draft ? ctx->head_s : ctx->head_v, act_map);
+  DVI_CUDA(launch_proj(a, ctx->tc ? &pm : nullptr, ctx->stream));
   ctx->launches += 1;
   return DVI_OK;
 }
@@ -515,15 +544,25 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
   const StepState st = step_state(ctx);
   dvi_status rc;
   for (int j = 0; j < ctx->K; ++j) {
-    Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, j};
+    Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, j, ctx->xg_dr, &ctx->map_xg_dr};
     if ((rc = enqueue_layers(ctx, 0, ctx->k, ps)) != DVI_OK) return rc;
-    HeadPrepArgs h = head_prep_args(ctx, ctx->x_dr, ctx->B);
+    // u = RMSNorm_final(h_k) into the replay buffer, B u, and h_k to the verify rows
+    HeadPrepArgs h{};
+    h.x = ctx->x_dr;
+    h.ldx = ctx->d;
+    h.rows = ctx->B;
+    h.gain = static_cast<const float*>(ctx->w.final_norm);
+    h.eps = ctx->cfg.rms_eps;
+    h.d = ctx->d;
+    h.dtype = ctx->cfg.dtype;
     h.x_copy = ctx->x_ver;
     h.ld_copy = ctx->d;
     h.copy_row_stride = ctx->K;
     h.copy_row_off = j;
     h.ss_copy = ctx->ss_ver;
     h.ss_copy_ld = ctx->B * ctx->K;
+    h.g_copy = norm_gain_before(ctx, ctx->k);
+    h.xg_copy = ctx->xg_ver;
     h.log_u = ctx->log_u;
     h.log_step = ctx->log_step;
     h.log_cap_steps = ctx->cap_steps;
@@ -537,7 +576,8 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
       h.r = ctx->r;
     }
     DVI_CUDA(launch_head_prep(h, s));
-    if ((rc = enqueue_head(ctx, true, ctx->B, 0)) != DVI_OK) return rc;
+    if ((rc = enqueue_head(ctx, true, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
+      return rc;
     DVI_CUDA(launch_finalize_draft(st, j, s));
     ctx->launches += 2;
   }
@@ -548,13 +588,14 @@ dvi_status enqueue_verify(dvi_ctx* ctx) {
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   dvi_status rc;
-  Pass pv{ctx->x_ver, ctx->ss_ver, ctx->B * ctx->K, ctx->B * ctx->K, ctx->K, 0, ctx->B, 0};
+  const int M = ctx->B * ctx->K;
+  Pass pv{ctx->x_ver, ctx->ss_ver, M, M, ctx->K, 0, ctx->B, 0, ctx->xg_ver, &ctx->map_xg_ver};
   if ((rc = enqueue_layers(ctx, ctx->k, ctx->L, pv)) != DVI_OK) return rc;
-  HeadPrepArgs h = head_prep_args(ctx, ctx->x_ver, ctx->B * ctx->K);
-  DVI_CUDA(launch_head_prep(h, s));
-  if ((rc = enqueue_head(ctx, false, ctx->B * ctx->K, ctx->log_enabled ? 2 : 0)) != DVI_OK) return rc;
+  if ((rc = enqueue_head(ctx, false, M, ctx->log_enabled ? 2 : 0, ctx->xg_ver, &ctx->map_xg_ver, 0, ctx->ss_ver,
+                         M)) != DVI_OK)
+    return rc;
   DVI_CUDA(launch_finalize_verify(st, s));
-  ctx->launches += 2;
+  ctx->launches += 1;
   return DVI_OK;
 }
 
@@ -682,11 +723,18 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
       LayerMaps& m = ctx->maps[l];
       ok = mk(&m.qkv.m0, lw.wq, ctx->nq, ctx->d) && mk(&m.qkv.m1, lw.wk, ctx->nkv, ctx->d) &&
            mk(&m.qkv.m2, lw.wv, ctx->nkv, ctx->d) && mk(&m.o.m0, lw.wo, ctx->d, ctx->nq) &&
-           mk(&m.gu.m0, lw.w_gate, ctx->F, ctx->d) && mk(&m.gu.m1, lw.w_up, ctx->F, ctx->d) &&
+           aligned16(lw.w_gate) && make_half_weight_map(&m.gu.m0, lw.w_gate, ctx->F, ctx->d) &&
+           aligned16(lw.w_up) && make_half_weight_map(&m.gu.m1, lw.w_up, ctx->F, ctx->d) &&
            mk(&m.down.m0, lw.w_down, ctx->d, ctx->F);
     }
     ok = ok && mk(&ctx->head_v.m0, weights->lm_head, ctx->V, ctx->d) &&
          mk(&ctx->head_s.m0, weights->draft_head, ctx->V, ctx->d);
+    ok = ok && make_act_map(&ctx->map_xg_dr, ctx->xg_dr, ctx->B, ctx->d) &&
+         make_act_map(&ctx->map_xg_ver, ctx->xg_ver, ctx->B * ctx->K, ctx->d) &&
+         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, ctx->chunk, ctx->d) &&
+         make_act_map(&ctx->map_attn_o, ctx->attn_o, ctx->M_max, ctx->nq) &&
+         make_act_map(&ctx->map_ffn_h, ctx->ffn_h, ctx->M_max, ctx->F) &&
+         make_act_map(&ctx->map_log_u, ctx->log_u, ctx->cap_rows, ctx->d);
     if (!ok) {
       fprintf(stderr, "dvi_create: TMA descriptor creation failed (weights must be 16-byte aligned)\n");
       delete ctx;
@@ -728,18 +776,21 @@ dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tok
     e.ldx = ctx->d;
     e.ss = ctx->ss_pf;
     e.ss_ld = ctx->chunk;
+    e.g = norm_gain_before(ctx, 0);
+    e.xg = ctx->xg_pf;
+    e.ldxg = ctx->d;
     e.rows = rows;
     e.status = ctx->status;
     DVI_CUDA(launch_embed(e, s));
     ctx->launches += 1;
-    Pass ps{ctx->x_pf, ctx->ss_pf, ctx->chunk, rows, rows, seq, 1, c0};
+    Pass ps{ctx->x_pf, ctx->ss_pf, ctx->chunk, rows, rows, seq, 1, c0, ctx->xg_pf, &ctx->map_xg_pf};
     dvi_status rc = enqueue_layers(ctx, 0, ctx->L, ps);
     if (rc != DVI_OK) return rc;
     last_rows = rows;
   }
-  HeadPrepArgs h = head_prep_args(ctx, ctx->x_pf + static_cast<size_t>(last_rows - 1) * ctx->d, 1);
-  DVI_CUDA(launch_head_prep(h, s));
-  dvi_status rc = enqueue_head(ctx, false, 1, 0);
+  // verifier head on the last prompt row
+  dvi_status rc = enqueue_head(ctx, false, 1, 0, ctx->xg_pf, &ctx->map_xg_pf, last_rows - 1,
+                               ctx->ss_pf + (last_rows - 1), ctx->chunk);
   if (rc != DVI_OK) return rc;
   DVI_CUDA(launch_finalize_prefill(st, seq, n_tokens, d_first_token, s));
   ctx->launches += 2;
@@ -821,9 +872,8 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   cudaEvent_t t0 = mark_begin(ctx);
   DVI_CUDA(launch_update_prep(a, s));
   // drafter logits of every buffer row: Z = U W^S^T + gamma (U B^T) A^T
-  Pass ps{nullptr, nullptr, 0, ctx->cap_rows, 1, 0, 1, 0};
+  Pass ps{nullptr, nullptr, 0, ctx->cap_rows, 1, 0, 1, 0, nullptr, nullptr};
   ProjArgs p = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
-  p.b_mode = B_COPY;
   p.act = ctx->log_u;
   p.ld_act = ctx->d;
   p.K = ctx->d;
@@ -836,7 +886,9 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   p.lora_bu = ctx->ub;
   p.lora_r = ctx->r;
   p.gamma = ctx->cfg.lora_gamma;
-  DVI_CUDA(launch_proj(p, ctx->tc ? &ctx->head_s : nullptr, s));
+  ProjMaps pm{};
+  if (ctx->tc) pm = with_act(ctx->head_s, &ctx->map_log_u);
+  DVI_CUDA(launch_proj(p, ctx->tc ? &pm : nullptr, s));
   DVI_CUDA(launch_update_rowstats(a, s));
   DVI_CUDA(launch_update_coef(a, s));
   DVI_CUDA(launch_update_grad_a(a, s));
@@ -852,14 +904,13 @@ dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
   cudaStream_t s = ctx->stream;
   StepState st = step_state(ctx);
   st.out_ids = ctx->ar_out;
-  Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0};
+  Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr};
   dvi_status rc = enqueue_layers(ctx, 0, ctx->L, ps);
   if (rc != DVI_OK) return rc;
-  HeadPrepArgs h = head_prep_args(ctx, ctx->x_dr, ctx->B);
-  DVI_CUDA(launch_head_prep(h, s));
-  if ((rc = enqueue_head(ctx, false, ctx->B, 0)) != DVI_OK) return rc;
+  if ((rc = enqueue_head(ctx, false, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
+    return rc;
   DVI_CUDA(launch_finalize_ar(st, s));
-  ctx->launches += 2;
+  ctx->launches += 1;
   if (d_out_ids) DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->ar_out, sizeof(int) * ctx->B, cudaMemcpyDeviceToDevice, s));
   return DVI_OK;
 }
@@ -967,9 +1018,9 @@ dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in, const 
   if (ctx->tc && (k_in % 8 || !aligned16(d_w) || !aligned16(d_x)))
     return fail(ctx, DVI_ERR_INVALID_ARG, "linear: bf16 needs k_in % 8 == 0 and 16-byte aligned pointers");
   Plan pl = plan_for(ctx, EPI_HEAD, n_out, k_in, 0, 0, 0);
-  Pass ps{nullptr, nullptr, 0, m_rows, 1, 0, 1, 0};
+  Pass ps{nullptr, nullptr, 0, m_rows, 1, 0, 1, 0, nullptr, nullptr};
   ProjArgs a = base_args(ctx, EPI_HEAD, pl, ps);
-  a.b_mode = B_COPY_F32;
+  a.b_mode = B_SOFT_F32;
   a.act = d_x;
   a.ld_act = k_in;
   a.K = k_in;

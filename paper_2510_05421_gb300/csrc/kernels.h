@@ -18,27 +18,28 @@ enum Flavor : int {
 };
 
 enum BMode : int {
-  B_NORM = 0,      // B[n][k] = x[n][k] * rstd[n] * gain[k], rstd from sum-of-squares partials
-  B_COPY = 1,      // B[n][k] = act[n][k] in the model dtype
-  B_COPY_F32 = 2   // B[n][k] = act[n][k] given as float32
+  B_ACT = 0,       // B rows from an activation buffer in the model dtype (bf16: TMA via map `mb`)
+  B_SOFT_F32 = 1   // bf16 path: float32 rows converted by warps 0-3 (dvi_linear)
 };
 
 struct ProjArgs {
   int flavor, b_mode, dtype;
   int M;              // token rows
   int n_pad;          // tcgen05 N: multiple of 16, >= M
-  int n_out;          // rows of one weight (GATEUP: F); QKV uses rows_q/k/v
+  int n_out;          // rows of one weight (GATEUP: F, tiles of 64 gate + 64 up rows); QKV uses rows_q/k/v
   int K;              // input features
   int n_tiles, n_splits, kb_total, kb_per_split, n_ttiles;
+  int prefetch_a;     // stream weight tiles before waiting for the previous kernel
   const void* w0;     // f32 path: weight pointers (QKV: wq, wk, wv; GATEUP: gate, up)
   const void* w1;
   const void* w2;
   int rows_q, rows_k, rows_v;
-  // B source
-  const float* x; int ldx;
-  const float* ss; int ss_ld; int ss_tiles;
-  const float* gain; float eps; int d_norm;
-  const void* act; int ld_act;
+  // B operand: rows act_row0 .. act_row0+M-1 of act[.][ld_act]
+  const void* act; int ld_act; int act_row0;
+  // Optional RMSNorm scale applied to every accumulator in the epilogue:
+  // rstd[n] = rsqrt(sum_t ss[t*ss_ld + n] / d_norm + eps) (the norm gain is
+  // already folded into the activation rows).
+  const float* ss; int ss_ld; int ss_tiles; float eps; int d_norm;
   // token row -> (sequence, position)
   const int* lens; int rows_per_seq; int seq0; int pos_off;
   // split-K scratch: partial tiles and arrival counters (counters start at 0
@@ -50,8 +51,10 @@ struct ProjArgs {
   void* kc; void* vc; int max_len; int head_dim;
   int n_kv_heads;
   const float2* rope;
-  // EPI_RESID
+  // EPI_RESID: x += y, per-tile sums of squares of the new x, and the next
+  // projection's activation rows xg = x * g_next in the model dtype
   float* x_res; int ld_res; float* ss_out; int ss_out_ld;
+  const float* g_next; void* xg_out; int ld_xg;
   // EPI_GATEUP
   void* h_out; int ld_h;
   // EPI_HEAD
@@ -64,6 +67,7 @@ struct ProjArgs {
 
 struct ProjMaps {
   CUtensorMap m0, m1, m2;     // bf16 path: TMA descriptors of w0, w1, w2
+  CUtensorMap mb;             // bf16 path: the activation buffer (box 64 x 16 rows)
 };
 
 // Picks n_splits / kb_per_split from the weight shape only (never from M),
@@ -72,6 +76,8 @@ void plan_splits(ProjArgs& a, int n_sms, bool tc);
 size_t proj_partial_floats(const ProjArgs& a, bool tc);
 cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s);
 bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
+bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols);   // 64-row boxes (gate/up)
+bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);
 
 struct AttnArgs {
   const float* q; int ld_q;          // rotated queries [M][H_q*hd]
@@ -94,27 +100,27 @@ cudaError_t launch_attn(const AttnArgs& a, cudaStream_t s);
 // ---- small kernels (misc.cu)
 struct EmbedArgs {
   const void* table; int dtype; int d; int vocab;
-  const int* tokens;                 // device ids, or null -> use `tok_src` indirection
+  const int* tokens;                 // device ids [rows]
   float* x; int ldx;                 // destination rows
-  float* ss; int ss_ld;              // per-128-feature sums of squares
+  float* ss; int ss_ld;              // per-128-feature sums of squares [d/128][ss_ld]
+  const float* g; void* xg; int ldxg;// activation rows x * g of the first projection (model dtype)
   int rows;
   int* status;
 };
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s);
 
+// Drafter-head preparation for draft pass j: u = RMSNorm_final(h_k) (logged
+// into the replay buffer), LoRA B u, and the hand-off of h_k to the verify
+// stream (x, its sums of squares, and x * g_copy for the verify's first layer).
 struct HeadPrepArgs {
-  const float* x; int ldx;           // rows to normalise
+  const float* x; int ldx; int rows;
   const float* gain; float eps; int d;
   int dtype;
-  void* u_out; int ld_u;             // normalised rows in dtype (B operand of the head)
-  int rows;
-  // optional: copy x rows into another residual stream (+ its ss)
   float* x_copy; int ld_copy; int copy_row_stride; int copy_row_off;
   float* ss_copy; int ss_copy_ld;
-  // optional: log u into the replay buffer at slot (log_step*rows_per_step + row*K + j)
+  const float* g_copy; void* xg_copy;
   void* log_u; const int* log_step; int log_cap_steps; int log_rows_per_step; int log_row_stride;
   int log_row_off; int log_enabled;
-  // optional LoRA down-projection: bu[row][j] = sum_c B[j][c] u[c]
   const float* lora_b; float* bu; int r;
 };
 cudaError_t launch_head_prep(const HeadPrepArgs& a, cudaStream_t s);
@@ -123,6 +129,7 @@ struct StepState {
   int B, K, d, vocab, max_len, dtype;
   int* lens; int* pending; int* draft_ids;      // [B][K+1]
   float* x_dr; float* ss_dr; int ss_dr_ld;
+  const float* g0; void* xg_dr;                 // first layer's attention-norm gain, x * g0
   const void* embed;
   unsigned long long* amax;
   int* out_ids; int* n_committed; int* n_accepted;

@@ -90,7 +90,8 @@ extern "C" dvi_status dvi_linear_noalloc(int dtype, const void* d_w, int n_out, 
   a.K = k_in;
   a.n_ttiles = 1;
   a.rows_per_seq = 1;
-  a.b_mode = B_COPY_F32;
+  a.b_mode = B_SOFT_F32;
+  a.prefetch_a = 1;
   a.act = d_x;
   a.ld_act = k_in;
   a.w0 = d_w;

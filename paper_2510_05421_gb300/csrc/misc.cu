@@ -1,7 +1,10 @@
-// Small kernels around the projections: embedding rows, head preparation
-// (final RMSNorm, LoRA down-projection B u, logging u, handing h_k to the
-// verify stream), and the single-CTA finalize kernels that turn argmax keys
+// Small kernels around the projections: embedding rows, drafter-head
+// preparation, and the single-CTA finalize kernels that turn argmax keys
 // into drafted / committed tokens.
+//
+// Every residual row these kernels write is written with its per-128-feature
+// sums of squares (the next RMSNorm's statistics) and with x * g, the next
+// projection's activation row (the norm gain folded in, model dtype).
 //
 // finalize_verify is the accept/commit/rollback step of Sec. 3.3: with
 // y*_{n+i} the verifier's argmax at block row i-1 and t~_i the drafts,
@@ -16,63 +19,80 @@
 
 namespace dvi {
 
+constexpr int kMaxTiles = 64;   // d <= 8192
+
+// One residual row from the embedding table (128 threads): x, x * g and the
+// per-tile sums of squares, with a single block barrier.
 template <typename T>
-__device__ void embed_row_block(const T* table, int tok, int d, float* x, float* ss, int ss_ld, int row,
-                                float* red) {
+__device__ void embed_row_block(const T* table, int tok, int d, float* x, const float* g, T* xg, float* ss,
+                                int ss_ld, int row, float* red) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  for (int t = 0; t < d / kTileRows; ++t) {
+  const int nt = d / kTileRows;
+  for (int t = 0; t < nt; ++t) {
     const int c = t * kTileRows + tid;
     const float v = DT<T>::ld(table + static_cast<size_t>(tok) * d + c);
     x[c] = v;
+    DT<T>::st(xg + c, v * g[c]);
     const float s = warp_sum(v * v);
-    if (lane == 0) red[warp] = s;
-    __syncthreads();
-    if (tid == 0) ss[static_cast<size_t>(t) * ss_ld + row] = (red[0] + red[1]) + (red[2] + red[3]);
-    __syncthreads();
+    if (lane == 0) red[t * 4 + warp] = s;
   }
+  __syncthreads();
+  for (int t = tid; t < nt; t += blockDim.x)
+    ss[static_cast<size_t>(t) * ss_ld + row] = (red[t * 4] + red[t * 4 + 1]) + (red[t * 4 + 2] + red[t * 4 + 3]);
+  __syncthreads();
 }
 
 // ---------------------------------------------------------------- embed
 template <typename T>
 __global__ void __launch_bounds__(128) embed_kernel(const EmbedArgs a) {
-  __shared__ float red[4];
+  __shared__ float red[kMaxTiles * 4];
+  griddep_launch();
+  griddep_wait();
   const int row = blockIdx.x;
   int tok = a.tokens[row];
   if (tok < 0 || tok >= a.vocab) {
     if (threadIdx.x == 0) flag_status(a.status, DVI_DEV_BAD_TOKEN);
     tok = 0;
   }
-  embed_row_block<T>(static_cast<const T*>(a.table), tok, a.d, a.x + static_cast<size_t>(row) * a.ldx, a.ss,
-                     a.ss_ld, row, red);
+  embed_row_block<T>(static_cast<const T*>(a.table), tok, a.d, a.x + static_cast<size_t>(row) * a.ldx, a.g,
+                     static_cast<T*>(a.xg) + static_cast<size_t>(row) * a.ldxg, a.ss, a.ss_ld, row, red);
 }
 
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s) {
-  if (a.dtype == DVI_BF16) embed_kernel<__nv_bfloat16><<<a.rows, 128, 0, s>>>(a);
-  else embed_kernel<float><<<a.rows, 128, 0, s>>>(a);
-  return cudaGetLastError();
+  cudaError_t e = a.dtype == DVI_BF16 ? launch_pdl(embed_kernel<__nv_bfloat16>, dim3(a.rows), dim3(128), 0, s, a)
+                                      : launch_pdl(embed_kernel<float>, dim3(a.rows), dim3(128), 0, s, a);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- head prep
-// grid (rows, ceil(r/4) or 1); block 128.  Every CTA recomputes the row's
-// RMSNorm; CTA y == 0 writes u, logs it and copies x; each CTA computes four
-// entries of B u (one warp each).
+// grid (rows, ceil(r/4) or 1); block 128.  Every CTA computes the row's
+// 1/rms; CTA y == 0 logs u and hands the row to the verify stream; each CTA
+// computes four entries of B u (one warp each).
 template <typename T>
 __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
-  __shared__ float red[4];
+  __shared__ float red[kMaxTiles * 4];
   __shared__ float rstd_s;
+  griddep_launch();
+  griddep_wait();
   const int row = blockIdx.x, grp = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float* x = a.x + static_cast<size_t>(row) * a.ldx;
-  float s = 0.f;
-  for (int c = tid; c < a.d; c += 128) s = fmaf(x[c], x[c], s);
-  s = warp_sum(s);
-  if (lane == 0) red[warp] = s;
+  const int nt = a.d / kTileRows;
+  // per-tile sums of squares (also the hand-off's statistics), then 1/rms
+  for (int t = 0; t < nt; ++t) {
+    const float v = x[t * kTileRows + tid];
+    const float s = warp_sum(v * v);
+    if (lane == 0) red[t * 4 + warp] = s;
+  }
   __syncthreads();
-  if (tid == 0) rstd_s = rsqrtf(((red[0] + red[1]) + (red[2] + red[3])) / static_cast<float>(a.d) + a.eps);
+  if (tid == 0) {
+    float s = 0.f;
+    for (int t = 0; t < nt; ++t) s += (red[t * 4] + red[t * 4 + 1]) + (red[t * 4 + 2] + red[t * 4 + 3]);
+    rstd_s = rsqrtf(s / static_cast<float>(a.d) + a.eps);
+  }
   __syncthreads();
   const float rstd = rstd_s;
   if (grp == 0) {
-    T* u = static_cast<T*>(a.u_out) + static_cast<size_t>(row) * a.ld_u;
     T* lu = nullptr;
     if (a.log_u && a.log_enabled) {
       const int ls = *a.log_step;
@@ -81,23 +101,19 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
              (static_cast<size_t>(ls) * a.log_rows_per_step + static_cast<size_t>(row) * a.log_row_stride +
               a.log_row_off) * a.d;
     }
-    for (int c = tid; c < a.d; c += 128) {
-      const float v = x[c] * rstd * a.gain[c];
-      DT<T>::st(u + c, v);
-      if (lu) DT<T>::st(lu + c, v);
-    }
+    if (lu)
+      for (int c = tid; c < a.d; c += 128) DT<T>::st(lu + c, x[c] * rstd * a.gain[c]);
     if (a.x_copy) {
       const int crow = row * a.copy_row_stride + a.copy_row_off;
       float* xc = a.x_copy + static_cast<size_t>(crow) * a.ld_copy;
-      for (int t = 0; t < a.d / kTileRows; ++t) {
-        const float v = x[t * kTileRows + tid];
-        xc[t * kTileRows + tid] = v;
-        const float q = warp_sum(v * v);
-        __syncthreads();
-        if (lane == 0) red[warp] = q;
-        __syncthreads();
-        if (tid == 0) a.ss_copy[static_cast<size_t>(t) * a.ss_copy_ld + crow] = (red[0] + red[1]) + (red[2] + red[3]);
+      T* xgc = static_cast<T*>(a.xg_copy) + static_cast<size_t>(crow) * a.ld_copy;
+      for (int c = tid; c < a.d; c += 128) {
+        xc[c] = x[c];
+        DT<T>::st(xgc + c, x[c] * a.g_copy[c]);
       }
+      for (int t = tid; t < nt; t += 128)
+        a.ss_copy[static_cast<size_t>(t) * a.ss_copy_ld + crow] =
+            (red[t * 4] + red[t * 4 + 1]) + (red[t * 4 + 2] + red[t * 4 + 3]);
     }
   }
   if (a.r > 0 && a.bu) {
@@ -114,9 +130,9 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
 
 cudaError_t launch_head_prep(const HeadPrepArgs& a, cudaStream_t s) {
   dim3 grid(a.rows, (a.r > 0 && a.bu) ? (a.r + 3) / 4 : 1);
-  if (a.dtype == DVI_BF16) head_prep_kernel<__nv_bfloat16><<<grid, 128, 0, s>>>(a);
-  else head_prep_kernel<float><<<grid, 128, 0, s>>>(a);
-  return cudaGetLastError();
+  cudaError_t e = a.dtype == DVI_BF16 ? launch_pdl(head_prep_kernel<__nv_bfloat16>, grid, dim3(128), 0, s, a)
+                                      : launch_pdl(head_prep_kernel<float>, grid, dim3(128), 0, s, a);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- finalize
@@ -130,17 +146,21 @@ __device__ __forceinline__ int take_argmax(unsigned long long* slot, int* status
   return argmax_idx(k);
 }
 
+// Embeds each sequence's next input token into the draft residual stream.
 template <typename T>
 __device__ void embed_rows(const StepState& st, const int* toks, float* red) {
   for (int b = 0; b < st.B; ++b)
     embed_row_block<T>(static_cast<const T*>(st.embed), toks[b], st.d, st.x_dr + static_cast<size_t>(b) * st.d,
-                       st.ss_dr, st.ss_dr_ld, b, red);
+                       st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(b) * st.d, st.ss_dr, st.ss_dr_ld, b,
+                       red);
 }
 
 template <typename T>
 __global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st, int j) {
   __shared__ int tok_s[64];
-  __shared__ float red[4];
+  __shared__ float red[kMaxTiles * 4];
+  griddep_launch();
+  griddep_wait();
   for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
     const int t = take_argmax(st.amax + b, st.status);
     st.draft_ids[b * (st.K + 1) + j + 1] = t;
@@ -153,7 +173,9 @@ __global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st,
 template <typename T>
 __global__ void __launch_bounds__(128) finalize_verify_kernel(const StepState st) {
   __shared__ int tok_s[64];
-  __shared__ float red[4];
+  __shared__ float red[kMaxTiles * 4];
+  griddep_launch();
+  griddep_wait();
   const int K = st.K;
   const int ls = *st.log_step;
   const bool log_ok = st.log_enabled && ls < st.log_cap_steps;
@@ -204,7 +226,9 @@ __global__ void __launch_bounds__(128) finalize_verify_kernel(const StepState st
 template <typename T>
 __global__ void __launch_bounds__(128) finalize_ar_kernel(const StepState st) {
   __shared__ int tok_s[64];
-  __shared__ float red[4];
+  __shared__ float red[kMaxTiles * 4];
+  griddep_launch();
+  griddep_wait();
   for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
     const int y = take_argmax(st.amax + b, st.status);
     st.out_ids[b] = y;
@@ -220,8 +244,10 @@ __global__ void __launch_bounds__(128) finalize_ar_kernel(const StepState st) {
 template <typename T>
 __global__ void __launch_bounds__(128) finalize_prefill_kernel(const StepState st, int seq, int n_tokens,
                                                                int32_t* first_out) {
-  __shared__ float red[4];
+  __shared__ float red[kMaxTiles * 4];
   __shared__ int tok;
+  griddep_launch();
+  griddep_wait();
   if (threadIdx.x == 0) {
     const int y = take_argmax(st.amax, st.status);
     st.lens[seq] = n_tokens;
@@ -232,37 +258,41 @@ __global__ void __launch_bounds__(128) finalize_prefill_kernel(const StepState s
   }
   __syncthreads();
   embed_row_block<T>(static_cast<const T*>(st.embed), tok, st.d, st.x_dr + static_cast<size_t>(seq) * st.d,
-                     st.ss_dr, st.ss_dr_ld, seq, red);
+                     st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(seq) * st.d, st.ss_dr, st.ss_dr_ld,
+                     seq, red);
 }
 
 __global__ void reset_seq_kernel(const StepState st, int seq) {
+  griddep_launch();
+  griddep_wait();
   st.lens[seq] = 0;
 }
 
+template <typename K, typename... Args>
+static cudaError_t launch1(K kern, cudaStream_t s, Args... args) {
+  const cudaError_t e = launch_pdl(kern, dim3(1), dim3(128), 0, s, args...);
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 cudaError_t launch_finalize_draft(const StepState& st, int j, cudaStream_t s) {
-  if (st.dtype == DVI_BF16) finalize_draft_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st, j);
-  else finalize_draft_kernel<float><<<1, 128, 0, s>>>(st, j);
-  return cudaGetLastError();
+  return st.dtype == DVI_BF16 ? launch1(finalize_draft_kernel<__nv_bfloat16>, s, st, j)
+                              : launch1(finalize_draft_kernel<float>, s, st, j);
 }
 cudaError_t launch_finalize_verify(const StepState& st, cudaStream_t s) {
-  if (st.dtype == DVI_BF16) finalize_verify_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st);
-  else finalize_verify_kernel<float><<<1, 128, 0, s>>>(st);
-  return cudaGetLastError();
+  return st.dtype == DVI_BF16 ? launch1(finalize_verify_kernel<__nv_bfloat16>, s, st)
+                              : launch1(finalize_verify_kernel<float>, s, st);
 }
 cudaError_t launch_finalize_ar(const StepState& st, cudaStream_t s) {
-  if (st.dtype == DVI_BF16) finalize_ar_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st);
-  else finalize_ar_kernel<float><<<1, 128, 0, s>>>(st);
-  return cudaGetLastError();
+  return st.dtype == DVI_BF16 ? launch1(finalize_ar_kernel<__nv_bfloat16>, s, st)
+                              : launch1(finalize_ar_kernel<float>, s, st);
 }
 cudaError_t launch_finalize_prefill(const StepState& st, int seq, int n_tokens, int32_t* first_out,
                                     cudaStream_t s) {
-  if (st.dtype == DVI_BF16) finalize_prefill_kernel<__nv_bfloat16><<<1, 128, 0, s>>>(st, seq, n_tokens, first_out);
-  else finalize_prefill_kernel<float><<<1, 128, 0, s>>>(st, seq, n_tokens, first_out);
-  return cudaGetLastError();
+  return st.dtype == DVI_BF16 ? launch1(finalize_prefill_kernel<__nv_bfloat16>, s, st, seq, n_tokens, first_out)
+                              : launch1(finalize_prefill_kernel<float>, s, st, seq, n_tokens, first_out);
 }
 cudaError_t launch_reset_seq(const StepState& st, int seq, cudaStream_t s) {
-  reset_seq_kernel<<<1, 1, 0, s>>>(st, seq);
-  return cudaGetLastError();
+  return launch1(reset_seq_kernel, s, st, seq);
 }
 
 }  // namespace dvi

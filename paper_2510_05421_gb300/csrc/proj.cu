@@ -6,29 +6,43 @@
 // features (the tcgen05 M dimension) is read from HBM exactly once, and the
 // token rows sit on the MMA's N dimension ("swap AB").
 //
-// bf16 (tcgen05): warp 4 streams 128x64 weight tiles by TMA (128-byte
-// swizzle) into a ring of shared-memory stages; warps 0-3 write the matching
-// B tile (the token rows, RMSNorm-ed on the fly from the f32 residual stream
-// or copied from a bf16 activation) in the same swizzled K-major layout;
-// warp 5 issues tcgen05.mma (M=128, N=n_pad, K=16) into a TMEM accumulator
-// and releases stages with tcgen05.commit.  Warps 0-3 then read TMEM and run
-// the fused epilogue.
+// bf16 (tcgen05): warp 4 streams the 128x64 weight tile and the matching
+// n_pad x 64 activation tile of each K block by TMA (128-byte swizzle, the
+// K-major layout tcgen05 reads) into a ring of shared-memory stages; warp 5
+// issues tcgen05.mma (M=128, N=n_pad, K=16) into a TMEM accumulator and frees
+// stages with tcgen05.commit; warps 0-3 then read TMEM and run the fused
+// epilogue.  A gate/up tile holds 64 rows of W_gate and the same 64 rows of
+// W_up (two 64-row TMA boxes), so SwiGLU pairs rows r and r+64 of one tile.
+// The RMSNorm feeding a projection is split in two: its gain is folded into
+// the activation rows by the kernel that produced them, and its 1/rms (a
+// per-row scalar) multiplies the accumulators in the epilogue.
+// Launches use programmatic dependent launch: the weight tiles of the first
+// stages (which no earlier kernel writes) stream in before the kernel waits
+// for its predecessor.
 //
 // f32 (FP32 FMA, no TF32): the same decomposition with a shared-memory tiled
 // FFMA main loop of 16 token columns per CTA.
 //
 // K is split over `n_splits` CTAs per tile when there are too few tiles to
-// fill the GPU.  Each split stores its partial tile; the last CTA to arrive
-// (an atomic counter per tile) sums the partials in split order -- so results
-// are deterministic -- and runs the epilogue.  The split plan depends only on
-// the weight shape, never on the number of token rows.
+// fill the GPU.  bf16: the splits of a tile form one thread-block cluster;
+// each leaves its partial tile in shared memory and, after a cluster barrier,
+// rank 0 sums the partials of all ranks in rank order through distributed
+// shared memory and runs the epilogue.  f32: each split stores its partial in
+// global scratch and the last CTA to arrive (an atomic counter per tile) sums
+// them in split order.  Both are deterministic, and the split plan depends on
+// the weight shape only (never on the number of decode rows).
 #include <algorithm>
+#include <cooperative_groups.h>
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
 #include "kernels.h"
 
 namespace dvi {
+
+namespace cg = cooperative_groups;
+
+constexpr int kGuRows = 64;   // features per gate/up tile (64 gate rows + 64 up rows)
 
 struct EpiSmem {
   float stage[kTileRows][kChunk + 1];
@@ -42,12 +56,29 @@ __device__ __forceinline__ void row_seq_pos(const ProjArgs& p, int n, int& seq, 
   pos = p.lens[seq] + p.pos_off + n % p.rows_per_seq;
 }
 
+// rstd[n] for the token rows of the launch (1 when there is no norm).
+__device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int tid, int nthreads) {
+  for (int n = tid; n < p.M; n += nthreads) {
+    float r = 1.f;
+    if (p.ss) {
+      float s = 0.f;
+      for (int t = 0; t < p.ss_tiles; ++t) s += p.ss[static_cast<size_t>(t) * p.ss_ld + n];
+      r = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
+    }
+    rstd[n] = r;
+  }
+}
+
 // Fused epilogue for 16 token columns [c0, c0+16) of one 128-feature tile.
 // Called by the 128 epilogue threads together (row = feature within tile).
 template <typename T>
-__device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, const float (&v)[kChunk],
-                               const float (&v2)[kChunk], EpiSmem& es) {
+__device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, float (&v)[kChunk],
+                               const float* rstd, EpiSmem& es) {
   const int warp = row >> 5, lane = row & 31;
+  if (p.ss) {
+#pragma unroll
+    for (int j = 0; j < kChunk; ++j) v[j] *= (c0 + j < p.M) ? rstd[c0 + j] : 0.f;
+  }
   if (p.flavor == EPI_QKV) {
     const int tq = p.rows_q / kTileRows, tk = p.rows_k / kTileRows;
     int sec, lt;
@@ -90,6 +121,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, con
     if (sec < 2) named_bar(1, kTileRows);
   } else if (p.flavor == EPI_RESID) {
     const int f = tile * kTileRows + row;
+    const float g = (p.xg_out && f < p.n_out) ? p.g_next[f] : 0.f;
     float sq[kChunk];
 #pragma unroll
     for (int j = 0; j < kChunk; ++j) {
@@ -99,6 +131,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, con
         float* xp = p.x_res + static_cast<size_t>(n) * p.ld_res + f;
         xn = *xp + v[j];
         *xp = xn;
+        if (p.xg_out) DT<T>::st(static_cast<T*>(p.xg_out) + static_cast<size_t>(n) * p.ld_xg + f, xn * g);
       }
       sq[j] = xn * xn;
     }
@@ -113,18 +146,23 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, con
           (es.red[0][row] + es.red[1][row]) + (es.red[2][row] + es.red[3][row]);
     named_bar(1, kTileRows);
   } else if (p.flavor == EPI_GATEUP) {
-    const int f = tile * kTileRows + row;
-    if (f < p.n_out) {
+    // rows 0..63: W_gate, rows 64..127: W_up, same 64 features
+#pragma unroll
+    for (int j = 0; j < kChunk; ++j) es.stage[row][j] = v[j];
+    named_bar(1, kTileRows);
+    const int f = tile * kGuRows + row;
+    if (row < kGuRows && f < p.n_out) {
 #pragma unroll
       for (int j = 0; j < kChunk; ++j) {
         const int n = c0 + j;
         if (n < p.M) {
-          const float g = v[j];
-          const float h = g / (1.f + expf(-g)) * v2[j];
+          const float gt = es.stage[row][j];
+          const float h = gt / (1.f + expf(-gt)) * es.stage[row + kGuRows][j];
           DT<T>::st(static_cast<T*>(p.h_out) + static_cast<size_t>(n) * p.ld_h + f, h);
         }
       }
     }
+    named_bar(1, kTileRows);
   } else {  // EPI_HEAD
     const int f = tile * kTileRows + row;
     const bool ok = f < p.n_out;
@@ -199,76 +237,61 @@ __device__ __forceinline__ bool split_arrive(const ProjArgs& p, int ci, int row,
   return last;
 }
 
+// Sum of the split partials of one element, in split order; the loads of up
+// to eight splits are issued before their sum so their latencies overlap.
+__device__ __forceinline__ float sum_splits(const float* base, size_t stride, int n_splits) {
+  float a = 0.f;
+  for (int s0 = 0; s0 < n_splits; s0 += 8) {
+    float t[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) t[u] = (s0 + u < n_splits) ? __ldcg(base + (s0 + u) * stride) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (s0 + u < n_splits) a += t[u];
+  }
+  return a;
+}
+
 __device__ __forceinline__ uint32_t tmem_cols(int n) {
   uint32_t c = 32;
   while (c < static_cast<uint32_t>(n)) c <<= 1;
   return c;
 }
 
-// Writes one 64-wide K block of the B operand (token rows) for stage `bs`.
-__device__ __forceinline__ void produce_b_tile(const ProjArgs& p, const float* rstd, uint8_t* bs, int kb,
-                                               int tid) {
+// Writes one 64-wide K block of the B operand from float32 rows (B_SOFT_F32).
+__device__ __forceinline__ void produce_b_f32(const ProjArgs& p, uint8_t* bs, int kb, int tid) {
   const int nslots = p.n_pad * 8;
   for (int slot = tid; slot < nslots; slot += kTileRows) {
     const int n = slot >> 3, c = slot & 7;
     const int k0 = kb * kKBlock + c * 8;
     uint4 val = make_uint4(0u, 0u, 0u, 0u);
     if (n < p.M && k0 < p.K) {
+      const float* src = static_cast<const float*>(p.act) + static_cast<size_t>(p.act_row0 + n) * p.ld_act + k0;
       float f[8];
-      const bool full8 = (k0 + 8 <= p.K);
-      if (p.b_mode == B_COPY) {
-        const __nv_bfloat16* src = static_cast<const __nv_bfloat16*>(p.act) + static_cast<size_t>(n) * p.ld_act + k0;
-        if (full8) {
-          val = *reinterpret_cast<const uint4*>(src);
-        } else {
-          uint32_t w[4] = {0u, 0u, 0u, 0u};
-          for (int e = 0; e < 8 && k0 + e < p.K; ++e) {
-            const uint32_t b = __bfloat16_as_ushort(src[e]);
-            w[e >> 1] |= (e & 1) ? (b << 16) : b;
-          }
-          val = make_uint4(w[0], w[1], w[2], w[3]);
-        }
+      if (k0 + 8 <= p.K) {
+        const float4 a = *reinterpret_cast<const float4*>(src);
+        const float4 b = *reinterpret_cast<const float4*>(src + 4);
+        f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
       } else {
-        const float* src = (p.b_mode == B_NORM ? p.x : static_cast<const float*>(p.act)) +
-                           static_cast<size_t>(n) * (p.b_mode == B_NORM ? p.ldx : p.ld_act) + k0;
-        if (full8) {
-          const float4 a = *reinterpret_cast<const float4*>(src);
-          const float4 b = *reinterpret_cast<const float4*>(src + 4);
-          f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
-        } else {
 #pragma unroll
-          for (int e = 0; e < 8; ++e) f[e] = (k0 + e < p.K) ? src[e] : 0.f;
-        }
-        if (p.b_mode == B_NORM) {
-          const float r = rstd[n];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) f[e] = (k0 + e < p.K) ? f[e] * r * p.gain[k0 + e] : 0.f;
-        }
-        val = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
-                         pack_bf16x2(f[6], f[7]));
+        for (int e = 0; e < 8; ++e) f[e] = (k0 + e < p.K) ? src[e] : 0.f;
       }
+      val = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
+                       pack_bf16x2(f[6], f[7]));
     }
     *reinterpret_cast<uint4*>(bs + n * 128 + ((c ^ (n & 7)) << 4)) = val;
   }
 }
 
-__device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int tid) {
-  for (int n = tid; n < p.M; n += kTileRows) {
-    float s = 0.f;
-    for (int t = 0; t < p.ss_tiles; ++t) s += p.ss[static_cast<size_t>(t) * p.ss_ld + n];
-    rstd[n] = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
-  }
-}
-
 // ------------------------------------------------------------------ tcgen05
-template <bool DUAL>
-__global__ void __launch_bounds__(192, 2)
+__global__ void __launch_bounds__(192, 3)
     proj_tc_kernel(const __grid_constant__ CUtensorMap m0, const __grid_constant__ CUtensorMap m1,
-                   const __grid_constant__ CUtensorMap m2, const ProjArgs p, int stages) {
+                   const __grid_constant__ CUtensorMap m2, const __grid_constant__ CUtensorMap mb,
+                   const ProjArgs p, int stages) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-  constexpr int abytes = DUAL ? 32768 : 16384;
+  constexpr int abytes = 16384;
   const int bbytes = p.n_pad * 128;
   uint8_t* sA = base;
   uint8_t* sB = base + stages * abytes;
@@ -277,18 +300,23 @@ __global__ void __launch_bounds__(192, 2)
   uint64_t* done = empty + stages;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   float* rstd = reinterpret_cast<float*>(tmem_holder + 4);
-  EpiSmem& es = *reinterpret_cast<EpiSmem*>(sA);   // A stages are free once `done` fired
+  // after `done` the A stages are free: epilogue scratch, then this split's
+  // partial tile [n_pad][128] for the cluster reduction
+  EpiSmem& es = *reinterpret_cast<EpiSmem*>(sA);
+  float* part = reinterpret_cast<float*>(sA + abytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile = blockIdx.x / p.n_splits, split = blockIdx.x % p.n_splits;
   const int kb0 = split * p.kb_per_split;
   const int nkb = min(p.kb_per_split, p.kb_total - kb0);
-  const uint32_t ncols = tmem_cols(p.n_pad * (DUAL ? 2 : 1));
+  const uint32_t ncols = tmem_cols(p.n_pad);
+  const bool soft_b = p.b_mode == B_SOFT_F32;
+  const bool gu = p.flavor == EPI_GATEUP;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
-      mbar_init(&full[s], 5);     // TMA expect_tx arrival + one arrival per B-producer warp
-      mbar_init(&empty[s], 1);    // tcgen05.commit
+      mbar_init(&full[s], soft_b ? 5 : 1);   // TMA arrival (+ one per B-producer warp)
+      mbar_init(&empty[s], 1);               // tcgen05.commit
     }
     mbar_init(done, 1);
     mbar_fence_init();
@@ -296,16 +324,19 @@ __global__ void __launch_bounds__(192, 2)
   if (warp == 0) tmem_alloc(tmem_holder, ncols);
   if (warp == 4 && lane == 0) {
     tma_prefetch_desc(&m0);
-    if (DUAL || p.flavor == EPI_QKV) tma_prefetch_desc(&m1);
+    if (gu || p.flavor == EPI_QKV) tma_prefetch_desc(&m1);
     if (p.flavor == EPI_QKV) tma_prefetch_desc(&m2);
+    if (!soft_b) tma_prefetch_desc(&mb);
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  griddep_launch();
   const uint32_t tmem = *tmem_holder;
+  bool ok = true;
 
   if (warp == 4) {
-    // ---------------- TMA producer (weights)
+    // ---------------- TMA producer: weight tile (+ activation tile) per stage
     if (lane == 0) {
       const CUtensorMap* map = &m0;
       int y = tile * kTileRows;
@@ -313,26 +344,53 @@ __global__ void __launch_bounds__(192, 2)
         const int tq = p.rows_q / kTileRows, tk = p.rows_k / kTileRows;
         if (tile >= tq + tk) { map = &m2; y = (tile - tq - tk) * kTileRows; }
         else if (tile >= tq) { map = &m1; y = (tile - tq) * kTileRows; }
+      } else if (gu) {
+        y = tile * kGuRows;
       }
       const uint64_t pol = l2_evict_first_policy();
-      int issued = 0;
-      for (int i = 0; i < nkb; ++i) {
+      const int nbox = p.n_pad / 16;
+      const uint32_t tx = abytes + (soft_b ? 0u : static_cast<uint32_t>(bbytes));
+      auto load_a = [&](int i) {
+        const int s = i % stages;
+        const int x = (kb0 + i) * kKBlock;
+        if (gu) {
+          tma_load_2d(sA + s * abytes, &m0, x, y, &full[s], pol);
+          tma_load_2d(sA + s * abytes + abytes / 2, &m1, x, y, &full[s], pol);
+        } else {
+          tma_load_2d(sA + s * abytes, map, x, y, &full[s], pol);
+        }
+      };
+      auto load_b = [&](int i) {
+        if (soft_b) return;
+        const int s = i % stages;
+        const int x = (kb0 + i) * kKBlock;
+        for (int b = 0; b < nbox; ++b)
+          tma_load_2d(sB + s * bbytes + b * 2048, &mb, x, p.act_row0 + b * 16, &full[s], 0ull);
+      };
+      // The first stages' weight tiles do not depend on earlier kernels.
+      const int pre = p.prefetch_a ? min(stages, nkb) : 0;
+      for (int i = 0; i < pre; ++i) {
+        mbar_arrive_expect_tx(&full[i], tx);
+        load_a(i);
+      }
+      griddep_wait();
+      for (int i = 0; i < pre; ++i) load_b(i);
+      int issued = pre;
+      for (int i = pre; i < nkb; ++i) {
         const int s = i % stages;
         const uint32_t ph = (i / stages) & 1;
         if (!mbar_wait(&empty[s], ph ^ 1, p.status)) break;
-        mbar_arrive_expect_tx(&full[s], abytes);
-        const int x = (kb0 + i) * kKBlock;
-        tma_load_2d(sA + s * abytes, map, x, y, &full[s], pol);
-        if (DUAL) tma_load_2d(sA + s * abytes + 16384, &m1, x, y, &full[s], pol);
+        mbar_arrive_expect_tx(&full[s], tx);
+        load_a(i);
+        load_b(i);
         issued = i + 1;
       }
-      // Drain: every issued copy has landed before this warp exits.
+      // Drain: every issued copy has landed before the CTA moves on.
       for (int i = max(0, issued - stages); i < issued; ++i)
         mbar_wait(&full[i % stages], (i / stages) & 1, p.status);
     }
-    return;
-  }
-  if (warp == 5) {
+    __syncwarp();
+  } else if (warp == 5) {
     // ---------------- MMA issuer
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_m128(static_cast<uint32_t>(p.n_pad));
@@ -344,48 +402,44 @@ __global__ void __launch_bounds__(192, 2)
         const uint32_t a = smem_u32(sA + s * abytes);
         const uint32_t b = smem_u32(sB + s * bbytes);
 #pragma unroll
-        for (int kk = 0; kk < kKBlock / 16; ++kk) {
-          const uint64_t bd = smem_desc_sw128(b + kk * 32);
-          const uint32_t acc = (i | kk) != 0;
-          tc_mma_bf16(tmem, smem_desc_sw128(a + kk * 32), bd, idesc, acc);
-          if (DUAL) tc_mma_bf16(tmem + static_cast<uint32_t>(p.n_pad), smem_desc_sw128(a + 16384 + kk * 32), bd,
-                                idesc, acc);
-        }
+        for (int kk = 0; kk < kKBlock / 16; ++kk)
+          tc_mma_bf16(tmem, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc, (i | kk) != 0);
         tc_commit(&empty[s]);
       }
       tc_commit(done);
     }
-    return;
-  }
-
-  // ---------------- warps 0-3: B producer, then epilogue
-  const int tid = threadIdx.x;
-  if (p.b_mode == B_NORM) compute_rstd(p, rstd, tid);
-  named_bar(1, kTileRows);
-  for (int i = 0; i < nkb; ++i) {
-    const int s = i % stages;
-    const uint32_t ph = (i / stages) & 1;
-    if (!mbar_wait(&empty[s], ph ^ 1, p.status)) break;
-    produce_b_tile(p, rstd, sB + s * bbytes, kb0 + i, tid);
-    fence_proxy_async_smem();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&full[s]);
-  }
-
-  const bool ok = mbar_wait(done, 0, p.status);
-  tc_fence_after();
-  const int row = tid;
-  const uint32_t lane_base = tmem + ((static_cast<uint32_t>(warp) * 32u) << 16);
-  const int nchunks = (p.M + kChunk - 1) / kChunk;
-  float v[kChunk], v2[kChunk];
-#pragma unroll
-  for (int j = 0; j < kChunk; ++j) v2[j] = 0.f;
-  using T = __nv_bfloat16;
-  if (p.n_splits == 1) {
+  } else {
+    // ---------------- warps 0-3: (B producer for f32 rows), norm scales, TMEM
+    const int tid = threadIdx.x;
+    griddep_wait();
+    if (soft_b) {
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % stages;
+        const uint32_t ph = (i / stages) & 1;
+        if (!mbar_wait(&empty[s], ph ^ 1, p.status)) break;
+        produce_b_f32(p, sB + s * bbytes, kb0 + i, tid);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&full[s]);
+      }
+    }
+    compute_rstd(p, rstd, tid, kTileRows);
+    named_bar(1, kTileRows);
+    ok = mbar_wait(done, 0, p.status);
+    tc_fence_after();
+    const uint32_t lane_base = tmem + ((static_cast<uint32_t>(warp) * 32u) << 16);
+    const int nchunks = (p.M + kChunk - 1) / kChunk;
+    float v[kChunk];
     for (int c = 0; c < nchunks; ++c) {
       tmem_ld16(lane_base + c * kChunk, v);
-      if (DUAL) tmem_ld16(lane_base + p.n_pad + c * kChunk, v2);
-      if (ok) epilogue_chunk<T>(p, tile, row, c * kChunk, v, v2, es);
+      if (p.n_splits == 1) {
+        if (ok) epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es);
+      } else {
+#pragma unroll
+        for (int j = 0; j < kChunk; ++j)
+          if (c * kChunk + j < p.M) part[(c * kChunk + j) * kTileRows + tid] = v[j];
+      }
     }
     tc_fence_before();
     named_bar(1, kTileRows);
@@ -393,62 +447,47 @@ __global__ void __launch_bounds__(192, 2)
       tc_fence_after();
       tmem_dealloc(tmem, ncols);
     }
-    return;
   }
-  const size_t reg = static_cast<size_t>(kTileRows) * p.n_pad * (DUAL ? 2 : 1);
-  float* mine = p.part + (static_cast<size_t>(tile) * p.n_splits + split) * reg;
-  for (int c = 0; c < nchunks; ++c) {
-    tmem_ld16(lane_base + c * kChunk, v);
-    if (DUAL) tmem_ld16(lane_base + p.n_pad + c * kChunk, v2);
+  if (p.n_splits > 1) {
+    // ---------------- split-K across the cluster: rank 0 sums the ranks' partials
+    cg::cluster_group cluster = cg::this_cluster();
+    cluster.sync();
+    if (split == 0 && warp < 4) {
+      const int tid = threadIdx.x;
+      const int nchunks = (p.M + kChunk - 1) / kChunk;
+      float v[kChunk];
+      for (int c = 0; c < nchunks; ++c) {
 #pragma unroll
-    for (int j = 0; j < kChunk; ++j) {
-      const int n = c * kChunk + j;
-      if (n < p.M) {
-        mine[static_cast<size_t>(n) * kTileRows + row] = v[j];
-        if (DUAL) mine[static_cast<size_t>(p.n_pad + n) * kTileRows + row] = v2[j];
-      }
-    }
-  }
-  tc_fence_before();
-  named_bar(1, kTileRows);
-  if (warp == 0) {
-    tc_fence_after();
-    tmem_dealloc(tmem, ncols);
-  }
-  if (!ok) return;
-  if (!split_arrive(p, tile, row, es)) return;
-  const float* all = p.part + static_cast<size_t>(tile) * p.n_splits * reg;
-  for (int c = 0; c < nchunks; ++c) {
+        for (int j = 0; j < kChunk; ++j) v[j] = 0.f;
+        for (int r = 0; r < p.n_splits; ++r) {
+          const float* peer = cluster.map_shared_rank(part, r);
 #pragma unroll
-    for (int j = 0; j < kChunk; ++j) {
-      const int n = c * kChunk + j;
-      float a = 0.f, b = 0.f;
-      if (n < p.M) {
-        for (int s = 0; s < p.n_splits; ++s) {
-          a += __ldcg(all + s * reg + static_cast<size_t>(n) * kTileRows + row);
-          if (DUAL) b += __ldcg(all + s * reg + static_cast<size_t>(p.n_pad + n) * kTileRows + row);
+          for (int j = 0; j < kChunk; ++j)
+            if (c * kChunk + j < p.M) v[j] += peer[(c * kChunk + j) * kTileRows + tid];
         }
+        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es);
       }
-      v[j] = a;
-      v2[j] = b;
     }
-    epilogue_chunk<T>(p, tile, row, c * kChunk, v, v2, es);
+    cluster.sync();   // peers keep their shared memory until rank 0 has read it
   }
 }
 
 // ------------------------------------------------------------------ FP32 FMA
-template <bool DUAL>
 __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
-  __shared__ float Ws[DUAL ? 2 : 1][kTileRows][kKBlockF32 + 1];
+  __shared__ float Ws[kTileRows][kKBlockF32 + 1];
   __shared__ float Bs[kChunk][kKBlockF32];
   __shared__ float rstd[kChunk];
   __shared__ EpiSmem es;
+  griddep_launch();
+  griddep_wait();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int tile = blockIdx.x / p.n_splits, split = blockIdx.x % p.n_splits;
   const int ttile = blockIdx.y, c0 = ttile * kChunk;
   const int kb0 = split * p.kb_per_split;
   const int nkb = min(p.kb_per_split, p.kb_total - kb0);
+  const bool gu = p.flavor == EPI_GATEUP;
 
+  // weight row of tile row r (nullptr = zero row)
   const float* w0 = static_cast<const float*>(p.w0);
   int row0 = tile * kTileRows, rows = p.n_out;
   if (p.flavor == EPI_QKV) {
@@ -457,95 +496,98 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
     else if (tile >= tq) { w0 = static_cast<const float*>(p.w1); row0 = (tile - tq) * kTileRows; rows = p.rows_k; }
     else rows = p.rows_q;
   }
-  const float* w1 = static_cast<const float*>(p.w1);
-  if (p.b_mode == B_NORM && tid < kChunk) {
+  auto wrow = [&](int r) -> const float* {
+    if (gu) {
+      const int f = tile * kGuRows + (r & (kGuRows - 1));
+      if (f >= p.n_out) return nullptr;
+      return static_cast<const float*>(r < kGuRows ? p.w0 : p.w1) + static_cast<size_t>(f) * p.K;
+    }
+    return row0 + r < rows ? w0 + static_cast<size_t>(row0 + r) * p.K : nullptr;
+  };
+  const float* act = static_cast<const float*>(p.act);
+  if (tid < kChunk) {
+    float r = 1.f;
     const int n = c0 + tid;
-    float s = 0.f;
-    if (n < p.M)
+    if (p.ss && n < p.M) {
+      float s = 0.f;
       for (int t = 0; t < p.ss_tiles; ++t) s += p.ss[static_cast<size_t>(t) * p.ss_ld + n];
-    rstd[tid] = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
+      r = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
+    }
+    rstd[tid] = r;
   }
   __syncthreads();
-  float acc[kChunk], acc2[kChunk];
+  float acc[kChunk];
 #pragma unroll
-  for (int j = 0; j < kChunk; ++j) { acc[j] = 0.f; acc2[j] = 0.f; }
+  for (int j = 0; j < kChunk; ++j) acc[j] = 0.f;
   for (int i = 0; i < nkb; ++i) {
     const int k = (kb0 + i) * kKBlockF32 + lane;
     for (int q = 0; q < kTileRows / 4; ++q) {
       const int r = warp + 4 * q;
-      const int grow = row0 + r;
-      const bool in = grow < rows && k < p.K;
-      Ws[0][r][lane] = in ? w0[static_cast<size_t>(grow) * p.K + k] : 0.f;
-      if (DUAL) Ws[DUAL ? 1 : 0][r][lane] = in ? w1[static_cast<size_t>(grow) * p.K + k] : 0.f;
+      const float* wr = wrow(r);
+      Ws[r][lane] = (wr && k < p.K) ? wr[k] : 0.f;
     }
     for (int e = 0; e < (kChunk * kKBlockF32) / 128; ++e) {
       const int idx = tid + 128 * e;
       const int j = idx / kKBlockF32, kk = idx % kKBlockF32;
       const int n = c0 + j, kg = (kb0 + i) * kKBlockF32 + kk;
-      float val = 0.f;
-      if (n < p.M && kg < p.K) {
-        if (p.b_mode == B_NORM) val = p.x[static_cast<size_t>(n) * p.ldx + kg] * rstd[j] * p.gain[kg];
-        else val = static_cast<const float*>(p.act)[static_cast<size_t>(n) * p.ld_act + kg];
-      }
-      Bs[j][kk] = val;
+      Bs[j][kk] = (n < p.M && kg < p.K) ? act[static_cast<size_t>(p.act_row0 + n) * p.ld_act + kg] : 0.f;
     }
     __syncthreads();
 #pragma unroll 8
     for (int kk = 0; kk < kKBlockF32; ++kk) {
-      const float w = Ws[0][tid][kk];
+      const float w = Ws[tid][kk];
 #pragma unroll
       for (int j = 0; j < kChunk; ++j) acc[j] = fmaf(w, Bs[j][kk], acc[j]);
-      if (DUAL) {
-        const float w2 = Ws[DUAL ? 1 : 0][tid][kk];
-#pragma unroll
-        for (int j = 0; j < kChunk; ++j) acc2[j] = fmaf(w2, Bs[j][kk], acc2[j]);
-      }
     }
     __syncthreads();
   }
   const int row = tid;
+  // epilogue_chunk indexes rstd by token; shift so rstd[c0 + j] is this tile's
+  float* rs = rstd - c0;
   if (p.n_splits == 1) {
-    epilogue_chunk<float>(p, tile, row, c0, acc, acc2, es);
+    epilogue_chunk<float>(p, tile, row, c0, acc, rs, es);
     return;
   }
-  const size_t reg = static_cast<size_t>(kTileRows) * kChunk * (DUAL ? 2 : 1);
+  const size_t reg = static_cast<size_t>(kTileRows) * kChunk;
   const int ci = tile * p.n_ttiles + ttile;
   float* mine = p.part + (static_cast<size_t>(ci) * p.n_splits + split) * reg;
 #pragma unroll
-  for (int j = 0; j < kChunk; ++j) {
-    mine[j * kTileRows + row] = acc[j];
-    if (DUAL) mine[(kChunk + j) * kTileRows + row] = acc2[j];
-  }
+  for (int j = 0; j < kChunk; ++j) mine[j * kTileRows + row] = acc[j];
   if (!split_arrive(p, ci, row, es)) return;
   const float* all = p.part + static_cast<size_t>(ci) * p.n_splits * reg;
 #pragma unroll
-  for (int j = 0; j < kChunk; ++j) {
-    float a = 0.f, b = 0.f;
-    for (int s = 0; s < p.n_splits; ++s) {
-      a += __ldcg(all + s * reg + j * kTileRows + row);
-      if (DUAL) b += __ldcg(all + s * reg + (kChunk + j) * kTileRows + row);
-    }
-    acc[j] = a;
-    acc2[j] = b;
-  }
-  epilogue_chunk<float>(p, tile, row, c0, acc, acc2, es);
+  for (int j = 0; j < kChunk; ++j) acc[j] = sum_splits(all + j * kTileRows + row, reg, p.n_splits);
+  epilogue_chunk<float>(p, tile, row, c0, acc, rs, es);
 }
 
 // ------------------------------------------------------------------ host
+// Work per launch: n_tiles output tiles x n_splits K ranges.  bf16: one wave
+// of at most two CTAs per SM (a third fits, which lets the next kernel's CTAs
+// start streaming weights under programmatic dependent launch), splits only
+// while tiles are too few, at most 8 (a portable cluster) and at least 4 K
+// blocks each.  f32: balanced waves of the FFMA kernel.
 void plan_splits(ProjArgs& a, int n_sms, bool tc) {
   if (a.flavor == EPI_QKV)
     a.n_tiles = a.rows_q / kTileRows + a.rows_k / kTileRows + a.rows_v / kTileRows;
+  else if (a.flavor == EPI_GATEUP)
+    a.n_tiles = (a.n_out + kGuRows - 1) / kGuRows;
   else
     a.n_tiles = (a.n_out + kTileRows - 1) / kTileRows;
   const int kbw = tc ? kKBlock : kKBlockF32;
   a.kb_total = (a.K + kbw - 1) / kbw;
-  const int slots = (tc ? 2 : 4) * n_sms;
-  const int min_kb = tc ? 4 : 2;
+  if (tc) {
+    int s = std::max(1, std::min(8, (2 * n_sms) / std::max(1, a.n_tiles)));
+    s = std::max(1, std::min(s, a.kb_total / 4));
+    a.kb_per_split = (a.kb_total + s - 1) / s;
+    a.n_splits = (a.kb_total + a.kb_per_split - 1) / a.kb_per_split;
+    return;
+  }
+  const int slots = 4 * n_sms;
   int best_s = 1, best_kbps = a.kb_total;
   double best_cost = 1e30;
   for (int s = 1; s <= 32 && s <= a.kb_total; ++s) {
     const int kbps = (a.kb_total + s - 1) / s;
-    if (s > 1 && kbps < min_kb) break;
+    if (s > 1 && kbps < 2) break;
     const int s_eff = (a.kb_total + kbps - 1) / kbps;
     const long units = static_cast<long>(a.n_tiles) * s_eff;
     const long waves = (units + slots - 1) / slots;
@@ -556,57 +598,61 @@ void plan_splits(ProjArgs& a, int n_sms, bool tc) {
   a.kb_per_split = best_kbps;
 }
 
+// Global split-K scratch (f32 path only; bf16 reduces inside the cluster).
 size_t proj_partial_floats(const ProjArgs& a, bool tc) {
-  if (a.n_splits <= 1) return 0;
-  const int dual = a.flavor == EPI_GATEUP ? 2 : 1;
-  const int ntt = tc ? 1 : (a.M + kChunk - 1) / kChunk;
-  const int cols = tc ? a.n_pad : kChunk;
-  return static_cast<size_t>(a.n_tiles) * ntt * a.n_splits * kTileRows * cols * dual;
+  if (tc || a.n_splits <= 1) return 0;
+  const int ntt = (a.M + kChunk - 1) / kChunk;
+  return static_cast<size_t>(a.n_tiles) * ntt * a.n_splits * kTileRows * kChunk;
 }
 
-static int tc_stages(int n_pad, bool dual, size_t* smem_bytes) {
-  const int per = (dual ? 32768 : 16384) + n_pad * 128;
-  const int fixed = 1024 /*align*/ + 1024 /*barriers, tmem slot, rstd*/ + 4 * kMaxTokens;
-  int stages = (112 * 1024 - fixed) / per;
-  if (stages < 3) stages = (220 * 1024 - fixed) / per;
-  stages = std::min(stages, 8);
-  stages = std::max(stages, 2);
+static int tc_stages(int n_pad, size_t* smem_bytes) {
+  const int per = 16384 + n_pad * 128;
+  const int fixed = 1024 /*align*/ + 1024 /*barriers, tmem slot*/ + 4 * kMaxTokens /*rstd*/;
+  int stages = n_pad <= 64 ? 4 : std::max(2, std::min(8, (112 * 1024 - fixed) / per));
   *smem_bytes = static_cast<size_t>(fixed) + static_cast<size_t>(stages) * per;
   return stages;
 }
 
-cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s) {
-  if (a.dtype == DVI_BF16) {
-    const bool dual = a.flavor == EPI_GATEUP;
-    size_t smem = 0;
-    const int stages = tc_stages(a.n_pad, dual, &smem);
-    dim3 grid(a.n_tiles * a.n_splits);
-    if (dual) {
-      static bool attr = false;
-      if (!attr) {
-        cudaFuncSetAttribute(proj_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-        attr = true;
-      }
-      proj_tc_kernel<true><<<grid, 192, smem, s>>>(maps->m0, maps->m1, maps->m2, a, stages);
-    } else {
-      static bool attr = false;
-      if (!attr) {
-        cudaFuncSetAttribute(proj_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-        attr = true;
-      }
-      proj_tc_kernel<false><<<grid, 192, smem, s>>>(maps->m0, maps->m1, maps->m2, a, stages);
+cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s) {
+  cudaError_t e;
+  if (a0.dtype == DVI_BF16) {
+    static bool attr = false;
+    if (!attr) {
+      cudaFuncSetAttribute(proj_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      attr = true;
     }
+    ProjArgs a = a0;
+    // the cluster reduction keeps a [n_pad][128] partial in the A stages
+    if (a.n_pad > 64 && a.n_splits > 1) {
+      a.n_splits = 1;
+      a.kb_per_split = a.kb_total;
+    }
+    size_t smem = 0;
+    const int stages = tc_stages(a.n_pad, &smem);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.n_tiles * a.n_splits);
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = a.n_splits;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = a.n_splits > 1 ? 2 : 1;
+    e = cudaLaunchKernelEx(&cfg, proj_tc_kernel, maps->m0, maps->m1, maps->m2, maps->mb, a, stages);
   } else {
-    ProjArgs b = a;
-    b.n_ttiles = (a.M + kChunk - 1) / kChunk;
-    dim3 grid(a.n_tiles * a.n_splits, b.n_ttiles);
-    if (a.flavor == EPI_GATEUP) proj_f32_kernel<true><<<grid, 128, 0, s>>>(b);
-    else proj_f32_kernel<false><<<grid, 128, 0, s>>>(b);
+    ProjArgs b = a0;
+    b.n_ttiles = (a0.M + kChunk - 1) / kChunk;
+    e = launch_pdl(proj_f32_kernel, dim3(a0.n_tiles * a0.n_splits, b.n_ttiles), dim3(128), 0, s, b);
   }
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
+static PFN_cuTensorMapEncodeTiled_v12000 encoder() {
   static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
   if (!encode) {
     void* fn = nullptr;
@@ -614,17 +660,33 @@ bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
             cudaSuccess ||
         q != cudaDriverEntryPointSuccess || !fn)
-      return false;
+      return nullptr;
     encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }
+  return encode;
+}
+
+static bool make_map(CUtensorMap* map, const void* ptr, int rows, int cols, int box_rows) {
+  auto encode = encoder();
+  if (!encode) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
-  cuuint32_t box[2] = {kKBlock, kTileRows};
+  cuuint32_t box[2] = {kKBlock, static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
-  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(w), dims, strides, box,
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
                             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
+  return make_map(map, w, rows, cols, kTileRows);
+}
+bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
+  return make_map(map, w, rows, cols, kGuRows);
+}
+bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols) {
+  return make_map(map, act, rows, cols, 16);
 }
 
 }  // namespace dvi

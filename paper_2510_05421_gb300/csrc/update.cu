@@ -39,6 +39,8 @@ __device__ __forceinline__ bool row_valid(const UpdateArgs& a, int n) { return a
 
 template <typename T>
 __global__ void __launch_bounds__(128) update_prep_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   const int n = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (!row_valid(a, n)) {
@@ -67,6 +69,8 @@ __device__ float block_reduce(float v, float* red, bool is_max) {
 }
 
 __global__ void __launch_bounds__(256) update_rowstats_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   __shared__ float red[8];
   const int n = blockIdx.x;
   float* rs = a.rowstat + n * RS_N;
@@ -150,6 +154,8 @@ __device__ TermW term_weights(const dvi_update_config& c, int t) {
 }
 
 __global__ void update_coef_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   if (threadIdx.x != 0) return;
   const int t = static_cast<int>(a.dev_state[DS_T]);
   const float b = a.dev_state[DS_B];
@@ -221,6 +227,8 @@ __device__ __forceinline__ void opt_step(const dvi_update_config& c, float step,
 
 // grid = ceil(V/128); dynamic smem: G tile [cap][128] + A tile [128][r]
 __global__ void __launch_bounds__(128) update_grad_a_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   extern __shared__ float sm[];
   if (a.dev_state[DS_SKIP] != 0.f) return;
   float* Gs = sm;                              // [cap][128]
@@ -277,6 +285,8 @@ __global__ void __launch_bounds__(128) update_grad_a_kernel(const UpdateArgs a) 
 }
 
 __global__ void update_ga_reduce_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   if (a.dev_state[DS_SKIP] != 0.f) return;
   const int n = blockIdx.x, j = threadIdx.x;
   if (j >= a.r) return;
@@ -287,6 +297,8 @@ __global__ void update_ga_reduce_kernel(const UpdateArgs a) {
 
 template <typename T>
 __global__ void __launch_bounds__(128) update_grad_b_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   if (a.dev_state[DS_SKIP] != 0.f) return;
   const int c = blockIdx.x * 128 + threadIdx.x;
   if (c >= a.d) return;
@@ -306,6 +318,8 @@ __global__ void __launch_bounds__(128) update_grad_b_kernel(const UpdateArgs a) 
 }
 
 __global__ void update_finish_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
   for (int n = blockIdx.x * blockDim.x + threadIdx.x; n < a.cap; n += gridDim.x * blockDim.x) a.log_meta[n * 6] = 0;
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     a.dev_state[DS_T] += 1.f;
@@ -316,16 +330,19 @@ __global__ void update_finish_kernel(const UpdateArgs a) {
 
 cudaError_t launch_update_prep(const UpdateArgs& a, cudaStream_t s) {
   if (a.r == 0) return cudaSuccess;
-  if (a.dtype == DVI_BF16) update_prep_kernel<__nv_bfloat16><<<a.cap, 128, 0, s>>>(a);
-  else update_prep_kernel<float><<<a.cap, 128, 0, s>>>(a);
+  const cudaError_t e = a.dtype == DVI_BF16 ? launch_pdl(update_prep_kernel<__nv_bfloat16>, dim3(a.cap), dim3(128), 0, s, a)
+                                            : launch_pdl(update_prep_kernel<float>, dim3(a.cap), dim3(128), 0, s, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 cudaError_t launch_update_rowstats(const UpdateArgs& a, cudaStream_t s) {
-  update_rowstats_kernel<<<a.cap, 256, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(update_rowstats_kernel, dim3(a.cap), dim3(256), 0, s, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 cudaError_t launch_update_coef(const UpdateArgs& a, cudaStream_t s) {
-  update_coef_kernel<<<1, 32, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(update_coef_kernel, dim3(1), dim3(32), 0, s, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s) {
@@ -336,18 +353,22 @@ cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s) {
     cudaFuncSetAttribute(update_grad_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     attr = smem;
   }
-  update_grad_a_kernel<<<a.n_vtiles, 128, smem, s>>>(a);
+  const cudaError_t e = launch_pdl(update_grad_a_kernel, dim3(a.n_vtiles), dim3(128), smem, s, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s) {
   if (a.r == 0) return cudaSuccess;
-  update_ga_reduce_kernel<<<a.cap, 64, 0, s>>>(a);
-  if (a.dtype == DVI_BF16) update_grad_b_kernel<__nv_bfloat16><<<(a.d + 127) / 128, 128, 0, s>>>(a);
-  else update_grad_b_kernel<float><<<(a.d + 127) / 128, 128, 0, s>>>(a);
+  cudaError_t e = launch_pdl(update_ga_reduce_kernel, dim3(a.cap), dim3(64), 0, s, a);
+  if (e != cudaSuccess) return e;
+  e = a.dtype == DVI_BF16 ? launch_pdl(update_grad_b_kernel<__nv_bfloat16>, dim3((a.d + 127) / 128), dim3(128), 0, s, a)
+                          : launch_pdl(update_grad_b_kernel<float>, dim3((a.d + 127) / 128), dim3(128), 0, s, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 cudaError_t launch_update_finish(const UpdateArgs& a, cudaStream_t s) {
-  update_finish_kernel<<<(a.cap + 255) / 256, 256, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(update_finish_kernel, dim3((a.cap + 255) / 256), dim3(256), 0, s, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -40,8 +40,9 @@ def test_noalloc_matches_linear_twice(dtype, tol):
 
 def test_noalloc_rejects_shapes_beyond_its_scratch():
     from paper_2510_05421_gb300.dvi import linear_noalloc
-    # 32 tiles x 9 K-splits x 128 x 256 partial sums > the 2^21-float scratch
-    w = torch.zeros(4096, 11008, dtype=torch.bfloat16, device="cuda")
+    # f32 path: 32 tiles x 16 row tiles x several K-splits x 128 x 16 partial
+    # sums > the 2^21-float scratch
+    w = torch.zeros(4096, 11008, dtype=torch.float32, device="cuda")
     x = torch.zeros(256, 11008, dtype=torch.float32, device="cuda")
     y = torch.zeros(256, 4096, dtype=torch.float32, device="cuda")
     assert linear_noalloc(w, x, y) == -2
