@@ -15,13 +15,15 @@
 // rule, and positions a row must not see contribute exact zeros, so a row's
 // output does not depend on how many rows share the launch.
 //
-// Decode (<= 16 rows per sequence): attn_reg_kernel keeps a query group's
+// Decode (<= 16 rows per sequence): attn_dec_kernel streams the split's K/V
+// through a shared-memory ring by bulk copies and keeps a query group's
 // vectors, scores and accumulators in registers; each warp walks its
-// positions four at a time (lane = hd/32 dims, 8-byte coalesced K/V loads),
-// reduces the dot products with shuffles and runs an online softmax; the four
-// warps merge through shared memory at the end.
+// positions four at a time (lane = hd/32 dims), reduces the dot products
+// with shuffles and runs an online softmax; the four warps merge through
+// shared memory at the end.
 // Prefill chunks: attn_smem_kernel stages 64-position K/V blocks in shared
 // memory for 16 queries at a time.
+#include <algorithm>
 #include <cmath>
 
 #include "common.cuh"
@@ -67,13 +69,17 @@ __device__ __forceinline__ void load_n<float, 8>(const float* src, float* dst) {
   dst[0] = a.x; dst[1] = a.y; dst[2] = a.z; dst[3] = a.w; dst[4] = b.x; dst[5] = b.y; dst[6] = b.z; dst[7] = b.w;
 }
 
-// Decode launches (<= 16 rows per sequence, GQA group <= 8) use the register
-// kernel with 8 query vectors per CTA; others the shared-memory kernel with 16.
+// Decode launches (<= 16 rows per sequence, GQA group <= 8): bf16 caches use
+// the tensor-core kernel (16 query vectors per CTA), f32 caches the CUDA-core
+// kernel (8); prefill chunks the shared-memory kernel (16).
 static __host__ __device__ inline bool use_reg_kernel(int rows_per_seq, int G) {
   return rows_per_seq <= 16 && G <= kRegQ;
 }
-static __host__ __device__ inline int rows_per_group(int rows_per_seq, int G) {
-  return (use_reg_kernel(rows_per_seq, G) ? kRegQ : kAttnQ) / G;
+// Query rows per CTA; scratch is sized with the f32 decode grouping, the
+// largest number of groups any kernel uses.
+static __host__ __device__ inline int rows_per_group(int rows_per_seq, int G, bool bf16) {
+  if (!use_reg_kernel(rows_per_seq, G)) return kAttnQ / G;
+  return (bf16 ? kAttnQ : kRegQ) / G;
 }
 
 // Combine of the splits of one (sequence, group, head): the CTA that finishes
@@ -107,15 +113,34 @@ __device__ void combine_splits(const AttnArgs& a, const float* all, size_t per, 
 }
 
 // ------------------------------------------------------------------ decode
-template <typename T, typename TO, int DPL>
-__global__ void __launch_bounds__(128) attn_reg_kernel(const AttnArgs a) {
+// K/V of the CTA's positions stream through a ring of kDecStages shared-memory
+// stages in 64-position chunks (one 1D bulk copy each for K and V: the rows of
+// one (sequence, KV head) are contiguous).  The four warps split the work as
+// WQ query pairs x WP position slices (WQ*WP = 4): warp (wq, wp) handles
+// queries 2wq, 2wq+1 on positions of slice wp of every chunk, four at a time;
+// a lane holds hd/32 dims of its two queries.  Scores are kept in base 2
+// (log2 e folded into the query scale) so the softmax uses exp2.
+constexpr int kDecStages = 2;
+constexpr int kChunkPos = 64;
+constexpr int kQPW = 2;                 // query vectors per warp
+constexpr float kLog2e = 1.4426950408889634f;
+
+template <typename T, int DPL>
+__global__ void __launch_bounds__(128) attn_dec_kernel(const AttnArgs a, int wq_count) {
   constexpr int HD = 32 * DPL;
-  __shared__ float wm[4][kRegQ], wl[4][kRegQ];
-  __shared__ float wacc[4][kRegQ][HD];
+  constexpr int kRowBytes = HD * sizeof(T);
+  constexpr int kStageBytes = kChunkPos * kRowBytes;   // one of K or V
+  extern __shared__ __align__(128) uint8_t dsm[];
+  __shared__ __align__(8) uint64_t full[kDecStages];
+  __shared__ float wm[4][kQPW], wl[4][kQPW];
+  __shared__ float wacc[4][kQPW][HD];
   __shared__ int flag;
+  uint8_t* ring = dsm;    // [stage][K | V][64][HD]
   griddep_launch();
   griddep_wait();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int WQ = wq_count, WP = 4 / wq_count;
+  const int wq = warp % WQ, wp = warp / WQ;
   const int G = a.n_heads / a.n_kv_heads;
   const int RQ = kRegQ / G;
   const int n_qg = (a.rows_per_seq + RQ - 1) / RQ;
@@ -131,92 +156,386 @@ __global__ void __launch_bounds__(128) attn_reg_kernel(const AttnArgs a) {
   if (p0 >= t_cta) return;
   const int p1 = min(p0 + a.split_len, t_cta);
   const int n_active = (t_cta + a.split_len - 1) / a.split_len;
+  const int nch = (p1 - p0 + kChunkPos - 1) / kChunkPos;
 
-  float q[kRegQ][DPL];
-  int lim[kRegQ];
+  const size_t head_off = (static_cast<size_t>(seq) * a.n_kv_heads + g) * a.max_len * HD;
+  const T* kb = static_cast<const T*>(a.kc) + head_off;
+  const T* vb = static_cast<const T*>(a.vc) + head_off;
+  auto issue = [&](int ch) {
+    const int st = ch % kDecStages;
+    const int pc = p0 + ch * kChunkPos;
+    const uint32_t bytes = static_cast<uint32_t>(min(kChunkPos, p1 - pc)) * kRowBytes;
+    mbar_arrive_expect_tx(&full[st], 2 * bytes);
+    bulk_load(ring + st * 2 * kStageBytes, kb + static_cast<size_t>(pc) * HD, bytes, &full[st]);
+    bulk_load(ring + st * 2 * kStageBytes + kStageBytes, vb + static_cast<size_t>(pc) * HD, bytes, &full[st]);
+  };
+  if (tid == 0) {
+    for (int st = 0; st < kDecStages; ++st) mbar_init(&full[st], 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  if (tid == 0)
+    for (int ch = 0; ch < min(kDecStages, nch); ++ch) issue(ch);
+
+  float q[kQPW][DPL], m[kQPW], l[kQPW], acc[kQPW][DPL];
+  int lim[kQPW];
 #pragma unroll
-  for (int qi = 0; qi < kRegQ; ++qi) {
-    lim[qi] = -1;
+  for (int u = 0; u < kQPW; ++u) {
+    const int qi = wq * kQPW + u;
+    lim[u] = -1;
+    m[u] = -INFINITY;
+    l[u] = 0.f;
 #pragma unroll
-    for (int e = 0; e < DPL; ++e) q[qi][e] = 0.f;
+    for (int e = 0; e < DPL; ++e) {
+      q[u][e] = 0.f;
+      acc[u][e] = 0.f;
+    }
     if (qi < Q) {
       const int ii = qi / G, hh = qi % G;
       const int n = sl * a.rows_per_seq + i0 + ii;
       const float* src = a.q + static_cast<size_t>(n) * a.ld_q + (g * G + hh) * HD + lane * DPL;
 #pragma unroll
-      for (int e = 0; e < DPL; ++e) q[qi][e] = src[e] * a.scale;
-      lim[qi] = base + i0 + ii;          // last position row ii may see
+      for (int e = 0; e < DPL; ++e) q[u][e] = src[e] * (a.scale * kLog2e);
+      lim[u] = base + i0 + ii;            // last position row ii may see
     }
   }
-  float m[kRegQ], l[kRegQ], acc[kRegQ][DPL];
-#pragma unroll
-  for (int qi = 0; qi < kRegQ; ++qi) {
-    m[qi] = -INFINITY;
-    l[qi] = 0.f;
-#pragma unroll
-    for (int e = 0; e < DPL; ++e) acc[qi][e] = 0.f;
-  }
-  const size_t head_off = (static_cast<size_t>(seq) * a.n_kv_heads + g) * a.max_len * HD + lane * DPL;
-  const T* kb = static_cast<const T*>(a.kc) + head_off;
-  const T* vb = static_cast<const T*>(a.vc) + head_off;
+  const bool active = wq * kQPW < Q;      // warp-uniform
+  const int slice = kChunkPos / WP;
 
-  for (int gp = p0 + warp * kRegPos; gp < p1; gp += 4 * kRegPos) {
-    float kr[kRegPos][DPL], vr[kRegPos][DPL];
+  for (int ch = 0; ch < nch; ++ch) {
+    const int st = ch % kDecStages;
+    // a wait that runs out only flags the status: every warp must still reach
+    // the block barrier below
+    mbar_wait(&full[st], (ch / kDecStages) & 1, a.status);
+    const T* ks = reinterpret_cast<const T*>(ring + st * 2 * kStageBytes);
+    const T* vs = reinterpret_cast<const T*>(ring + st * 2 * kStageBytes + kStageBytes);
+    const int pc = p0 + ch * kChunkPos;
+    if (active) {
+      for (int o0 = wp * slice; o0 < (wp + 1) * slice; o0 += kRegPos) {
+        float kr[kRegPos][DPL], vr[kRegPos][DPL];
 #pragma unroll
-    for (int j = 0; j < kRegPos; ++j) {
-      if (gp + j < p1) {
-        load_n<T, DPL>(kb + static_cast<size_t>(gp + j) * HD, kr[j]);
-        load_n<T, DPL>(vb + static_cast<size_t>(gp + j) * HD, vr[j]);
-      } else {
+        for (int j = 0; j < kRegPos; ++j) {
+          if (pc + o0 + j < p1) {
+            load_n<T, DPL>(ks + (o0 + j) * HD + lane * DPL, kr[j]);
+            load_n<T, DPL>(vs + (o0 + j) * HD + lane * DPL, vr[j]);
+          } else {
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) { kr[j][e] = 0.f; vr[j][e] = 0.f; }
-      }
-    }
-    float s[kRegPos][kRegQ];
+            for (int e = 0; e < DPL; ++e) { kr[j][e] = 0.f; vr[j][e] = 0.f; }
+          }
+        }
+        float sc[kRegPos][kQPW];
 #pragma unroll
-    for (int j = 0; j < kRegPos; ++j)
+        for (int j = 0; j < kRegPos; ++j)
 #pragma unroll
-      for (int qi = 0; qi < kRegQ; ++qi) {
-        s[j][qi] = -INFINITY;
-        if (qi < Q) {                       // warp-uniform
-          float t = 0.f;
+          for (int u = 0; u < kQPW; ++u) {
+            float t = 0.f;
 #pragma unroll
-          for (int e = 0; e < DPL; ++e) t = fmaf(q[qi][e], kr[j][e], t);
-          t = warp_sum(t);
-          if (gp + j < p1 && gp + j <= lim[qi]) s[j][qi] = t;
+            for (int e = 0; e < DPL; ++e) t = fmaf(q[u][e], kr[j][e], t);
+            t = warp_sum(t);
+            const int pos = pc + o0 + j;
+            sc[j][u] = (pos < p1 && pos <= lim[u]) ? t : -INFINITY;
+          }
+#pragma unroll
+        for (int u = 0; u < kQPW; ++u) {
+          float bm = sc[0][u];
+#pragma unroll
+          for (int j = 1; j < kRegPos; ++j) bm = fmaxf(bm, sc[j][u]);
+          if (bm == -INFINITY) continue;      // nothing this row may see here
+          const float mn = fmaxf(m[u], bm);
+          const float c = (m[u] == -INFINITY) ? 0.f : exp2f(m[u] - mn);
+          l[u] *= c;
+#pragma unroll
+          for (int e = 0; e < DPL; ++e) acc[u][e] *= c;
+#pragma unroll
+          for (int j = 0; j < kRegPos; ++j) {
+            const float pj = exp2f(sc[j][u] - mn);
+            l[u] += pj;
+#pragma unroll
+            for (int e = 0; e < DPL; ++e) acc[u][e] = fmaf(pj, vr[j][e], acc[u][e]);
+          }
+          m[u] = mn;
         }
       }
+    }
+    __syncthreads();                      // stage `st` consumed by every warp
+    if (tid == 0 && ch + kDecStages < nch) issue(ch + kDecStages);
+  }
+  // merge the position slices of each query
 #pragma unroll
-    for (int qi = 0; qi < kRegQ; ++qi) {
-      if (qi >= Q) continue;
-      float bm = s[0][qi];
+  for (int u = 0; u < kQPW; ++u) {
+    if (lane == 0) {
+      wm[warp][u] = m[u];
+      wl[warp][u] = l[u];
+    }
 #pragma unroll
-      for (int j = 1; j < kRegPos; ++j) bm = fmaxf(bm, s[j][qi]);
-      if (bm == -INFINITY) continue;      // nothing this row may see here
-      const float mn = fmaxf(m[qi], bm);
-      const float c = (m[qi] == -INFINITY) ? 0.f : expf(m[qi] - mn);
-      l[qi] *= c;
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) acc[qi][e] *= c;
-#pragma unroll
-      for (int j = 0; j < kRegPos; ++j) {
-        const float pj = expf(s[j][qi] - mn);
-        l[qi] += pj;
-#pragma unroll
-        for (int e = 0; e < DPL; ++e) acc[qi][e] = fmaf(pj, vr[j][e], acc[qi][e]);
+    for (int e = 0; e < DPL; ++e) wacc[warp][u][lane * DPL + e] = acc[u][e];
+  }
+  __syncthreads();
+  const int hq_base = g * G;
+  const int slot = (sl * n_qg + qg) * a.n_kv_heads + g;
+  const size_t per = static_cast<size_t>(kAttnQ) * (HD + 2);
+  float* mine = a.part + (static_cast<size_t>(slot) * a.n_splits_max + split) * per;
+  for (int idx = tid; idx < Q * HD; idx += 128) {
+    const int qi = idx / HD, d = idx % HD;
+    const int w0 = qi / kQPW, u = qi % kQPW;           // warps w0 + WQ*p hold query qi
+    float M = -INFINITY;
+    for (int p = 0; p < WP; ++p) M = fmaxf(M, wm[w0 + WQ * p][u]);
+    float Ls = 0.f, O = 0.f;
+    for (int p = 0; p < WP; ++p) {
+      const float mw = wm[w0 + WQ * p][u];
+      const float ww = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+      Ls = fmaf(wl[w0 + WQ * p][u], ww, Ls);
+      O = fmaf(wacc[w0 + WQ * p][u][d], ww, O);
+    }
+    if (n_active == 1) {
+      const int ii = qi / G, hh = qi % G;
+      const int n = sl * a.rows_per_seq + i0 + ii;
+      DT<T>::st(static_cast<T*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, O / Ls);
+    } else {
+      mine[qi * HD + d] = O;
+      if (d == 0) {
+        mine[kAttnQ * HD + qi] = M;
+        mine[kAttnQ * HD + kAttnQ + qi] = Ls;
       }
-      m[qi] = mn;
     }
   }
-  // merge the four warps
-#pragma unroll
-  for (int qi = 0; qi < kRegQ; ++qi) {
-    if (lane == 0) {
-      wm[warp][qi] = m[qi];
-      wl[warp][qi] = l[qi];
+  if (n_active == 1) return;
+  if (!split_combine_arrive(a, slot, n_active, &flag)) return;
+  // combine the splits in split order (maxima in base 2)
+  const float* all = a.part + static_cast<size_t>(slot) * a.n_splits_max * per;
+  __shared__ float cw[kAttnQ];      // 1 / sum of weights, per query
+  __shared__ float cM[kAttnQ];
+  if (tid < Q) {
+    float M = -INFINITY;
+    for (int s2 = 0; s2 < n_active; ++s2) M = fmaxf(M, __ldcg(all + s2 * per + kAttnQ * HD + tid));
+    float Ls = 0.f;
+    for (int s2 = 0; s2 < n_active; ++s2) {
+      const float ms = __ldcg(all + s2 * per + kAttnQ * HD + tid);
+      Ls = fmaf(__ldcg(all + s2 * per + kAttnQ * HD + kAttnQ + tid), ms == -INFINITY ? 0.f : exp2f(ms - M), Ls);
+    }
+    cM[tid] = M;
+    cw[tid] = 1.f / Ls;
+  }
+  __syncthreads();
+  for (int idx = tid; idx < Q * HD; idx += 128) {
+    const int qi = idx / HD, d = idx % HD;
+    float O = 0.f;
+    for (int s2 = 0; s2 < n_active; ++s2) {
+      const float ms = __ldcg(all + s2 * per + kAttnQ * HD + qi);
+      O = fmaf(__ldcg(all + s2 * per + qi * HD + d), ms == -INFINITY ? 0.f : exp2f(ms - cM[qi]), O);
+    }
+    const int ii = qi / G, hh = qi % G;
+    const int n = sl * a.rows_per_seq + i0 + ii;
+    DT<T>::st(static_cast<T*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, O * cw[qi]);
+  }
+}
+
+// ------------------------------------------------------------------ decode, bf16
+// Tensor-core decode attention (bf16 cache).  A CTA covers 16 query rows (the
+// block's rows x the GQA heads of one KV head, zero-padded) and its split's
+// positions in 64-position chunks, double-buffered by TMA (128-byte swizzle,
+// so the fragment loads below are bank-conflict free).  Warp w owns chunk
+// positions 16w..16w+15: S = Q K^T with mma.m16n8k16 (Q fragments held in
+// registers, K as the column-major operand read straight from the swizzled
+// rows), an online softmax over its columns in base 2, then O += P V with the
+// accumulator fragments of S reused as the A operand and V fragments loaded
+// transposed by ldmatrix.  The four warps merge at the end.
+constexpr int kMmaQ = 16;
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ CUtensorMap mk,
+                                                       const __grid_constant__ CUtensorMap mv, const AttnArgs a) {
+  constexpr int kBoxes = HD / 64;                    // 64-dim TMA boxes per row
+  constexpr int kBoxBytes = 64 * 128;                // 64 positions x 128 B
+  constexpr int kStage = 2 * kBoxes * kBoxBytes;     // K boxes, then V boxes
+  constexpr int kNT = HD / 8;                        // O n-tiles
+  extern __shared__ __align__(1024) uint8_t dsm_raw[];
+  __shared__ __align__(8) uint64_t full[kDecStages];
+  __shared__ float wm[4][kMmaQ], wl[4][kMmaQ];
+  __shared__ int flag;
+  __shared__ float cw[kMmaQ], cM[kMmaQ];
+  const uint32_t raw = smem_u32(dsm_raw);
+  uint8_t* ring = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+  griddep_launch();
+  griddep_wait();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int gq = lane >> 2, tq = lane & 3;           // mma fragment coordinates
+  const int G = a.n_heads / a.n_kv_heads;
+  const int RQ = kMmaQ / G;
+  const int n_qg = (a.rows_per_seq + RQ - 1) / RQ;
+  const int split = blockIdx.x, g = blockIdx.y;
+  const int sl = blockIdx.z / n_qg, qg = blockIdx.z % n_qg;
+  const int seq = a.seq0 + sl;
+  const int i0 = qg * RQ;
+  const int nrows = min(RQ, a.rows_per_seq - i0);
+  const int Q = nrows * G;
+  const int base = a.lens[seq] + a.pos_off;
+  const int t_cta = min(base + i0 + nrows, a.max_len);
+  const int p0 = split * a.split_len;
+  if (p0 >= t_cta) return;
+  const int p1 = min(p0 + a.split_len, t_cta);
+  const int n_active = (t_cta + a.split_len - 1) / a.split_len;
+  const int nch = (p1 - p0 + kChunkPos - 1) / kChunkPos;
+  const int row0 = static_cast<int>(a.kv_row0 + (static_cast<long long>(seq) * a.n_kv_heads + g) * a.max_len);
+
+  auto issue = [&](int ch) {
+    const int st = ch % kDecStages;
+    const int y = row0 + p0 + ch * kChunkPos;
+    mbar_arrive_expect_tx(&full[st], kStage);
+    for (int b = 0; b < kBoxes; ++b) {
+      tma_load_2d(ring + st * kStage + b * kBoxBytes, &mk, b * 64, y, &full[st], 0ull);
+      tma_load_2d(ring + st * kStage + (kBoxes + b) * kBoxBytes, &mv, b * 64, y, &full[st], 0ull);
+    }
+  };
+  if (tid == 0) {
+    for (int st = 0; st < kDecStages; ++st) mbar_init(&full[st], 1);
+    mbar_fence_init();
+    tma_prefetch_desc(&mk);
+    tma_prefetch_desc(&mv);
+  }
+  __syncthreads();
+  if (tid == 0)
+    for (int ch = 0; ch < min(kDecStages, nch); ++ch) issue(ch);
+
+  // Q fragments (rows gq and gq+8), scaled by 1/sqrt(hd) * log2(e), bf16
+  uint32_t qa[HD / 16][4];
+  int lim0 = -1, lim1 = -1;
+  {
+    const float sc = a.scale * kLog2e;
+    const float* qrow[2] = {nullptr, nullptr};
+    for (int h = 0; h < 2; ++h) {
+      const int qi = gq + 8 * h;
+      if (qi < Q) {
+        const int ii = qi / G, hh = qi % G;
+        const int n = sl * a.rows_per_seq + i0 + ii;
+        qrow[h] = a.q + static_cast<size_t>(n) * a.ld_q + (g * G + hh) * HD;
+        if (h == 0) lim0 = base + i0 + ii;
+        else lim1 = base + i0 + ii;
+      }
     }
 #pragma unroll
-    for (int e = 0; e < DPL; ++e) wacc[warp][qi][lane * DPL + e] = acc[qi][e];
+    for (int kk = 0; kk < HD / 16; ++kk) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const float* qr = qrow[r & 1];
+        const int col = kk * 16 + (r >> 1) * 8 + 2 * tq;
+        qa[kk][r] = qr ? pack_bf16x2(qr[col] * sc, qr[col + 1] * sc) : 0u;
+      }
+    }
+  }
+  float o[kNT][4];
+#pragma unroll
+  for (int nt = 0; nt < kNT; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o[nt][e] = 0.f;
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+
+  for (int ch = 0; ch < nch; ++ch) {
+    const int st = ch % kDecStages;
+    mbar_wait(&full[st], (ch / kDecStages) & 1, a.status);
+    const uint8_t* ks = ring + st * kStage;
+    const uint8_t* vs = ks + kBoxes * kBoxBytes;
+    const int pc = p0 + ch * kChunkPos;
+    // S = Q K^T for this warp's 16 positions (two n-tiles of 8)
+    float sacc[2][4];
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) sacc[nt][e] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      const int box = (kk * 16) / 64, c = ((kk * 16) % 64) / 8;
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        const int pr = warp * 16 + nt * 8 + gq;                   // row of the chunk
+        const uint8_t* rowp = ks + box * kBoxBytes + pr * 128;
+        const uint32_t b0 = *reinterpret_cast<const uint32_t*>(rowp + ((c ^ (pr & 7)) << 4) + 4 * tq);
+        const uint32_t b1 = *reinterpret_cast<const uint32_t*>(rowp + (((c + 1) ^ (pr & 7)) << 4) + 4 * tq);
+        mma_bf16_16816(sacc[nt], qa[kk], b0, b1);
+      }
+    }
+    // mask, online softmax (rows gq and gq+8; columns spread over the 4 lanes tq)
+    float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int pos = pc + warp * 16 + nt * 8 + 2 * tq + e;
+        if (!(pos < p1 && pos <= lim0)) sacc[nt][e] = -INFINITY;
+        if (!(pos < p1 && pos <= lim1)) sacc[nt][2 + e] = -INFINITY;
+        mx0 = fmaxf(mx0, sacc[nt][e]);
+        mx1 = fmaxf(mx1, sacc[nt][2 + e]);
+      }
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+    // a row with nothing visible so far keeps its state untouched
+    const float c0 = (mn0 == -INFINITY) ? 1.f : (m0 == -INFINITY ? 0.f : exp2f(m0 - mn0));
+    const float c1 = (mn1 == -INFINITY) ? 1.f : (m1 == -INFINITY ? 0.f : exp2f(m1 - mn1));
+    uint32_t pa[4];
+    {
+      float pv[2][4];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          pv[nt][e] = (sacc[nt][e] == -INFINITY) ? 0.f : exp2f(sacc[nt][e] - mn0);
+          pv[nt][2 + e] = (sacc[nt][2 + e] == -INFINITY) ? 0.f : exp2f(sacc[nt][2 + e] - mn1);
+        }
+      l0 = l0 * c0 + ((pv[0][0] + pv[0][1]) + (pv[1][0] + pv[1][1]));
+      l1 = l1 * c1 + ((pv[0][2] + pv[0][3]) + (pv[1][2] + pv[1][3]));
+      pa[0] = pack_bf16x2(pv[0][0], pv[0][1]);
+      pa[1] = pack_bf16x2(pv[0][2], pv[0][3]);
+      pa[2] = pack_bf16x2(pv[1][0], pv[1][1]);
+      pa[3] = pack_bf16x2(pv[1][2], pv[1][3]);
+    }
+    m0 = mn0;
+    m1 = mn1;
+#pragma unroll
+    for (int nt = 0; nt < kNT; ++nt) {
+      o[nt][0] *= c0;
+      o[nt][1] *= c0;
+      o[nt][2] *= c1;
+      o[nt][3] *= c1;
+    }
+    // O += P V: V rows are this warp's 16 positions, read transposed
+#pragma unroll
+    for (int nt = 0; nt < kNT; nt += 2) {
+      const int mi = lane >> 3, rr = lane & 7;
+      const int pr = warp * 16 + (mi & 1) * 8 + rr;
+      const int db = nt + (mi >> 1);                              // 8-dim block
+      const int box = db / 8, c = db % 8;
+      const uint32_t addr = smem_u32(vs + box * kBoxBytes + pr * 128 + ((c ^ (pr & 7)) << 4));
+      uint32_t r[4];
+      ldmatrix_x4_trans(r, addr);
+      mma_bf16_16816(o[nt], pa, r[0], r[1]);
+      mma_bf16_16816(o[nt + 1], pa, r[2], r[3]);
+    }
+    __syncthreads();                      // stage `st` consumed by every warp
+    if (tid == 0 && ch + kDecStages < nch) issue(ch + kDecStages);
+  }
+  // full row sums across the four lanes of a row
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  // merge the four warps (the ring is free now: O partials [4][16][HD] there)
+  float* wO = reinterpret_cast<float*>(ring);
+  if (tq == 0) {
+    wm[warp][gq] = m0;
+    wm[warp][gq + 8] = m1;
+    wl[warp][gq] = l0;
+    wl[warp][gq + 8] = l1;
+  }
+#pragma unroll
+  for (int nt = 0; nt < kNT; ++nt) {
+    const int d = nt * 8 + 2 * tq;
+    wO[(warp * kMmaQ + gq) * HD + d] = o[nt][0];
+    wO[(warp * kMmaQ + gq) * HD + d + 1] = o[nt][1];
+    wO[(warp * kMmaQ + gq + 8) * HD + d] = o[nt][2];
+    wO[(warp * kMmaQ + gq + 8) * HD + d + 1] = o[nt][3];
   }
   __syncthreads();
   const int hq_base = g * G;
@@ -228,34 +547,52 @@ __global__ void __launch_bounds__(128) attn_reg_kernel(const AttnArgs a) {
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w][qi]);
-    float L = 0.f, O = 0.f;
+    float Ls = 0.f, O = 0.f;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
-      const float ww = (wm[w][qi] == -INFINITY) ? 0.f : expf(wm[w][qi] - M);
-      L = fmaf(wl[w][qi], ww, L);
-      O = fmaf(wacc[w][qi][d], ww, O);
+      const float ww = (wm[w][qi] == -INFINITY) ? 0.f : exp2f(wm[w][qi] - M);
+      Ls = fmaf(wl[w][qi], ww, Ls);
+      O = fmaf(wO[(w * kMmaQ + qi) * HD + d], ww, O);
     }
     if (n_active == 1) {
       const int ii = qi / G, hh = qi % G;
       const int n = sl * a.rows_per_seq + i0 + ii;
-      DT<TO>::st(static_cast<TO*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, O / L);
+      DT<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
+                            O / Ls);
     } else {
       mine[qi * HD + d] = O;
       if (d == 0) {
         mine[kAttnQ * HD + qi] = M;
-        mine[kAttnQ * HD + kAttnQ + qi] = L;
+        mine[kAttnQ * HD + kAttnQ + qi] = Ls;
       }
     }
   }
   if (n_active == 1) return;
   if (!split_combine_arrive(a, slot, n_active, &flag)) return;
   const float* all = a.part + static_cast<size_t>(slot) * a.n_splits_max * per;
+  if (tid < Q) {
+    float M = -INFINITY;
+    for (int s2 = 0; s2 < n_active; ++s2) M = fmaxf(M, __ldcg(all + s2 * per + kAttnQ * HD + tid));
+    float Ls = 0.f;
+    for (int s2 = 0; s2 < n_active; ++s2) {
+      const float ms = __ldcg(all + s2 * per + kAttnQ * HD + tid);
+      Ls = fmaf(__ldcg(all + s2 * per + kAttnQ * HD + kAttnQ + tid), ms == -INFINITY ? 0.f : exp2f(ms - M), Ls);
+    }
+    cM[tid] = M;
+    cw[tid] = 1.f / Ls;
+  }
+  __syncthreads();
   for (int idx = tid; idx < Q * HD; idx += 128) {
     const int qi = idx / HD, d = idx % HD;
+    float O = 0.f;
+    for (int s2 = 0; s2 < n_active; ++s2) {
+      const float ms = __ldcg(all + s2 * per + kAttnQ * HD + qi);
+      O = fmaf(__ldcg(all + s2 * per + qi * HD + d), ms == -INFINITY ? 0.f : exp2f(ms - cM[qi]), O);
+    }
     const int ii = qi / G, hh = qi % G;
     const int n = sl * a.rows_per_seq + i0 + ii;
-    combine_splits<TO>(a, all, per, n_active, qi, d,
-                       static_cast<TO*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d);
+    DT<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
+                          O * cw[qi]);
   }
 }
 
@@ -433,22 +770,44 @@ static size_t attn_smem(int hd) {
   return sizeof(float) * (kAttnQ * hd + kAttnBlk * (hd + 1) + kAttnBlk * hd + kAttnQ * kAttnBlk + 3 * kAttnQ) + 16;
 }
 
-static int n_qgroups(const AttnArgs& a) {
-  const int RQ = rows_per_group(a.rows_per_seq, a.n_heads / a.n_kv_heads);
+static int n_qgroups(const AttnArgs& a, bool bf16) {
+  const int RQ = rows_per_group(a.rows_per_seq, a.n_heads / a.n_kv_heads, bf16);
   return (a.rows_per_seq + RQ - 1) / RQ;
 }
 
 size_t attn_partial_floats(const AttnArgs& a) {
-  return static_cast<size_t>(a.n_seqs) * n_qgroups(a) * a.n_kv_heads * a.n_splits_max * kAttnQ * (a.head_dim + 2);
+  return static_cast<size_t>(a.n_seqs) * n_qgroups(a, false) * a.n_kv_heads * a.n_splits_max * kAttnQ *
+         (a.head_dim + 2);
 }
-int attn_counters(const AttnArgs& a) { return a.n_seqs * n_qgroups(a) * a.n_kv_heads; }
+int attn_counters(const AttnArgs& a) { return a.n_seqs * n_qgroups(a, false) * a.n_kv_heads; }
 
 template <typename T>
 static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
-  dim3 grid(a.n_splits_max, a.n_kv_heads, a.n_seqs * n_qgroups(a));
+  const bool bf16 = sizeof(T) == 2;
+  dim3 grid(a.n_splits_max, a.n_kv_heads, a.n_seqs * n_qgroups(a, bf16));
+  if (bf16 && use_reg_kernel(a.rows_per_seq, a.n_heads / a.n_kv_heads)) {
+    const size_t smem = 1024 + static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * 2;
+    static bool mma_attr = false;
+    if (!mma_attr) {
+      cudaFuncSetAttribute(attn_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+      cudaFuncSetAttribute(attn_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+      mma_attr = true;
+    }
+    if (a.head_dim == 128) return launch_pdl(attn_mma_kernel<128>, grid, dim3(128), smem, s, *a.kmap, *a.vmap, a);
+    return launch_pdl(attn_mma_kernel<64>, grid, dim3(128), smem, s, *a.kmap, *a.vmap, a);
+  }
   if (use_reg_kernel(a.rows_per_seq, a.n_heads / a.n_kv_heads)) {
-    if (a.head_dim == 128) return launch_pdl(attn_reg_kernel<T, T, 4>, grid, dim3(128), 0, s, a);
-    return launch_pdl(attn_reg_kernel<T, T, 2>, grid, dim3(128), 0, s, a);
+    const size_t ring = static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * sizeof(T);
+    const int qmax = std::min(kRegQ, a.rows_per_seq * (a.n_heads / a.n_kv_heads));
+    const int wq = qmax <= kQPW ? 1 : (qmax <= 2 * kQPW ? 2 : 4);
+    static bool dec_attr = false;
+    if (!dec_attr) {
+      cudaFuncSetAttribute(attn_dec_kernel<T, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+      cudaFuncSetAttribute(attn_dec_kernel<T, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+      dec_attr = true;
+    }
+    if (a.head_dim == 128) return launch_pdl(attn_dec_kernel<T, 4>, grid, dim3(128), ring, s, a, wq);
+    return launch_pdl(attn_dec_kernel<T, 2>, grid, dim3(128), ring, s, a, wq);
   }
   static bool attr = false;
   if (!attr) {

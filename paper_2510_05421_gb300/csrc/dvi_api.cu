@@ -91,6 +91,7 @@ struct dvi_ctx {
   ProjMaps head_v, head_s;
   // TMA descriptors of the activation buffers (bf16 model)
   CUtensorMap map_xg_dr, map_xg_ver, map_xg_pf, map_attn_o, map_ffn_h, map_log_u;
+  CUtensorMap map_kc, map_vc;   // K / V caches as [L*B*H_kv*max_len][hd]
   int log_enabled = 1;
   // graphs of one decode step: the K draft passes, then the verify pass
   cudaGraphExec_t draft_exec = nullptr, verify_exec = nullptr;
@@ -248,8 +249,8 @@ void size_scratch(dvi_ctx* c) {
   c->part_floats = std::max(part, static_cast<size_t>(8) << 20);
   c->n_proj_counters = std::max(ctr, 4096);
   // attention: fixed split length from the capacity so row results do not
-  // depend on the number of rows; about 3 CTAs per SM at full length.
-  const int target = 3 * c->n_sms;
+  // depend on the number of rows; about 4 CTAs per SM at full length.
+  const int target = 4 * c->n_sms;
   int splits = std::max(1, target / std::max(1, c->B * c->Hkv));
   int sl = (c->max_len + splits - 1) / splits;
   sl = std::max(kAttnBlk, (sl + kAttnBlk - 1) / kAttnBlk * kAttnBlk);
@@ -405,6 +406,9 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   t.counters = ctx->attn_ctr;
   t.status = ctx->status;
   t.scale = 1.f / sqrtf(static_cast<float>(ctx->hd));
+  t.kv_row0 = static_cast<long long>(l) * ctx->B * ctx->Hkv * ctx->max_len;
+  t.kmap = &ctx->map_kc;
+  t.vmap = &ctx->map_vc;
   DVI_CUDA(launch_attn(t, s));
   // x += W_o . attn, then xg = x * ffn_norm for the FFN
   a = base_args(ctx, EPI_RESID, ctx->p_o, ps);
@@ -735,6 +739,9 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
          make_act_map(&ctx->map_attn_o, ctx->attn_o, ctx->M_max, ctx->nq) &&
          make_act_map(&ctx->map_ffn_h, ctx->ffn_h, ctx->M_max, ctx->F) &&
          make_act_map(&ctx->map_log_u, ctx->log_u, ctx->cap_rows, ctx->d);
+    const long long kv_rows = static_cast<long long>(ctx->L) * ctx->B * ctx->Hkv * ctx->max_len;
+    ok = ok && make_kv_map(&ctx->map_kc, ctx->kcache, kv_rows, ctx->hd) &&
+         make_kv_map(&ctx->map_vc, ctx->vcache, kv_rows, ctx->hd);
     if (!ok) {
       fprintf(stderr, "dvi_create: TMA descriptor creation failed (weights must be 16-byte aligned)\n");
       delete ctx;

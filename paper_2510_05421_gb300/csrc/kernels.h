@@ -92,7 +92,11 @@ struct AttnArgs {
   float* part; int* counters;        // combine scratch
   int* status;
   float scale;
+  long long kv_row0;                 // bf16 decode: row of (layer, seq 0, head 0, pos 0) in the cache maps
+  const CUtensorMap* kmap;           // bf16 decode: the K / V caches as [rows][hd] (box 64 x 64)
+  const CUtensorMap* vmap;
 };
+bool make_kv_map(CUtensorMap* map, const void* cache, long long rows, int hd);
 size_t attn_partial_floats(const AttnArgs& a);
 int attn_counters(const AttnArgs& a);
 cudaError_t launch_attn(const AttnArgs& a, cudaStream_t s);

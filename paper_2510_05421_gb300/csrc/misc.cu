@@ -22,19 +22,31 @@ namespace dvi {
 constexpr int kMaxTiles = 64;   // d <= 8192
 
 // One residual row from the embedding table (128 threads): x, x * g and the
-// per-tile sums of squares, with a single block barrier.
+// per-tile sums of squares.  All of the row's loads are issued before any is
+// used (one memory round trip), then a single block barrier.
 template <typename T>
 __device__ void embed_row_block(const T* table, int tok, int d, float* x, const float* g, T* xg, float* ss,
                                 int ss_ld, int row, float* red) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nt = d / kTileRows;
-  for (int t = 0; t < nt; ++t) {
-    const int c = t * kTileRows + tid;
-    const float v = DT<T>::ld(table + static_cast<size_t>(tok) * d + c);
-    x[c] = v;
-    DT<T>::st(xg + c, v * g[c]);
-    const float s = warp_sum(v * v);
-    if (lane == 0) red[t * 4 + warp] = s;
+  const T* src = table + static_cast<size_t>(tok) * d;
+  float v[kMaxTiles], gv[kMaxTiles];
+#pragma unroll
+  for (int t = 0; t < kMaxTiles; ++t) {
+    if (t < nt) {
+      v[t] = DT<T>::ld(src + t * kTileRows + tid);
+      gv[t] = g[t * kTileRows + tid];
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < kMaxTiles; ++t) {
+    if (t < nt) {
+      const int c = t * kTileRows + tid;
+      x[c] = v[t];
+      DT<T>::st(xg + c, v[t] * gv[t]);
+      const float s = warp_sum(v[t] * v[t]);
+      if (lane == 0) red[t * 4 + warp] = s;
+    }
   }
   __syncthreads();
   for (int t = tid; t < nt; t += blockDim.x)
@@ -72,18 +84,27 @@ template <typename T>
 __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
   __shared__ float red[kMaxTiles * 4];
   __shared__ float rstd_s;
+  __shared__ __align__(16) float us[kMaxTiles * kTileRows];   // u = x * rstd * gain
   griddep_launch();
   griddep_wait();
   const int row = blockIdx.x, grp = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float* x = a.x + static_cast<size_t>(row) * a.ldx;
   const int nt = a.d / kTileRows;
+  float xv[kMaxTiles], gv[kMaxTiles];
+#pragma unroll
+  for (int t = 0; t < kMaxTiles; ++t)
+    if (t < nt) {
+      xv[t] = x[t * kTileRows + tid];
+      gv[t] = a.gain[t * kTileRows + tid];
+    }
   // per-tile sums of squares (also the hand-off's statistics), then 1/rms
-  for (int t = 0; t < nt; ++t) {
-    const float v = x[t * kTileRows + tid];
-    const float s = warp_sum(v * v);
-    if (lane == 0) red[t * 4 + warp] = s;
-  }
+#pragma unroll
+  for (int t = 0; t < kMaxTiles; ++t)
+    if (t < nt) {
+      const float s = warp_sum(xv[t] * xv[t]);
+      if (lane == 0) red[t * 4 + warp] = s;
+    }
   __syncthreads();
   if (tid == 0) {
     float s = 0.f;
@@ -92,6 +113,9 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
   }
   __syncthreads();
   const float rstd = rstd_s;
+#pragma unroll
+  for (int t = 0; t < kMaxTiles; ++t)
+    if (t < nt) us[t * kTileRows + tid] = xv[t] * rstd * gv[t];
   if (grp == 0) {
     T* lu = nullptr;
     if (a.log_u && a.log_enabled) {
@@ -101,27 +125,47 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
              (static_cast<size_t>(ls) * a.log_rows_per_step + static_cast<size_t>(row) * a.log_row_stride +
               a.log_row_off) * a.d;
     }
-    if (lu)
-      for (int c = tid; c < a.d; c += 128) DT<T>::st(lu + c, x[c] * rstd * a.gain[c]);
+    if (lu) {
+#pragma unroll
+      for (int t = 0; t < kMaxTiles; ++t)
+        if (t < nt) DT<T>::st(lu + t * kTileRows + tid, xv[t] * rstd * gv[t]);
+    }
     if (a.x_copy) {
       const int crow = row * a.copy_row_stride + a.copy_row_off;
       float* xc = a.x_copy + static_cast<size_t>(crow) * a.ld_copy;
       T* xgc = static_cast<T*>(a.xg_copy) + static_cast<size_t>(crow) * a.ld_copy;
-      for (int c = tid; c < a.d; c += 128) {
-        xc[c] = x[c];
-        DT<T>::st(xgc + c, x[c] * a.g_copy[c]);
-      }
+      float gc[kMaxTiles];
+#pragma unroll
+      for (int t = 0; t < kMaxTiles; ++t)
+        if (t < nt) gc[t] = a.g_copy[t * kTileRows + tid];
+#pragma unroll
+      for (int t = 0; t < kMaxTiles; ++t)
+        if (t < nt) {
+          xc[t * kTileRows + tid] = xv[t];
+          DT<T>::st(xgc + t * kTileRows + tid, xv[t] * gc[t]);
+        }
       for (int t = tid; t < nt; t += 128)
         a.ss_copy[static_cast<size_t>(t) * a.ss_copy_ld + crow] =
             (red[t * 4] + red[t * 4 + 1]) + (red[t * 4 + 2] + red[t * 4 + 3]);
     }
   }
   if (a.r > 0 && a.bu) {
+    __syncthreads();
     const int j = grp * 4 + warp;
     if (j < a.r) {
-      const float* br = a.lora_b + static_cast<size_t>(j) * a.d;
+      // B row j (f32) against u from shared memory, 4 floats per lane per step
+      const float4* br = reinterpret_cast<const float4*>(a.lora_b + static_cast<size_t>(j) * a.d);
+      const float4* u4 = reinterpret_cast<const float4*>(us);
       float acc = 0.f;
-      for (int c = lane; c < a.d; c += 32) acc = fmaf(br[c], x[c] * rstd * a.gain[c], acc);
+#pragma unroll 8
+      for (int c = lane; c < a.d / 4; c += 32) {
+        const float4 b = br[c];
+        const float4 u = u4[c];
+        acc = fmaf(b.x, u.x, acc);
+        acc = fmaf(b.y, u.y, acc);
+        acc = fmaf(b.z, u.z, acc);
+        acc = fmaf(b.w, u.w, acc);
+      }
       acc = warp_sum(acc);
       if (lane == 0) a.bu[static_cast<size_t>(row) * a.r + j] = acc;
     }

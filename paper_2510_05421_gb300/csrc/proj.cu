@@ -688,5 +688,17 @@ bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
 bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols) {
   return make_map(map, act, rows, cols, 16);
 }
+bool make_kv_map(CUtensorMap* map, const void* cache, long long rows, int hd) {
+  auto encode = encoder();
+  if (!encode) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(hd), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(hd) * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(cache), dims, strides, box,
+                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
 
 }  // namespace dvi
