@@ -25,11 +25,14 @@
 // memory for 16 queries at a time.
 #include <algorithm>
 #include <cmath>
+#include <cooperative_groups.h>
 
 #include "common.cuh"
 #include "kernels.h"
 
 namespace dvi {
+
+namespace cg = cooperative_groups;
 
 constexpr int kRegQ = 8;      // query vectors per CTA in the decode kernel
 constexpr int kRegPos = 4;    // positions per warp step
@@ -339,7 +342,10 @@ __global__ void __launch_bounds__(128) attn_dec_kernel(const AttnArgs a, int wq_
 // registers, K as the column-major operand read straight from the swizzled
 // rows), an online softmax over its columns in base 2, then O += P V with the
 // accumulator fragments of S reused as the A operand and V fragments loaded
-// transposed by ldmatrix.  The four warps merge at the end.
+// transposed by ldmatrix.  The four warps merge in shared memory; the splits
+// of one (sequence, query group, KV head) form a thread-block cluster and
+// each rank combines a slice of the outputs over every rank's (m, l, O)
+// through distributed shared memory, in rank order.
 constexpr int kMmaQ = 16;
 
 template <int HD>
@@ -352,17 +358,20 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   extern __shared__ __align__(1024) uint8_t dsm_raw[];
   __shared__ __align__(8) uint64_t full[kDecStages];
   __shared__ float wm[4][kMmaQ], wl[4][kMmaQ];
-  __shared__ int flag;
-  __shared__ float cw[kMmaQ], cM[kMmaQ];
+  __shared__ float cm[kMmaQ], cl[kMmaQ];             // this split's merged max / sum
   const uint32_t raw = smem_u32(dsm_raw);
   uint8_t* ring = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+  float* wO = reinterpret_cast<float*>(ring);                       // [4][16][HD], after the loop
+  float* cO = reinterpret_cast<float*>(ring) + 4 * kMmaQ * HD;      // [16][HD] this split's O
   griddep_launch();
   griddep_wait();
+  cg::cluster_group cluster = cg::this_cluster();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, tq = lane & 3;           // mma fragment coordinates
   const int G = a.n_heads / a.n_kv_heads;
   const int RQ = kMmaQ / G;
   const int n_qg = (a.rows_per_seq + RQ - 1) / RQ;
+  const int S = a.n_splits_max;                      // cluster size
   const int split = blockIdx.x, g = blockIdx.y;
   const int sl = blockIdx.z / n_qg, qg = blockIdx.z % n_qg;
   const int seq = a.seq0 + sl;
@@ -372,10 +381,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   const int base = a.lens[seq] + a.pos_off;
   const int t_cta = min(base + i0 + nrows, a.max_len);
   const int p0 = split * a.split_len;
-  if (p0 >= t_cta) return;
-  const int p1 = min(p0 + a.split_len, t_cta);
-  const int n_active = (t_cta + a.split_len - 1) / a.split_len;
-  const int nch = (p1 - p0 + kChunkPos - 1) / kChunkPos;
+  const int p1 = max(p0, min(p0 + a.split_len, t_cta));
+  const int nch = (p1 - p0 + kChunkPos - 1) / kChunkPos;   // 0 for a split past the rows' positions
   const int row0 = static_cast<int>(a.kv_row0 + (static_cast<long long>(seq) * a.n_kv_heads + g) * a.max_len);
 
   auto issue = [&](int ch) {
@@ -521,8 +528,7 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  // merge the four warps (the ring is free now: O partials [4][16][HD] there)
-  float* wO = reinterpret_cast<float*>(ring);
+  // merge the four warps into this split's (m, l, O) (the ring is free now)
   if (tq == 0) {
     wm[warp][gq] = m0;
     wm[warp][gq + 8] = m1;
@@ -538,62 +544,66 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
     wO[(warp * kMmaQ + gq + 8) * HD + d + 1] = o[nt][3];
   }
   __syncthreads();
-  const int hq_base = g * G;
-  const int slot = (sl * n_qg + qg) * a.n_kv_heads + g;
-  const size_t per = static_cast<size_t>(kAttnQ) * (HD + 2);
-  float* mine = a.part + (static_cast<size_t>(slot) * a.n_splits_max + split) * per;
-  for (int idx = tid; idx < Q * HD; idx += 128) {
+  if (tid < kMmaQ) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w][tid]);
+    float Ls = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) Ls = fmaf(wl[w][tid], (wm[w][tid] == -INFINITY) ? 0.f : exp2f(wm[w][tid] - M), Ls);
+    cm[tid] = M;
+    cl[tid] = Ls;
+  }
+  for (int idx = tid; idx < kMmaQ * HD; idx += 128) {
     const int qi = idx / HD, d = idx % HD;
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w][qi]);
+    float O = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w)
+      O = fmaf(wO[(w * kMmaQ + qi) * HD + d], (wm[w][qi] == -INFINITY) ? 0.f : exp2f(wm[w][qi] - M), O);
+    cO[idx] = O;
+  }
+  // combine the splits of the cluster: rank r finishes output elements
+  // r*128 + tid, (r + S)*128 + tid, ...
+  cluster.sync();
+  const float* pm[8];
+  const float* pl[8];
+  const float* pO[8];
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    const int rr = r < S ? r : 0;
+    pm[r] = cluster.map_shared_rank(cm, rr);
+    pl[r] = cluster.map_shared_rank(cl, rr);
+    pO[r] = cluster.map_shared_rank(cO, rr);
+  }
+  const int hq_base = g * G;
+  for (int idx = split * 128 + tid; idx < Q * HD; idx += S * 128) {
+    const int qi = idx / HD, d = idx % HD;
+    float ms[8], ls[8], os[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      ms[r] = r < S ? pm[r][qi] : -INFINITY;
+      ls[r] = r < S ? pl[r][qi] : 0.f;
+      os[r] = r < S ? pO[r][idx] : 0.f;
+    }
+    float M = ms[0];
+#pragma unroll
+    for (int r = 1; r < 8; ++r) M = fmaxf(M, ms[r]);
     float Ls = 0.f, O = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) {
-      const float ww = (wm[w][qi] == -INFINITY) ? 0.f : exp2f(wm[w][qi] - M);
-      Ls = fmaf(wl[w][qi], ww, Ls);
-      O = fmaf(wO[(w * kMmaQ + qi) * HD + d], ww, O);
-    }
-    if (n_active == 1) {
-      const int ii = qi / G, hh = qi % G;
-      const int n = sl * a.rows_per_seq + i0 + ii;
-      DT<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
-                            O / Ls);
-    } else {
-      mine[qi * HD + d] = O;
-      if (d == 0) {
-        mine[kAttnQ * HD + qi] = M;
-        mine[kAttnQ * HD + kAttnQ + qi] = Ls;
-      }
-    }
-  }
-  if (n_active == 1) return;
-  if (!split_combine_arrive(a, slot, n_active, &flag)) return;
-  const float* all = a.part + static_cast<size_t>(slot) * a.n_splits_max * per;
-  if (tid < Q) {
-    float M = -INFINITY;
-    for (int s2 = 0; s2 < n_active; ++s2) M = fmaxf(M, __ldcg(all + s2 * per + kAttnQ * HD + tid));
-    float Ls = 0.f;
-    for (int s2 = 0; s2 < n_active; ++s2) {
-      const float ms = __ldcg(all + s2 * per + kAttnQ * HD + tid);
-      Ls = fmaf(__ldcg(all + s2 * per + kAttnQ * HD + kAttnQ + tid), ms == -INFINITY ? 0.f : exp2f(ms - M), Ls);
-    }
-    cM[tid] = M;
-    cw[tid] = 1.f / Ls;
-  }
-  __syncthreads();
-  for (int idx = tid; idx < Q * HD; idx += 128) {
-    const int qi = idx / HD, d = idx % HD;
-    float O = 0.f;
-    for (int s2 = 0; s2 < n_active; ++s2) {
-      const float ms = __ldcg(all + s2 * per + kAttnQ * HD + qi);
-      O = fmaf(__ldcg(all + s2 * per + qi * HD + d), ms == -INFINITY ? 0.f : exp2f(ms - cM[qi]), O);
+    for (int r = 0; r < 8; ++r) {
+      const float w = (ms[r] == -INFINITY) ? 0.f : exp2f(ms[r] - M);
+      Ls = fmaf(ls[r], w, Ls);
+      O = fmaf(os[r], w, O);
     }
     const int ii = qi / G, hh = qi % G;
     const int n = sl * a.rows_per_seq + i0 + ii;
     DT<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
-                          O * cw[qi]);
+                          O / Ls);
   }
+  cluster.sync();   // every rank keeps its shared memory until all have read it
 }
 
 // ------------------------------------------------------------------ prefill
@@ -786,6 +796,7 @@ static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
   const bool bf16 = sizeof(T) == 2;
   dim3 grid(a.n_splits_max, a.n_kv_heads, a.n_seqs * n_qgroups(a, bf16));
   if (bf16 && use_reg_kernel(a.rows_per_seq, a.n_heads / a.n_kv_heads)) {
+    // one cluster of n_splits_max (<= 8) CTAs per (sequence, query group, KV head)
     const size_t smem = 1024 + static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * 2;
     static bool mma_attr = false;
     if (!mma_attr) {
@@ -793,8 +804,22 @@ static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
       cudaFuncSetAttribute(attn_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
       mma_attr = true;
     }
-    if (a.head_dim == 128) return launch_pdl(attn_mma_kernel<128>, grid, dim3(128), smem, s, *a.kmap, *a.vmap, a);
-    return launch_pdl(attn_mma_kernel<64>, grid, dim3(128), smem, s, *a.kmap, *a.vmap, a);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(128);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = a.n_splits_max;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    if (a.head_dim == 128) return cudaLaunchKernelEx(&cfg, attn_mma_kernel<128>, *a.kmap, *a.vmap, a);
+    return cudaLaunchKernelEx(&cfg, attn_mma_kernel<64>, *a.kmap, *a.vmap, a);
   }
   if (use_reg_kernel(a.rows_per_seq, a.n_heads / a.n_kv_heads)) {
     const size_t ring = static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * sizeof(T);

@@ -26,8 +26,9 @@
 // K is split over `n_splits` CTAs per tile when there are too few tiles to
 // fill the GPU.  bf16: the splits of a tile form one thread-block cluster;
 // each leaves its partial tile in shared memory and, after a cluster barrier,
-// rank 0 sums the partials of all ranks in rank order through distributed
-// shared memory and runs the epilogue.  f32: each split stores its partial in
+// rank r sums the partials of all ranks in rank order through distributed
+// shared memory for the token columns n = r (mod n_splits) and runs their
+// epilogue.  f32: each split stores its partial in
 // global scratch and the last CTA to arrive (an atomic counter per tile) sums
 // them in split order.  Both are deterministic, and the split plan depends on
 // the weight shape only (never on the number of decode rows).
@@ -69,15 +70,22 @@ __device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int
   }
 }
 
-// Fused epilogue for 16 token columns [c0, c0+16) of one 128-feature tile.
-// Called by the 128 epilogue threads together (row = feature within tile).
+// Token columns [c0, c0+16) that hold rows of the launch.
+__device__ __forceinline__ uint32_t valid_cols(const ProjArgs& p, int c0) {
+  const int n = min(kChunk, p.M - c0);
+  return n >= kChunk ? 0xffffu : ((1u << max(n, 0)) - 1u);
+}
+
+// Fused epilogue for the token columns of [c0, c0+16) set in `own` (a
+// subset of the valid ones) of one 128-feature tile.  Called by the 128
+// epilogue threads together (row = feature within tile).
 template <typename T>
 __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, float (&v)[kChunk],
-                               const float* rstd, EpiSmem& es) {
+                               const float* rstd, EpiSmem& es, uint32_t own) {
   const int warp = row >> 5, lane = row & 31;
   if (p.ss) {
 #pragma unroll
-    for (int j = 0; j < kChunk; ++j) v[j] *= (c0 + j < p.M) ? rstd[c0 + j] : 0.f;
+    for (int j = 0; j < kChunk; ++j) v[j] *= ((own >> j) & 1u) ? rstd[c0 + j] : 0.f;
   }
   if (p.flavor == EPI_QKV) {
     const int tq = p.rows_q / kTileRows, tk = p.rows_k / kTileRows;
@@ -97,7 +105,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
 #pragma unroll
     for (int j = 0; j < kChunk; ++j) {
       const int n = c0 + j;
-      if (n < p.M) {
+      if ((own >> j) & 1u) {
         int seq, pos;
         row_seq_pos(p, n, seq, pos);
         if (pos >= p.max_len || pos < 0) {
@@ -127,7 +135,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
     for (int j = 0; j < kChunk; ++j) {
       const int n = c0 + j;
       float xn = 0.f;
-      if (n < p.M && f < p.n_out) {
+      if (((own >> j) & 1u) && f < p.n_out) {
         float* xp = p.x_res + static_cast<size_t>(n) * p.ld_res + f;
         xn = *xp + v[j];
         *xp = xn;
@@ -141,7 +149,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
       if (lane == 0) es.red[warp][j] = s;
     }
     named_bar(1, kTileRows);
-    if (row < kChunk && c0 + row < p.M)
+    if (row < kChunk && ((own >> row) & 1u))
       p.ss_out[static_cast<size_t>(tile) * p.ss_out_ld + c0 + row] =
           (es.red[0][row] + es.red[1][row]) + (es.red[2][row] + es.red[3][row]);
     named_bar(1, kTileRows);
@@ -155,7 +163,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
 #pragma unroll
       for (int j = 0; j < kChunk; ++j) {
         const int n = c0 + j;
-        if (n < p.M) {
+        if ((own >> j) & 1u) {
           const float gt = es.stage[row][j];
           const float h = gt / (1.f + expf(-gt)) * es.stage[row + kGuRows][j];
           DT<T>::st(static_cast<T*>(p.h_out) + static_cast<size_t>(n) * p.ld_h + f, h);
@@ -173,7 +181,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
       const float* arow = p.lora_a + static_cast<size_t>(f) * p.lora_r;
       for (int j = 0; j < kChunk; ++j) {
         const int n = c0 + j;
-        if (n < p.M) {
+        if ((own >> j) & 1u) {
           const float* bu = p.lora_bu + static_cast<size_t>(n) * p.lora_r;
           float acc = 0.f;
           for (int q = 0; q < p.lora_r; ++q) acc = fmaf(arow[q], bu[q], acc);
@@ -193,14 +201,14 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
       if (dst) {
 #pragma unroll
         for (int j = 0; j < kChunk; ++j)
-          if (c0 + j < p.M) dst[static_cast<size_t>(c0 + j) * p.ld_logits + f] = z[j];
+          if ((own >> j) & 1u) dst[static_cast<size_t>(c0 + j) * p.ld_logits + f] = z[j];
       }
     }
     if (p.amax) {
 #pragma unroll
       for (int j = 0; j < kChunk; ++j) {
         unsigned long long key = 0;
-        if (ok && c0 + j < p.M) {
+        if (ok && ((own >> j) & 1u)) {
           if (isfinite(z[j])) key = argmax_key(z[j], f);
           else flag_status(p.status, DVI_DEV_NONFINITE);
         }
@@ -208,7 +216,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
         if (lane == 0) es.redk[warp][j] = key;
       }
       named_bar(1, kTileRows);
-      if (row < kChunk && c0 + row < p.M) {
+      if (row < kChunk && ((own >> row) & 1u)) {
         unsigned long long k0 = es.redk[0][row], k1 = es.redk[1][row];
         unsigned long long k2 = es.redk[2][row], k3 = es.redk[3][row];
         k0 = k0 > k1 ? k0 : k1;
@@ -434,7 +442,7 @@ __global__ void __launch_bounds__(192, 3)
     for (int c = 0; c < nchunks; ++c) {
       tmem_ld16(lane_base + c * kChunk, v);
       if (p.n_splits == 1) {
-        if (ok) epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es);
+        if (ok) epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es, valid_cols(p, c * kChunk));
       } else {
 #pragma unroll
         for (int j = 0; j < kChunk; ++j)
@@ -449,26 +457,44 @@ __global__ void __launch_bounds__(192, 3)
     }
   }
   if (p.n_splits > 1) {
-    // ---------------- split-K across the cluster: rank 0 sums the ranks' partials
+    // ---------------- split-K across the cluster: rank r finishes the token
+    // columns n with n % n_splits == r, summing every rank's partial in rank
+    // order (all of a column's loads are issued before the sum)
     cg::cluster_group cluster = cg::this_cluster();
     cluster.sync();
-    if (split == 0 && warp < 4) {
+    if (warp < 4) {
       const int tid = threadIdx.x;
+      const int S = p.n_splits;
+      const float* peer[8];
+#pragma unroll
+      for (int r = 0; r < 8; ++r) peer[r] = r < S ? cluster.map_shared_rank(part, r) : part;
       const int nchunks = (p.M + kChunk - 1) / kChunk;
-      float v[kChunk];
       for (int c = 0; c < nchunks; ++c) {
+        uint32_t own = 0;
 #pragma unroll
-        for (int j = 0; j < kChunk; ++j) v[j] = 0.f;
-        for (int r = 0; r < p.n_splits; ++r) {
-          const float* peer = cluster.map_shared_rank(part, r);
+        for (int j = 0; j < kChunk; ++j)
+          if (c * kChunk + j < p.M && (c * kChunk + j) % S == split) own |= 1u << j;
+        if (!own) continue;
+        float v[kChunk];
 #pragma unroll
-          for (int j = 0; j < kChunk; ++j)
-            if (c * kChunk + j < p.M) v[j] += peer[(c * kChunk + j) * kTileRows + tid];
+        for (int j = 0; j < kChunk; ++j) {
+          v[j] = 0.f;
+          if ((own >> j) & 1u) {
+            float t[8];
+            const int off = (c * kChunk + j) * kTileRows + tid;
+#pragma unroll
+            for (int r = 0; r < 8; ++r) t[r] = r < S ? peer[r][off] : 0.f;
+            float acc = t[0];
+#pragma unroll
+            for (int r = 1; r < 8; ++r)
+              if (r < S) acc += t[r];
+            v[j] = acc;
+          }
         }
-        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es);
+        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es, own);
       }
     }
-    cluster.sync();   // peers keep their shared memory until rank 0 has read it
+    cluster.sync();   // every rank keeps its shared memory until all have read it
   }
 }
 
@@ -545,7 +571,7 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
   // epilogue_chunk indexes rstd by token; shift so rstd[c0 + j] is this tile's
   float* rs = rstd - c0;
   if (p.n_splits == 1) {
-    epilogue_chunk<float>(p, tile, row, c0, acc, rs, es);
+    epilogue_chunk<float>(p, tile, row, c0, acc, rs, es, valid_cols(p, c0));
     return;
   }
   const size_t reg = static_cast<size_t>(kTileRows) * kChunk;
@@ -557,7 +583,7 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
   const float* all = p.part + static_cast<size_t>(ci) * p.n_splits * reg;
 #pragma unroll
   for (int j = 0; j < kChunk; ++j) acc[j] = sum_splits(all + j * kTileRows + row, reg, p.n_splits);
-  epilogue_chunk<float>(p, tile, row, c0, acc, rs, es);
+  epilogue_chunk<float>(p, tile, row, c0, acc, rs, es, valid_cols(p, c0));
 }
 
 // ------------------------------------------------------------------ host
