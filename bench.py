@@ -72,6 +72,32 @@ def step_bytes(w, n_ctx):
     return draft, verify
 
 
+def measured_traffic(w, n_attended):
+    """Per-launch DRAM traffic of the verify pass from the committed ncu summary.
+
+    The summary holds the bytes ncu counted per deep layer's projections, the
+    LM head, and one deep layer's attention at a given number of 64-position
+    chunks; the pass's traffic is scaled to this workload's layer count and
+    context.  Returns None when no capture matches the workload.
+    """
+    p = os.path.join(ROOT, "profiles", "verify_pass_dram_7b_width.md")
+    if not os.path.exists(p):
+        return None
+    m = None
+    for ln in open(p):
+        if ln.startswith("traffic-model:"):
+            m = json.loads(ln.split(":", 1)[1])
+    s = w.shape
+    if m is None or (m["d_model"], m["n_heads"], m["d_ffn"], m["vocab"]) != (s.d_model, s.n_heads, s.d_ffn,
+                                                                             s.vocab) \
+            or m["dtype"] != w.dtype or m["batch"] != w.batch or m["k_spec"] != w.k_spec:
+        return None
+    deep = w.shape.n_layers - w.split_k
+    chunks = float(np.mean([-(-int(round(n + w.k_spec)) // 64) * 64 for n in n_attended]))
+    return deep * (m["proj_bytes_per_deep_layer"] + m["attn_bytes_per_deep_layer"] * chunks
+                   / m["attn_chunk_positions"]) + m["head_bytes"]
+
+
 # ---------------------------------------------------------------- clocks
 class ClockSampler:
     REASONS = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
@@ -163,12 +189,19 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling cases)")
+    ap.add_argument("--prompt", type=int, default=0, help="override the prompt length (small profiling cases)")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     w = workload(args.workload)
+    if args.layers:
+        from dataclasses import replace
+        w = w.with_(shape=replace(w.shape, n_layers=args.layers), name=f"{w.name}-L{args.layers}")
+    if args.prompt:
+        w = w.with_(prompt_len=(args.prompt, args.prompt), name=f"{w.name}-p{args.prompt}")
     assert args.warmup >= 3, "at least 3 warm-up steps"
 
     if args.impl == "reference":
@@ -272,6 +305,7 @@ def main():
     u_ms = phases["update"][0] / max(1, phases["update"][1])
     hbm = pk["hbm_gbs"]
     v_gbs = verify_b / (v_ms / 1e3) / 1e9
+    v_traffic = measured_traffic(w, n_mid)
     d_gbs = draft_b / (d_ms / 1e3) / 1e9
 
     e2e = None
@@ -307,7 +341,9 @@ def main():
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "mean_accepted_length": mat,
         "roofline": {"bound": "hbm", "achieved": v_gbs, "peak": hbm, "unit": "GB/s", "frac": v_gbs / hbm,
-                     "traffic": None, "kernel": "verify pass (layers k+1..L + LM head, CUDA-graph replay)",
+                     "traffic": v_traffic, "kernel": "verify pass (layers k+1..L + LM head, CUDA-graph replay)",
+                     "traffic_source": "profiles/verify_pass_dram_7b_width.md (ncu, 4-layer case scaled)"
+                     if v_traffic else None,
                      "bytes_per_launch": verify_b, "ms_per_launch": v_ms, "peak_source": pk_src},
         "roofline_draft": {"bound": "hbm", "achieved": d_gbs, "peak": hbm, "unit": "GB/s", "frac": d_gbs / hbm,
                            "bytes_per_launch": draft_b, "ms_per_launch": d_ms},
