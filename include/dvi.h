@@ -82,7 +82,10 @@ typedef struct {
   int k_spec;           /* K: drafted tokens per step, 1 <= K <= 16 / (H_q / H_kv) */
   int max_seq_len;      /* KV rows per sequence: prompt + generated + K */
   int log_steps;        /* decode steps the replay buffer holds between updates (U) */
-  int head_mode;        /* 0: train LoRA A_s, B_s on the frozen W^(S); 1: train W^(S) itself */
+  int head_mode;        /* 0: train LoRA A_s, B_s on the frozen W^(S); 1: train W^(S) itself
+                           (the LoRA factors, if any, stay frozen; the workspace then holds
+                           the Adam moments of W^(S), an f32 master copy of it when dtype is
+                           bf16, and the gradient buffer: 12 (f32) or 16 (bf16) B per entry) */
   int max_prefill_chunk;/* rows per prefill pass, 16..128 (multiple of 16); 0 = 128 */
   int use_graphs;       /* capture the decode step in a CUDA graph on first use */
 } dvi_runtime_config;
@@ -102,7 +105,9 @@ typedef struct {
 /* Device pointers, caller-owned, read for the whole life of the context.
  * draft_head (W^(S)) may alias lm_head (W^(V)) only when head_mode == 0.
  * lora_a / lora_b are updated in place by dvi_update_drafter (head_mode 0);
- * draft_head is updated in place in head_mode 1. */
+ * draft_head is updated in place in head_mode 1: with dtype bf16 the
+ * optimizer steps an f32 master copy (taken from draft_head by dvi_create)
+ * and writes its bf16 rounding back to draft_head after every update. */
 typedef struct {
   const void* embed;              /* [V][d] */
   const dvi_layer_weights* layers;/* host array of L entries */
@@ -127,6 +132,8 @@ typedef struct {
   float w_ce, w_ent, w_rl_max;
   float beta0, beta_min, t_beta;              /* beta(t) of L_policy */
   float baseline_rho;                         /* EMA constant of the reward baseline b */
+  int keep_grad_w;                            /* head_mode 1: also store dL/dW^(S) in DVI_BUF_GRAD_W
+                                                 (4 more bytes of traffic per W^(S) entry) */
 } dvi_update_config;
 
 typedef struct {
@@ -177,8 +184,12 @@ dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids,
 dvi_status dvi_log(dvi_ctx* ctx, int enable);
 
 /* One drafter-head update on every tuple logged since the last update
- * (Sec. 3.4), then clear the buffer and advance t.  A non-finite loss skips
- * the parameter step and sets DVI_DEV_NONFINITE. */
+ * (Sec. 3.4), then clear the buffer and advance t.  With the per-row logit
+ * gradients G [N][V] of the loss, head_mode 0 steps A_s and B_s with
+ * dA = gamma G^T (U B^T) and dB = gamma (G A)^T U; head_mode 1 steps W^(S)
+ * with dW = G^T U.  A non-finite loss skips the parameter step and sets
+ * DVI_DEV_NONFINITE.  DVI_ERR_UNIMPLEMENTED in head_mode 0 without LoRA
+ * factors (nothing to train). */
 dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* ucfg);
 
 /* Baseline: one greedy autoregressive step of the full model for every
@@ -212,7 +223,7 @@ enum {
   DVI_BUF_K_CACHE = 10,    /* dtype [L][B][H_kv][max_seq_len][hd] */
   DVI_BUF_V_CACHE = 11,
   DVI_BUF_STATUS = 12,     /* int32 device status word */
-  DVI_BUF_GRAD_W = 13,     /* f32 [V][d] last dL/dW^(S) (head_mode 1) */
+  DVI_BUF_GRAD_W = 13,     /* f32 [V][d] last dL/dW^(S) (head_mode 1, written when keep_grad_w) */
   DVI_BUF_Z = 14,          /* f32 [cap][V] drafter logits of the last update */
   DVI_BUF_COUNT
 };

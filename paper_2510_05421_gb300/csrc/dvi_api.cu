@@ -83,6 +83,9 @@ struct dvi_ctx {
   float* log_logits;
   float *Z, *rowstat, *coef, *ub, *ga, *ga_part;
   float *m_a, *v_a, *m_b, *v_b, *grad_a, *grad_b;
+  // full-head mode (head_mode 1): f32 master of W^S (bf16 only), Adam
+  // moments, per-row logit gradients G, the optional gradient copy
+  float *w_master = nullptr, *m_w = nullptr, *v_w = nullptr, *G = nullptr, *grad_w = nullptr;
   int *out_ids, *n_committed, *n_accepted, *ar_out;
   size_t ws_bytes;
   void* ws;
@@ -142,7 +145,7 @@ bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::
   if (rt->max_seq_len < rt->k_spec + 2) return bad("max_seq_len too small");
   if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
     return bad("log_steps * batch * k_spec must be in [1, 256]");
-  if (rt->head_mode != 0) return bad("head_mode 1 (full W^S training) is not available");
+  if (rt->head_mode != 0 && rt->head_mode != 1) return bad("head_mode must be 0 (LoRA) or 1 (full W^S)");
   if (rt->max_prefill_chunk && (rt->max_prefill_chunk < 16 || rt->max_prefill_chunk > 128 || rt->max_prefill_chunk % 16))
     return bad("max_prefill_chunk must be 16..128, a multiple of 16");
   if (rt->batch * rt->k_spec > kMaxTokens) return bad("batch * k_spec > 256");
@@ -208,6 +211,14 @@ size_t layout(dvi_ctx* c, char* base) {
   c->m_b = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(rr) * d));
   c->v_b = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(rr) * d));
   c->grad_b = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(rr) * d));
+  if (c->rt.head_mode == 1) {
+    const size_t vd = static_cast<size_t>(V) * d;
+    c->w_master = c->tc ? reinterpret_cast<float*>(take(sizeof(float) * vd)) : nullptr;
+    c->m_w = reinterpret_cast<float*>(take(sizeof(float) * vd));
+    c->v_w = reinterpret_cast<float*>(take(sizeof(float) * vd));
+    c->grad_w = reinterpret_cast<float*>(take(sizeof(float) * vd));
+    c->G = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
+  }
   c->out_ids = reinterpret_cast<int*>(take(sizeof(int) * B * K));
   c->n_committed = reinterpret_cast<int*>(take(sizeof(int) * B));
   c->n_accepted = reinterpret_cast<int*>(take(sizeof(int) * B));
@@ -710,6 +721,11 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
       !weights->draft_head || !workspace)
     return DVI_ERR_INVALID_ARG;
   if (cfg->lora_rank > 0 && (!weights->lora_a || !weights->lora_b)) return DVI_ERR_INVALID_ARG;
+  if (rt->head_mode == 1 && (weights->draft_head == weights->lm_head || !aligned16(weights->draft_head))) {
+    fprintf(stderr, "dvi_create: head_mode 1 trains draft_head in place: it must not alias lm_head and must be "
+                    "16-byte aligned\n");
+    return DVI_ERR_INVALID_ARG;
+  }
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return DVI_ERR_INVALID_ARG;
   dvi_ctx* ctx = new dvi_ctx();
   init_dims(ctx, cfg, rt);
@@ -761,6 +777,8 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
   if (cudaMemsetAsync(workspace, 0, ctx->ws_bytes, ctx->stream) != cudaSuccess ||
       cudaMemcpyAsync(ctx->rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice, ctx->stream) !=
           cudaSuccess ||
+      (ctx->w_master && launch_master_init(weights->draft_head, ctx->w_master,
+                                           static_cast<size_t>(ctx->V) * ctx->d, ctx->stream) != cudaSuccess) ||
       cudaStreamSynchronize(ctx->stream) != cudaSuccess) {
     delete ctx;
     return DVI_ERR_CUDA;
@@ -850,7 +868,8 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   if (!(u->tau > 0.f) || u->t_ramp < 0 || u->t_warmup < 0 || u->objective < 0 || u->objective > 3 ||
       u->optimizer < 0 || u->optimizer > 1 || !(u->t_beta > 0.f))
     return fail(ctx, DVI_ERR_INVALID_ARG, "update: bad hyper-parameters");
-  if (ctx->r == 0) return fail(ctx, DVI_ERR_UNIMPLEMENTED, "update: no LoRA factors (lora_rank 0)");
+  const bool full = ctx->rt.head_mode == 1;
+  if (!full && ctx->r == 0) return fail(ctx, DVI_ERR_UNIMPLEMENTED, "update: no LoRA factors (lora_rank 0)");
   cudaStream_t s = ctx->stream;
   UpdateArgs a{};
   a.cap = ctx->cap_rows;
@@ -880,6 +899,13 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   a.v_b = ctx->v_b;
   a.grad_a = ctx->grad_a;
   a.grad_b = ctx->grad_b;
+  a.w_head = ctx->w.draft_head;
+  a.w_master = ctx->w_master;
+  a.m_w = ctx->m_w;
+  a.v_w = ctx->v_w;
+  a.G = ctx->G;
+  a.grad_w = ctx->grad_w;
+  a.keep_grad_w = u->keep_grad_w ? 1 : 0;
   a.dev_state = ctx->dev_state;
   a.counters = ctx->counters;
   a.status = ctx->status;
@@ -906,10 +932,15 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   DVI_CUDA(launch_proj(p, ctx->tc ? &pm : nullptr, s));
   DVI_CUDA(launch_update_rowstats(a, s));
   DVI_CUDA(launch_update_coef(a, s));
-  DVI_CUDA(launch_update_grad_a(a, s));
-  DVI_CUDA(launch_update_grad_b(a, s));
+  if (full) {
+    DVI_CUDA(launch_update_full(a, s));
+    ctx->launches += (ctx->r > 0 ? 1 : 0) + 6;
+  } else {
+    DVI_CUDA(launch_update_grad_a(a, s));
+    DVI_CUDA(launch_update_grad_b(a, s));
+    ctx->launches += 8;
+  }
   DVI_CUDA(launch_update_finish(a, s));
-  ctx->launches += 8;
   mark_end(ctx, 2, t0);
   return DVI_OK;
 }
@@ -993,6 +1024,11 @@ dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes)
     case DVI_BUF_K_CACHE: *dptr = ctx->kcache; *bytes = kv; break;
     case DVI_BUF_V_CACHE: *dptr = ctx->vcache; *bytes = kv; break;
     case DVI_BUF_STATUS: *dptr = ctx->status; *bytes = sizeof(int); break;
+    case DVI_BUF_GRAD_W:
+      if (!ctx->grad_w) return fail(ctx, DVI_ERR_INVALID_ARG, "debug_buffer: GRAD_W exists in head_mode 1 only");
+      *dptr = ctx->grad_w;
+      *bytes = sizeof(float) * static_cast<size_t>(ctx->V) * ctx->d;
+      break;
     case DVI_BUF_Z: *dptr = ctx->Z; *bytes = sizeof(float) * ctx->cap_rows * static_cast<size_t>(ctx->V); break;
     default: return fail(ctx, DVI_ERR_INVALID_ARG, "debug_buffer: unknown buffer");
   }

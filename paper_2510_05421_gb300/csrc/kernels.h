@@ -161,6 +161,9 @@ struct UpdateArgs {
   float* lora_a; float* lora_b; float gamma;
   float* m_a; float* v_a; float* m_b; float* v_b;
   float* grad_a; float* grad_b;
+  // full-head mode: W^S (model dtype), its f32 master (bf16 only, else null),
+  // Adam moments, G [cap][V], the optional gradient copy
+  void* w_head; float* w_master; float* m_w; float* v_w; float* G; float* grad_w; int keep_grad_w;
   float* dev_state;                             // [0]=t, [1]=b, [2..] loss parts
   long long* counters;
   int* status;
@@ -171,6 +174,8 @@ cudaError_t launch_update_rowstats(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_coef(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_update_full(const UpdateArgs& a, cudaStream_t s);
+cudaError_t launch_master_init(const void* w_bf16, float* master, size_t n, cudaStream_t s);
 cudaError_t launch_update_finish(const UpdateArgs& a, cudaStream_t s);
 
 }  // namespace dvi

@@ -20,6 +20,13 @@
 //  update_ga_reduce GA[n] = sum over vocabulary tiles (fixed order)
 //  update_grad_b    dB[j][c] = gamma sum_n GA[n][j] u_n[c], optimizer step
 //  update_finish    t += 1, empty the buffer
+//
+// Full-head mode (W^S itself is trained; LoRA factors, if any, stay frozen)
+// replaces grad_a .. grad_b by
+//  update_g         G[n][v] = dL/dz_{n,v} (the same closed forms)
+//  update_gw        dW[v][c] = sum_n G[n][v] u_n[c] and the optimizer step on
+//                   W^S (its f32 master when the weights are bf16; the bf16
+//                   rounding is written back for the next drafter passes)
 #include <cmath>
 
 #include "common.cuh"
@@ -225,6 +232,24 @@ __device__ __forceinline__ void opt_step(const dvi_update_config& c, float step,
   *p -= c.lr * mh / (sqrtf(vh) + c.adam_eps);
 }
 
+// dL/dz_{n,v} of a valid row n from its row statistics and term coefficients:
+//   KL(p||q):  p (log p - log q - KL)      KL(p||q1): p (log p - log q1 - KL1)
+//   -H[p]:     p (log p + H)               CE to a / to y*: p - [v = a / y*]
+__device__ __forceinline__ float logit_grad(const UpdateArgs& a, int n, int v, float it) {
+  const float* rs = a.rowstat + n * RS_N;
+  const float* cf = a.coef + n * CF_N;
+  const float z = a.Z[static_cast<size_t>(n) * a.V + v];
+  const float l = a.log_logits[static_cast<size_t>(n) * a.V + v];
+  const float lp = z - rs[RS_LSEZ];
+  const float p = expf(lp);
+  const float lq = l * it - rs[RS_LSEQ];
+  const float lq1 = l - rs[RS_LSEQ1];
+  const int* meta = a.log_meta + n * 6;
+  return cf[CF_KL] * p * (lp - lq - rs[RS_KL]) + cf[CF_KL1] * p * (lp - lq1 - rs[RS_KL1]) +
+         cf[CF_ENT] * p * (lp + rs[RS_ENT]) + cf[CF_A] * (p - (v == meta[1] ? 1.f : 0.f)) +
+         cf[CF_Y] * (p - (v == meta[5] ? 1.f : 0.f));
+}
+
 // grid = ceil(V/128); dynamic smem: G tile [cap][128] + A tile [128][r]
 __global__ void __launch_bounds__(128) update_grad_a_kernel(const UpdateArgs a) {
   griddep_launch();
@@ -247,18 +272,7 @@ __global__ void __launch_bounds__(128) update_grad_a_kernel(const UpdateArgs a) 
   for (int n = 0; n < a.cap; ++n) {
     float G = 0.f;
     if (ok && row_valid(a, n)) {
-      const float* rs = a.rowstat + n * RS_N;
-      const float* cf = a.coef + n * CF_N;
-      const float z = a.Z[static_cast<size_t>(n) * a.V + v];
-      const float l = a.log_logits[static_cast<size_t>(n) * a.V + v];
-      const float lp = z - rs[RS_LSEZ];
-      const float p = expf(lp);
-      const float lq = l * it - rs[RS_LSEQ];
-      const float lq1 = l - rs[RS_LSEQ1];
-      const int* meta = a.log_meta + n * 6;
-      G = cf[CF_KL] * p * (lp - lq - rs[RS_KL]) + cf[CF_KL1] * p * (lp - lq1 - rs[RS_KL1]) +
-          cf[CF_ENT] * p * (lp + rs[RS_ENT]) + cf[CF_A] * (p - (v == meta[1] ? 1.f : 0.f)) +
-          cf[CF_Y] * (p - (v == meta[5] ? 1.f : 0.f));
+      G = logit_grad(a, n, v, it);
       const float* ub = a.ub + n * a.r;
       for (int j = 0; j < a.r; ++j) dA[j] = fmaf(G, ub[j], dA[j]);
     }
@@ -317,6 +331,136 @@ __global__ void __launch_bounds__(128) update_grad_b_kernel(const UpdateArgs a) 
   }
 }
 
+// ---------------------------------------------------------------- full-head mode
+
+// G[n][v] for every buffer row (zeros for rows that are not valid).
+// grid = (ceil(V/256), cap), 256 threads.
+__global__ void __launch_bounds__(256) update_g_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
+  if (a.dev_state[DS_SKIP] != 0.f) return;
+  const int n = blockIdx.y;
+  const int v = blockIdx.x * 256 + threadIdx.x;
+  if (v >= a.V) return;
+  a.G[static_cast<size_t>(n) * a.V + v] = row_valid(a, n) ? logit_grad(a, n, v, 1.f / a.cfg.tau) : 0.f;
+}
+
+constexpr int kGwRows = 16;    // W^S rows per CTA (accumulators per thread: kGwRows x 4)
+constexpr int kGwCols = 512;   // W^S columns per CTA: 128 threads x 4 consecutive columns
+constexpr int kGwStage = 16;   // buffer rows staged in shared memory per round
+
+// dW = G^T U for a [kGwRows x kGwCols] tile of W^S, then the optimizer step
+// on it.  The contraction runs over the buffer rows (N <= 256), so it is a
+// few FMAs per W^S entry; the kernel streams W^S (master), m and v once.
+// grid = (ceil(V / kGwRows), ceil(d / kGwCols)), 128 threads.
+template <typename T>
+__global__ void __launch_bounds__(128) update_gw_kernel(const UpdateArgs a) {
+  griddep_launch();
+  griddep_wait();
+  if (a.dev_state[DS_SKIP] != 0.f) return;
+  __shared__ float4 us[kGwStage][kGwCols / 4];
+  __shared__ float gs[kGwStage][kGwRows];
+  const int tid = threadIdx.x;
+  const int v0 = blockIdx.x * kGwRows;
+  const int cb = blockIdx.y * kGwCols;
+  const int c = cb + tid * 4;
+  float4 acc[kGwRows];
+#pragma unroll
+  for (int i = 0; i < kGwRows; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  const T* U = static_cast<const T*>(a.log_u);
+  for (int n0 = 0; n0 < a.cap; n0 += kGwStage) {
+    __syncthreads();
+    for (int i = tid; i < kGwStage * (kGwCols / 4); i += 128) {
+      const int row = i / (kGwCols / 4), col = cb + (i % (kGwCols / 4)) * 4;
+      const int n = n0 + row;
+      float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (n < a.cap && col < a.d && row_valid(a, n)) {
+        const T* src = U + static_cast<size_t>(n) * a.d + col;
+        u = make_float4(DT<T>::ld(src), DT<T>::ld(src + 1), DT<T>::ld(src + 2), DT<T>::ld(src + 3));
+      }
+      us[row][i % (kGwCols / 4)] = u;
+    }
+    for (int i = tid; i < kGwStage * kGwRows; i += 128) {
+      const int row = i / kGwRows, vv = i % kGwRows;
+      const int n = n0 + row, v = v0 + vv;
+      gs[row][vv] = (n < a.cap && v < a.V) ? a.G[static_cast<size_t>(n) * a.V + v] : 0.f;
+    }
+    __syncthreads();
+    const int rows = min(kGwStage, a.cap - n0);
+    for (int row = 0; row < rows; ++row) {
+      const float4 u = us[row][tid];
+#pragma unroll
+      for (int vv = 0; vv < kGwRows; ++vv) {
+        const float g = gs[row][vv];
+        acc[vv].x = fmaf(g, u.x, acc[vv].x);
+        acc[vv].y = fmaf(g, u.y, acc[vv].y);
+        acc[vv].z = fmaf(g, u.z, acc[vv].z);
+        acc[vv].w = fmaf(g, u.w, acc[vv].w);
+      }
+    }
+  }
+  if (c >= a.d) return;
+  const dvi_update_config& cf = a.cfg;
+  const float step = a.dev_state[DS_ADAM];
+  const float bc1 = 1.f - powf(cf.beta1, step), bc2 = 1.f - powf(cf.beta2, step);
+  float* master = a.w_master ? a.w_master : static_cast<float*>(a.w_head);
+  // four rows at a time: their loads are issued before any store
+#pragma unroll
+  for (int g0 = 0; g0 < kGwRows; g0 += 4) {
+    float4 p[4], m[4], s[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int v = v0 + g0 + j;
+      if (v >= a.V) continue;
+      const size_t i = static_cast<size_t>(v) * a.d + c;
+      p[j] = *reinterpret_cast<const float4*>(master + i);
+      if (cf.optimizer == 0) {
+        m[j] = *reinterpret_cast<const float4*>(a.m_w + i);
+        s[j] = *reinterpret_cast<const float4*>(a.v_w + i);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int v = v0 + g0 + j;
+      if (v >= a.V) continue;
+      const size_t i = static_cast<size_t>(v) * a.d + c;
+      const float4 g = acc[g0 + j];
+      if (a.keep_grad_w) *reinterpret_cast<float4*>(a.grad_w + i) = g;
+      float gv[4] = {g.x, g.y, g.z, g.w};
+      float pv[4] = {p[j].x, p[j].y, p[j].z, p[j].w};
+      if (cf.optimizer == 1) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) pv[q] -= cf.lr * gv[q];
+      } else {
+        float mv[4] = {m[j].x, m[j].y, m[j].z, m[j].w};
+        float sv[4] = {s[j].x, s[j].y, s[j].z, s[j].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          mv[q] = cf.beta1 * mv[q] + (1.f - cf.beta1) * gv[q];
+          sv[q] = cf.beta2 * sv[q] + (1.f - cf.beta2) * gv[q] * gv[q];
+          pv[q] -= cf.lr * (mv[q] / bc1) / (sqrtf(sv[q] / bc2) + cf.adam_eps);
+        }
+        *reinterpret_cast<float4*>(a.m_w + i) = make_float4(mv[0], mv[1], mv[2], mv[3]);
+        *reinterpret_cast<float4*>(a.v_w + i) = make_float4(sv[0], sv[1], sv[2], sv[3]);
+      }
+      *reinterpret_cast<float4*>(master + i) = make_float4(pv[0], pv[1], pv[2], pv[3]);
+      if (a.w_master) {
+        uint2 packed;
+        packed.x = pack_bf16x2(pv[0], pv[1]);
+        packed.y = pack_bf16x2(pv[2], pv[3]);
+        *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(a.w_head) + i) = packed;
+      }
+    }
+  }
+}
+
+// master[i] = W^S[i] (bf16 -> f32), once at context creation.
+__global__ void update_master_init_kernel(const __nv_bfloat16* w, float* master, size_t n) {
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x)
+    master[i] = __bfloat162float(w[i]);
+}
+
 __global__ void update_finish_kernel(const UpdateArgs a) {
   griddep_launch();
   griddep_wait();
@@ -364,6 +508,19 @@ cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s) {
   e = a.dtype == DVI_BF16 ? launch_pdl(update_grad_b_kernel<__nv_bfloat16>, dim3((a.d + 127) / 128), dim3(128), 0, s, a)
                           : launch_pdl(update_grad_b_kernel<float>, dim3((a.d + 127) / 128), dim3(128), 0, s, a);
   if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+cudaError_t launch_update_full(const UpdateArgs& a, cudaStream_t s) {
+  cudaError_t e = launch_pdl(update_g_kernel, dim3((a.V + 255) / 256, a.cap), dim3(256), 0, s, a);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((a.V + kGwRows - 1) / kGwRows, (a.d + kGwCols - 1) / kGwCols);
+  e = a.dtype == DVI_BF16 ? launch_pdl(update_gw_kernel<__nv_bfloat16>, grid, dim3(128), 0, s, a)
+                          : launch_pdl(update_gw_kernel<float>, grid, dim3(128), 0, s, a);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+cudaError_t launch_master_init(const void* w_bf16, float* master, size_t n, cudaStream_t s) {
+  update_master_init_kernel<<<1024, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(w_bf16), master, n);
   return cudaGetLastError();
 }
 cudaError_t launch_update_finish(const UpdateArgs& a, cudaStream_t s) {

@@ -60,7 +60,7 @@ class UpdateConfigC(ctypes.Structure):
                 ("lambda_pg_max", ctypes.c_float), ("t_warmup", ctypes.c_int), ("t_ramp", ctypes.c_int),
                 ("w_ce", ctypes.c_float), ("w_ent", ctypes.c_float), ("w_rl_max", ctypes.c_float),
                 ("beta0", ctypes.c_float), ("beta_min", ctypes.c_float), ("t_beta", ctypes.c_float),
-                ("baseline_rho", ctypes.c_float)]
+                ("baseline_rho", ctypes.c_float), ("keep_grad_w", ctypes.c_int)]
 
 
 class StatsC(ctypes.Structure):
@@ -125,12 +125,12 @@ def _ptr(t: Optional[torch.Tensor]):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
-def update_config(h) -> UpdateConfigC:
+def update_config(h, keep_grad_w: bool = False) -> UpdateConfigC:
     """UpdateConfigC from a workloads.UpdateHyper (or any object with its fields)."""
     obj = {"dvi": 0, "kl": 1, "pg": 2, "ce": 3}[h.objective]
     return UpdateConfigC(obj, 0 if h.optimizer == "adam" else 1, h.lr, h.beta1, h.beta2, h.adam_eps, h.tau,
                          h.lambda0, h.lambda_kl_min, h.lambda_pg_max, h.t_warmup, h.t_ramp, h.w_ce, h.w_ent,
-                         h.w_rl_max, h.beta0, h.beta_min, h.t_beta, h.baseline_rho)
+                         h.w_rl_max, h.beta0, h.beta_min, h.t_beta, h.baseline_rho, 1 if keep_grad_w else 0)
 
 
 @dataclass
@@ -181,7 +181,7 @@ class DVIEngine:
 
     def __init__(self, shape, dtype: str, weights: DeviceWeights, *, batch: int, k_spec: int, split_k: int,
                  lora_rank: int, lora_gamma: float = 1.0, max_seq_len: int, log_steps: int,
-                 prefill_chunk: int = 128, use_graphs: bool = True, device: int = 0):
+                 prefill_chunk: int = 128, use_graphs: bool = True, device: int = 0, head_mode: int = 0):
         L = lib()
         self.shape, self.dtype, self.w = shape, dtype, weights
         self.B, self.K = batch, k_spec
@@ -189,7 +189,8 @@ class DVIEngine:
         self.cfg = ModelConfig(shape.n_layers, shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim,
                                shape.d_ffn, shape.vocab, split_k, lora_rank, lora_gamma, shape.rms_eps,
                                shape.rope_theta, DVI_BF16 if dtype == "bf16" else DVI_F32)
-        self.rt = RuntimeConfig(batch, k_spec, max_seq_len, log_steps, 0, prefill_chunk, 1 if use_graphs else 0)
+        self.rt = RuntimeConfig(batch, k_spec, max_seq_len, log_steps, head_mode, prefill_chunk,
+                                1 if use_graphs else 0)
         nbytes = L.dvi_workspace_bytes(ctypes.byref(self.cfg), ctypes.byref(self.rt))
         if nbytes == 0:
             raise DVIError("invalid configuration")
@@ -240,8 +241,8 @@ class DVIEngine:
         self._check(rc, "dvi_draft_verify_commit")
         return self.out_ids, self.n_committed, self.n_accepted
 
-    def update(self, hyper):
-        c = hyper if isinstance(hyper, UpdateConfigC) else update_config(hyper)
+    def update(self, hyper, keep_grad_w: bool = False):
+        c = hyper if isinstance(hyper, UpdateConfigC) else update_config(hyper, keep_grad_w)
         self._check(lib().dvi_update_drafter(self.ctx, ctypes.byref(c)), "dvi_update_drafter")
 
     def log(self, enable: bool):

@@ -56,7 +56,7 @@ def test_workspace_sizes(L, name):
 
 
 @pytest.mark.parametrize("bad", [dict(k_spec=0), dict(k_spec=17), dict(batch=0), dict(max_seq_len=3),
-                                 dict(log_steps=100), dict(max_prefill_chunk=24), dict(head_mode=1)])
+                                 dict(log_steps=100), dict(max_prefill_chunk=24), dict(head_mode=2)])
 def test_invalid_runtime_rejected(L, bad):
     cfg, rt = _cfgs(WORKLOADS["tiny"], **bad)
     assert L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt)) == 0
@@ -65,6 +65,20 @@ def test_invalid_runtime_rejected(L, bad):
     rc = L.dvi_create(ctypes.byref(cfg), ctypes.byref(rt), ctypes.byref(w), ctypes.c_void_p(256), 1 << 30, None,
                       ctypes.byref(ctx))
     assert rc == -1 and not ctx.value
+
+
+@pytest.mark.parametrize("name", ["tiny", "7b"])
+def test_full_head_mode_workspace(L, name):
+    """head_mode 1 adds the Adam moments, the gradient and (bf16) an f32 master of W^(S)."""
+    w = WORKLOADS[name]
+    cfg, rt0 = _cfgs(w)
+    _, rt1 = _cfgs(w, head_mode=1)
+    n0 = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt0))
+    n1 = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt1))
+    vd = w.shape.vocab * w.shape.d_model
+    per = 16 if w.dtype == "bf16" else 12
+    extra = n1 - n0
+    assert per * vd <= extra < per * vd + 4 * rt1.log_steps * rt1.batch * rt1.k_spec * w.shape.vocab + 4096
 
 
 def test_invalid_model_rejected(L):
