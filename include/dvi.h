@@ -58,9 +58,12 @@ enum {
 typedef enum { DVI_F32 = 0, DVI_BF16 = 1 } dvi_dtype;
 
 /* The decoder (Sec. 3.1; the backbone is Llama-style: pre-norm RMSNorm,
- * RoPE rotate-half, SwiGLU, GQA).  dtype applies to the weight matrices,
- * the KV cache and the activations fed to matrix products.  Norm gains and
- * the LoRA factors are always float32. */
+ * RoPE rotate-half, SwiGLU, GQA).  dtype is the storage type of the weight
+ * matrices and the KV cache.  The residual stream, norm gains, LoRA factors
+ * and logits are float32; with bf16, the activations that meet a weight
+ * matrix in a tensor-core product (and the queries and probabilities of the
+ * attention) enter it as a bf16 pair hi + lo, so the products carry the
+ * rounding of the stored weights and cache only. */
 typedef struct {
   int n_layers;       /* L */
   int d_model;        /* d, a multiple of 128 */
@@ -213,7 +216,8 @@ enum {
   DVI_BUF_LENS = 0,        /* int32 [B] committed KV length n per sequence */
   DVI_BUF_PENDING = 1,     /* int32 [B] pending (last committed) token */
   DVI_BUF_DRAFT_IDS = 2,   /* int32 [B][K+1]: pending, t~_1..t~_K of the last step */
-  DVI_BUF_LOG_U = 3,       /* dtype [cap][d] logged head inputs u = RMSNorm_final(h_k) */
+  DVI_BUF_LOG_U = 3,       /* logged head inputs u = RMSNorm_final(h_k): f32 [cap][d]; bf16
+                              [2][cap][d], a hi plane then a lo plane, u = hi + lo */
   DVI_BUF_LOG_LOGITS = 4,  /* f32 [cap][V] logged verifier logits */
   DVI_BUF_LOG_META = 5,    /* int32 [cap][6]: valid, a, r, i, prev_id, y* */
   DVI_BUF_GRAD_A = 6,      /* f32 [V][r] last dL/dA */
@@ -239,8 +243,9 @@ dvi_status dvi_timing(dvi_ctx* ctx, int enable);
 dvi_status dvi_get_timing(dvi_ctx* ctx, double* ms, int* counts);
 
 /* Y[M][n_out] = X[M][K] . W[n_out][K]^T through the library's projection
- * kernel (tcgen05 for bf16, FP32 FMA for f32), with X float32 (rounded to the
- * weight dtype first) and Y float32, on the context's stream.  M <= 256.
+ * kernel (tcgen05 for bf16, FP32 FMA for f32), with X float32 (for bf16
+ * weights carried as a bf16 pair hi + lo, about 16 significant bits) and Y
+ * float32, on the context's stream.  M <= 256.
  * A building block exposed for tests of the projection kernel itself. */
 dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in,
                       const float* d_x, int m_rows, float* d_y);

@@ -15,6 +15,12 @@ KV head floor(h * H_kv / H), RoPE "rotate-half" with theta = 10000 and
 RMSNorm eps = 1e-5.  Both heads read RMSNorm_final(h) (the model's frozen
 final norm).  Layer indices in the API are 0-based: the draft path is layers
 [0, k), the verify path [k, L).
+
+Storage precision: the bf16 workloads keep their KV cache in bf16 (two bytes
+per element: 16384 positions x 32 layers x 4096 x 2 tensors is the ~8 GB
+cache of the long-context workload), so with kv_dtype="bf16" every K/V row is
+rounded to the nearest bfloat16 when it is written to the cache; all other
+arithmetic stays in the model's dtype (fp64 by default).
 """
 from __future__ import annotations
 
@@ -46,6 +52,18 @@ def rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
     return np.concatenate([x1 * cos - x2 * sin, x2 * cos + x1 * sin], axis=-1)
 
 
+def to_bf16(a: np.ndarray) -> np.ndarray:
+    """Nearest bfloat16 value (ties to even) of every element, as float32.
+
+    bfloat16 is the top 16 bits of an IEEE float32; rounding adds half an
+    ulp of the kept part (minus one when the kept part is even) before the
+    low 16 bits are cleared.
+    """
+    b = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32)
+    bias = ((b >> np.uint32(16)) & np.uint32(1)) + np.uint32(0x7FFF)
+    return ((b + bias) & np.uint32(0xFFFF0000)).view(np.float32)
+
+
 def softmax(z: np.ndarray) -> np.ndarray:
     e = np.exp(z - z.max(axis=-1, keepdims=True))
     return e / e.sum(axis=-1, keepdims=True)
@@ -71,9 +89,11 @@ class KVCache:
 
 class OracleModel:
     def __init__(self, weights: Weights, shape: ModelShape, lora_gamma: float = 1.0,
-                 dtype=np.float64):
+                 dtype=np.float64, kv_dtype: str | None = None):
         self.s = shape
         self.dtype = dtype
+        assert kv_dtype in (None, "bf16")
+        self.kv_bf16 = kv_dtype == "bf16"
         self.gamma = lora_gamma
         c = lambda a: np.asarray(a, dtype=dtype)
         self.embed_w = c(weights.embed)
@@ -124,6 +144,8 @@ class OracleModel:
         k = rope(k, pos, s.rope_theta)
         if pos0 + R > cache.max_len:
             raise ValueError("KV cache capacity exceeded")
+        if self.kv_bf16:
+            k, v = to_bf16(k).astype(self.dtype), to_bf16(v).astype(self.dtype)
         cache.k[l, pos0:pos0 + R] = k
         cache.v[l, pos0:pos0 + R] = v
         o = self.attention(q, cache.k[l], cache.v[l], pos0)

@@ -112,7 +112,7 @@ __device__ void combine_splits(const AttnArgs& a, const float* all, size_t per, 
     L = fmaf(__ldcg(all + s * per + kAttnQ * hd + kAttnQ + qi), w, L);
     O = fmaf(__ldcg(all + s * per + qi * hd + d), w, O);
   }
-  DT<TO>::st(dst, O / L);
+  Act<TO>::st(dst, a.o_plane, O / L);
 }
 
 // ------------------------------------------------------------------ decode
@@ -293,7 +293,7 @@ __global__ void __launch_bounds__(128) attn_dec_kernel(const AttnArgs a, int wq_
     if (n_active == 1) {
       const int ii = qi / G, hh = qi % G;
       const int n = sl * a.rows_per_seq + i0 + ii;
-      DT<T>::st(static_cast<T*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, O / Ls);
+      Act<T>::st(static_cast<T*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, a.o_plane, O / Ls);
     } else {
       mine[qi * HD + d] = O;
       if (d == 0) {
@@ -329,12 +329,15 @@ __global__ void __launch_bounds__(128) attn_dec_kernel(const AttnArgs a, int wq_
     }
     const int ii = qi / G, hh = qi % G;
     const int n = sl * a.rows_per_seq + i0 + ii;
-    DT<T>::st(static_cast<T*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, O * cw[qi]);
+    Act<T>::st(static_cast<T*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d, a.o_plane,
+               O * cw[qi]);
   }
 }
 
 // ------------------------------------------------------------------ decode, bf16
-// Tensor-core decode attention (bf16 cache).  A CTA covers 16 query rows (the
+// Tensor-core decode attention (bf16 cache).  Queries and probabilities enter
+// the bf16 MMAs as hi + lo pairs, so only the cache itself is bf16-rounded.
+// A CTA covers 16 query rows (the
 // block's rows x the GQA heads of one KV head, zero-padded) and its split's
 // positions in 64-position chunks, double-buffered by TMA (128-byte swizzle,
 // so the fragment loads below are bank-conflict free).  Warp w owns chunk
@@ -404,8 +407,9 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   if (tid == 0)
     for (int ch = 0; ch < min(kDecStages, nch); ++ch) issue(ch);
 
-  // Q fragments (rows gq and gq+8), scaled by 1/sqrt(hd) * log2(e), bf16
-  uint32_t qa[HD / 16][4];
+  // Q fragments (rows gq and gq+8), scaled by 1/sqrt(hd) * log2(e), as a
+  // bf16 pair hi + lo (two products per K fragment keep 16 bits of q)
+  uint32_t qa[HD / 16][4], qb[HD / 16][4];
   int lim0 = -1, lim1 = -1;
   {
     const float sc = a.scale * kLog2e;
@@ -426,7 +430,9 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
       for (int r = 0; r < 4; ++r) {
         const float* qr = qrow[r & 1];
         const int col = kk * 16 + (r >> 1) * 8 + 2 * tq;
-        qa[kk][r] = qr ? pack_bf16x2(qr[col] * sc, qr[col + 1] * sc) : 0u;
+        qa[kk][r] = 0u;
+        qb[kk][r] = 0u;
+        if (qr) split_bf16x2(qr[col] * sc, qr[col + 1] * sc, qa[kk][r], qb[kk][r]);
       }
     }
   }
@@ -444,11 +450,11 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
     const uint8_t* vs = ks + kBoxes * kBoxBytes;
     const int pc = p0 + ch * kChunkPos;
     // S = Q K^T for this warp's 16 positions (two n-tiles of 8)
-    float sacc[2][4];
+    float sacc[2][4], slo[2][4];   // q_hi K^T and q_lo K^T: independent MMA chains
 #pragma unroll
     for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-      for (int e = 0; e < 4; ++e) sacc[nt][e] = 0.f;
+      for (int e = 0; e < 4; ++e) sacc[nt][e] = slo[nt][e] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < HD / 16; ++kk) {
       const int box = (kk * 16) / 64, c = ((kk * 16) % 64) / 8;
@@ -459,8 +465,13 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
         const uint32_t b0 = *reinterpret_cast<const uint32_t*>(rowp + ((c ^ (pr & 7)) << 4) + 4 * tq);
         const uint32_t b1 = *reinterpret_cast<const uint32_t*>(rowp + (((c + 1) ^ (pr & 7)) << 4) + 4 * tq);
         mma_bf16_16816(sacc[nt], qa[kk], b0, b1);
+        mma_bf16_16816(slo[nt], qb[kk], b0, b1);
       }
     }
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) sacc[nt][e] += slo[nt][e];
     // mask, online softmax (rows gq and gq+8; columns spread over the 4 lanes tq)
     float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
@@ -481,7 +492,7 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
     // a row with nothing visible so far keeps its state untouched
     const float c0 = (mn0 == -INFINITY) ? 1.f : (m0 == -INFINITY ? 0.f : exp2f(m0 - mn0));
     const float c1 = (mn1 == -INFINITY) ? 1.f : (m1 == -INFINITY ? 0.f : exp2f(m1 - mn1));
-    uint32_t pa[4];
+    uint32_t pa[4], pb[4];   // P as a bf16 pair hi + lo
     {
       float pv[2][4];
 #pragma unroll
@@ -493,10 +504,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
         }
       l0 = l0 * c0 + ((pv[0][0] + pv[0][1]) + (pv[1][0] + pv[1][1]));
       l1 = l1 * c1 + ((pv[0][2] + pv[0][3]) + (pv[1][2] + pv[1][3]));
-      pa[0] = pack_bf16x2(pv[0][0], pv[0][1]);
-      pa[1] = pack_bf16x2(pv[0][2], pv[0][3]);
-      pa[2] = pack_bf16x2(pv[1][0], pv[1][1]);
-      pa[3] = pack_bf16x2(pv[1][2], pv[1][3]);
+      split_bf16x2(pv[0][0], pv[0][1], pa[0], pb[0]);
+      split_bf16x2(pv[0][2], pv[0][3], pa[1], pb[1]);
+      split_bf16x2(pv[1][0], pv[1][1], pa[2], pb[2]);
+      split_bf16x2(pv[1][2], pv[1][3], pa[3], pb[3]);
     }
     m0 = mn0;
     m1 = mn1;
@@ -518,7 +529,9 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
       uint32_t r[4];
       ldmatrix_x4_trans(r, addr);
       mma_bf16_16816(o[nt], pa, r[0], r[1]);
+      mma_bf16_16816(o[nt], pb, r[0], r[1]);
       mma_bf16_16816(o[nt + 1], pa, r[2], r[3]);
+      mma_bf16_16816(o[nt + 1], pb, r[2], r[3]);
     }
     __syncthreads();                      // stage `st` consumed by every warp
     if (tid == 0 && ch + kDecStages < nch) issue(ch + kDecStages);
@@ -600,8 +613,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
     }
     const int ii = qi / G, hh = qi % G;
     const int n = sl * a.rows_per_seq + i0 + ii;
-    DT<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
-                          O / Ls);
+    Act<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
+                           a.o_plane, O / Ls);
   }
   cluster.sync();   // every rank keeps its shared memory until all have read it
 }
@@ -744,8 +757,8 @@ __global__ void __launch_bounds__(128, 2) attn_smem_kernel(const AttnArgs a) {
       if (qi < Q) {
         const int ii = qi / G, hh = qi % G;
         const int n = sl * a.rows_per_seq + i0 + ii;
-        DT<TO>::st(static_cast<TO*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * hd + d_pv,
-                   o_acc[u] / l_s[qi]);
+        Act<TO>::st(static_cast<TO*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * hd + d_pv, a.o_plane,
+                    o_acc[u] / l_s[qi]);
       }
     }
     return;

@@ -44,6 +44,39 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
+// Split of an f32 value into a bf16 pair v ~= hi + lo (hi = bf16(v),
+// lo = bf16(v - hi)): 16 significant bits instead of 8.  Matrix-product
+// operands that are activations travel in this form, so a bf16 tensor-core
+// product against them carries the rounding of the weights only.
+__device__ __forceinline__ void split_bf16(float v, __nv_bfloat16& hi, __nv_bfloat16& lo) {
+  hi = __float2bfloat16_rn(v);
+  lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+// Two packed pairs: (hi(a), hi(b)) and (lo(a), lo(b)).
+__device__ __forceinline__ void split_bf16x2(float a, float b, uint32_t& hi, uint32_t& lo) {
+  hi = pack_bf16x2(a, b);
+  lo = pack_bf16x2(a - bf16_lo(hi), b - bf16_hi(hi));
+}
+
+// Activation rows that feed a matrix product.  bf16: two planes `plane`
+// elements apart hold hi and lo of every value; f32: one plane, the value.
+template <typename T> struct Act;
+template <> struct Act<float> {
+  static __device__ __forceinline__ float ld(const float* p, size_t) { return *p; }
+  static __device__ __forceinline__ void st(float* p, size_t, float v) { *p = v; }
+};
+template <> struct Act<__nv_bfloat16> {
+  static __device__ __forceinline__ float ld(const __nv_bfloat16* p, size_t plane) {
+    return __bfloat162float(p[0]) + __bfloat162float(p[plane]);
+  }
+  static __device__ __forceinline__ void st(__nv_bfloat16* p, size_t plane, float v) {
+    __nv_bfloat16 hi, lo;
+    split_bf16(v, hi, lo);
+    p[0] = hi;
+    p[plane] = lo;
+  }
+};
+
 // ---------------------------------------------------------------- reductions
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll

@@ -179,13 +179,15 @@ size_t layout(dvi_ctx* c, char* base) {
   c->ss_ver = reinterpret_cast<float*>(take(sizeof(float) * st * B * K));
   c->x_pf = reinterpret_cast<float*>(take(sizeof(float) * c->chunk * d));
   c->ss_pf = reinterpret_cast<float*>(take(sizeof(float) * st * c->chunk));
-  c->xg_dr = take(e * B * d);
-  c->xg_ver = take(e * B * K * d);
-  c->xg_pf = take(e * c->chunk * d);
+  // activation rows feeding matrix products: bf16 keeps a hi and a lo plane
+  const size_t pl = c->tc ? 2 : 1;
+  c->xg_dr = take(pl * e * B * d);
+  c->xg_ver = take(pl * e * B * K * d);
+  c->xg_pf = take(pl * e * c->chunk * d);
   c->q = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * c->nq));
   c->bu = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * (r > 0 ? r : 1)));
-  c->attn_o = take(e * c->M_max * c->nq);
-  c->ffn_h = take(e * c->M_max * c->F);
+  c->attn_o = take(pl * e * c->M_max * c->nq);
+  c->ffn_h = take(pl * e * c->M_max * c->F);
   c->amax = reinterpret_cast<unsigned long long*>(take(sizeof(unsigned long long) * c->M_max));
   const size_t kv = static_cast<size_t>(c->L) * B * c->Hkv * c->max_len * c->hd;
   c->kcache = take(e * kv);
@@ -195,7 +197,7 @@ size_t layout(dvi_ctx* c, char* base) {
   c->proj_counters = reinterpret_cast<int*>(take(sizeof(int) * c->n_proj_counters));
   c->attn_part = reinterpret_cast<float*>(take(sizeof(float) * c->attn_part_floats));
   c->attn_ctr = reinterpret_cast<int*>(take(sizeof(int) * c->n_attn_ctr));
-  c->log_u = take(e * c->cap_rows * d);
+  c->log_u = take(pl * e * c->cap_rows * d);
   c->log_logits = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
   c->Z = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
   c->rowstat = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * 8));
@@ -366,6 +368,28 @@ ProjMaps with_act(const ProjMaps& w, const CUtensorMap* act) {
   return m;
 }
 
+// Rows of an activation buffer: with bf16 its lo plane starts that many rows
+// after its hi plane.
+int act_rows(const dvi_ctx* c, const void* buf) {
+  if (buf == c->xg_dr) return c->B;
+  if (buf == c->xg_ver) return c->B * c->K;
+  if (buf == c->xg_pf) return c->chunk;
+  if (buf == c->attn_o || buf == c->ffn_h) return c->M_max;
+  if (buf == c->log_u) return c->cap_rows;
+  return 0;
+}
+size_t act_plane(const dvi_ctx* c, const void* buf, int ld) {
+  return c->tc ? static_cast<size_t>(act_rows(c, buf)) * ld : 0;
+}
+
+// launch_proj with the plane offsets of the context's activation buffers.
+cudaError_t launch_proj_ctx(const dvi_ctx* c, ProjArgs a, const ProjMaps* m, cudaStream_t s) {
+  if (c->tc && a.b_mode == B_ACT) a.act_lo = act_rows(c, a.act);
+  if (a.xg_out) a.xg_plane = act_plane(c, a.xg_out, a.ld_xg);
+  if (a.h_out) a.h_plane = act_plane(c, a.h_out, a.ld_h);
+  return launch_proj(a, m, s);
+}
+
 // One decoder layer on the pass's rows.  `g_last` is the gain of whatever
 // consumes the pass's residual after this layer (the next layer's attention
 // norm, or the final norm before a head).
@@ -398,7 +422,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.n_kv_heads = ctx->Hkv;
   a.rope = ctx->rope;
   if (tc) pm = with_act(ctx->maps[l].qkv, ps.xg_map);
-  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
+  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
   // block-causal multi-query attention
   AttnArgs t{};
   t.q = ctx->q;
@@ -428,6 +452,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   t.kv_row0 = static_cast<long long>(l) * ctx->B * ctx->Hkv * ctx->max_len;
   t.kmap = &ctx->map_kc;
   t.vmap = &ctx->map_vc;
+  t.o_plane = act_plane(ctx, ctx->attn_o, ctx->nq);
   DVI_CUDA(launch_attn(t, s));
   // x += W_o . attn, then xg = x * ffn_norm for the FFN
   a = base_args(ctx, EPI_RESID, ctx->p_o, ps);
@@ -444,7 +469,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.xg_out = ps.xg;
   a.ld_xg = ctx->d;
   if (tc) pm = with_act(ctx->maps[l].o, &ctx->map_attn_o);
-  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
+  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
   // h = SiLU(W_gate n) * (W_up n) with n = RMSNorm(x)
   a = base_args(ctx, EPI_GATEUP, ctx->p_gu, ps);
   a.act = ps.xg;
@@ -458,7 +483,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.h_out = ctx->ffn_h;
   a.ld_h = ctx->F;
   if (tc) pm = with_act(ctx->maps[l].gu, ps.xg_map);
-  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
+  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
   // x += W_down . h, then xg = x * (next norm's gain)
   a = base_args(ctx, EPI_RESID, ctx->p_down, ps);
   a.act = ctx->ffn_h;
@@ -474,7 +499,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.xg_out = ps.xg;
   a.ld_xg = ctx->d;
   if (tc) pm = with_act(ctx->maps[l].down, &ctx->map_ffn_h);
-  DVI_CUDA(launch_proj(a, tc ? &pm : nullptr, s));
+  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
   ctx->launches += 5;
   return DVI_OK;
 }
@@ -512,6 +537,7 @@ StepState step_state(dvi_ctx* c) {
   st.ss_dr_ld = c->B;
   st.g0 = norm_gain_before(c, 0);
   st.xg_dr = c->xg_dr;
+  st.xg_dr_plane = act_plane(c, c->xg_dr, c->d);
   st.embed = c->w.embed;
   st.amax = c->amax;
   st.out_ids = c->out_ids;
@@ -557,7 +583,7 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
   }
   ProjMaps pm{};
   if (ctx->tc) pm = with_act(draft ? ctx->head_s : ctx->head_v, act_map);
-  DVI_CUDA(launch_proj(a, ctx->tc ? &pm : nullptr, ctx->stream));
+  DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &pm : nullptr, ctx->stream));
   ctx->launches += 1;
   return DVI_OK;
 }
@@ -586,7 +612,9 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
     h.ss_copy_ld = ctx->B * ctx->K;
     h.g_copy = norm_gain_before(ctx, ctx->k);
     h.xg_copy = ctx->xg_ver;
+    h.xg_copy_plane = act_plane(ctx, ctx->xg_ver, ctx->d);
     h.log_u = ctx->log_u;
+    h.log_plane = act_plane(ctx, ctx->log_u, ctx->d);
     h.log_step = ctx->log_step;
     h.log_cap_steps = ctx->cap_steps;
     h.log_rows_per_step = ctx->B * ctx->K;
@@ -757,12 +785,13 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
     }
     ok = ok && mk(&ctx->head_v.m0, weights->lm_head, ctx->V, ctx->d) &&
          mk(&ctx->head_s.m0, weights->draft_head, ctx->V, ctx->d);
-    ok = ok && make_act_map(&ctx->map_xg_dr, ctx->xg_dr, ctx->B, ctx->d) &&
-         make_act_map(&ctx->map_xg_ver, ctx->xg_ver, ctx->B * ctx->K, ctx->d) &&
-         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, ctx->chunk, ctx->d) &&
-         make_act_map(&ctx->map_attn_o, ctx->attn_o, ctx->M_max, ctx->nq) &&
-         make_act_map(&ctx->map_ffn_h, ctx->ffn_h, ctx->M_max, ctx->F) &&
-         make_act_map(&ctx->map_log_u, ctx->log_u, ctx->cap_rows, ctx->d);
+    // each map covers both planes: rows [0, R) hi, [R, 2R) lo
+    ok = ok && make_act_map(&ctx->map_xg_dr, ctx->xg_dr, 2 * ctx->B, ctx->d) &&
+         make_act_map(&ctx->map_xg_ver, ctx->xg_ver, 2 * ctx->B * ctx->K, ctx->d) &&
+         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, 2 * ctx->chunk, ctx->d) &&
+         make_act_map(&ctx->map_attn_o, ctx->attn_o, 2 * ctx->M_max, ctx->nq) &&
+         make_act_map(&ctx->map_ffn_h, ctx->ffn_h, 2 * ctx->M_max, ctx->F) &&
+         make_act_map(&ctx->map_log_u, ctx->log_u, 2 * ctx->cap_rows, ctx->d);
     const long long kv_rows = static_cast<long long>(ctx->L) * ctx->B * ctx->Hkv * ctx->max_len;
     ok = ok && make_kv_map(&ctx->map_kc, ctx->kcache, kv_rows, ctx->hd) &&
          make_kv_map(&ctx->map_vc, ctx->vcache, kv_rows, ctx->hd);
@@ -811,6 +840,7 @@ dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tok
     e.ss_ld = ctx->chunk;
     e.g = norm_gain_before(ctx, 0);
     e.xg = ctx->xg_pf;
+    e.xg_plane = act_plane(ctx, ctx->xg_pf, ctx->d);
     e.ldxg = ctx->d;
     e.rows = rows;
     e.status = ctx->status;
@@ -880,6 +910,7 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   a.B = ctx->B;
   a.K = ctx->K;
   a.log_u = ctx->log_u;
+  a.log_plane = act_plane(ctx, ctx->log_u, ctx->d);
   a.log_logits = ctx->log_logits;
   a.log_meta = ctx->log_meta;
   a.log_step = ctx->log_step;
@@ -929,7 +960,7 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   p.gamma = ctx->cfg.lora_gamma;
   ProjMaps pm{};
   if (ctx->tc) pm = with_act(ctx->head_s, &ctx->map_log_u);
-  DVI_CUDA(launch_proj(p, ctx->tc ? &pm : nullptr, s));
+  DVI_CUDA(launch_proj_ctx(ctx, p, ctx->tc ? &pm : nullptr, s));
   DVI_CUDA(launch_update_rowstats(a, s));
   DVI_CUDA(launch_update_coef(a, s));
   if (full) {
@@ -1014,7 +1045,7 @@ dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes)
     case DVI_BUF_LENS: *dptr = ctx->lens; *bytes = sizeof(int) * ctx->B; break;
     case DVI_BUF_PENDING: *dptr = ctx->pending; *bytes = sizeof(int) * ctx->B; break;
     case DVI_BUF_DRAFT_IDS: *dptr = ctx->draft_ids; *bytes = sizeof(int) * ctx->B * (ctx->K + 1); break;
-    case DVI_BUF_LOG_U: *dptr = ctx->log_u; *bytes = e * ctx->cap_rows * ctx->d; break;
+    case DVI_BUF_LOG_U: *dptr = ctx->log_u; *bytes = (ctx->tc ? 2 : 1) * e * ctx->cap_rows * ctx->d; break;
     case DVI_BUF_LOG_LOGITS: *dptr = ctx->log_logits; *bytes = sizeof(float) * ctx->cap_rows * static_cast<size_t>(ctx->V); break;
     case DVI_BUF_LOG_META: *dptr = ctx->log_meta; *bytes = sizeof(int) * 6 * ctx->cap_rows; break;
     case DVI_BUF_GRAD_A: *dptr = ctx->grad_a; *bytes = sizeof(float) * static_cast<size_t>(ctx->V) * rr; break;
@@ -1086,7 +1117,7 @@ dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in, const 
   ProjMaps m{};
   if (ctx->tc && !make_weight_map(&m.m0, d_w, n_out, k_in))
     return fail(ctx, DVI_ERR_INVALID_ARG, "linear: TMA descriptor creation failed");
-  DVI_CUDA(launch_proj(a, ctx->tc ? &m : nullptr, ctx->stream));
+  DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &m : nullptr, ctx->stream));
   ctx->launches += 1;
   return DVI_OK;
 }

@@ -34,8 +34,10 @@ struct ProjArgs {
   const void* w1;
   const void* w2;
   int rows_q, rows_k, rows_v;
-  // B operand: rows act_row0 .. act_row0+M-1 of act[.][ld_act]
-  const void* act; int ld_act; int act_row0;
+  // B operand: rows act_row0 .. act_row0+M-1 of act[.][ld_act]; bf16
+  // activations hold a hi plane and, act_lo rows further, a lo plane
+  // (value = hi + lo), so the MMA runs over 2 n_pad columns
+  const void* act; int ld_act; int act_row0; int act_lo;
   // Optional RMSNorm scale applied to every accumulator in the epilogue:
   // rstd[n] = rsqrt(sum_t ss[t*ss_ld + n] / d_norm + eps) (the norm gain is
   // already folded into the activation rows).
@@ -54,9 +56,9 @@ struct ProjArgs {
   // EPI_RESID: x += y, per-tile sums of squares of the new x, and the next
   // projection's activation rows xg = x * g_next in the model dtype
   float* x_res; int ld_res; float* ss_out; int ss_out_ld;
-  const float* g_next; void* xg_out; int ld_xg;
+  const float* g_next; void* xg_out; int ld_xg; size_t xg_plane;
   // EPI_GATEUP
-  void* h_out; int ld_h;
+  void* h_out; int ld_h; size_t h_plane;
   // EPI_HEAD
   float* logits_out; int ld_logits;
   int logits_mode;            // 0 none, 1 row n -> logits_out[n], 2 replay-buffer slot
@@ -82,7 +84,8 @@ bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);
 struct AttnArgs {
   const float* q; int ld_q;          // rotated queries [M][H_q*hd]
   const void* kc; const void* vc;    // layer base of the caches [B][H_kv][max_len][hd]
-  void* o; int ld_o;                 // output [M][H_q*hd] in `o_dtype`
+  void* o; int ld_o;                 // output [M][H_q*hd] in `o_dtype` (bf16: hi/lo planes)
+  size_t o_plane;
   int o_dtype;
   int dtype;                         // cache dtype
   int n_heads, n_kv_heads, head_dim, max_len;
@@ -108,6 +111,7 @@ struct EmbedArgs {
   float* x; int ldx;                 // destination rows
   float* ss; int ss_ld;              // per-128-feature sums of squares [d/128][ss_ld]
   const float* g; void* xg; int ldxg;// activation rows x * g of the first projection (model dtype)
+  size_t xg_plane;
   int rows;
   int* status;
 };
@@ -122,8 +126,8 @@ struct HeadPrepArgs {
   int dtype;
   float* x_copy; int ld_copy; int copy_row_stride; int copy_row_off;
   float* ss_copy; int ss_copy_ld;
-  const float* g_copy; void* xg_copy;
-  void* log_u; const int* log_step; int log_cap_steps; int log_rows_per_step; int log_row_stride;
+  const float* g_copy; void* xg_copy; size_t xg_copy_plane;
+  void* log_u; size_t log_plane; const int* log_step; int log_cap_steps; int log_rows_per_step; int log_row_stride;
   int log_row_off; int log_enabled;
   const float* lora_b; float* bu; int r;
 };
@@ -134,6 +138,7 @@ struct StepState {
   int* lens; int* pending; int* draft_ids;      // [B][K+1]
   float* x_dr; float* ss_dr; int ss_dr_ld;
   const float* g0; void* xg_dr;                 // first layer's attention-norm gain, x * g0
+  size_t xg_dr_plane;
   const void* embed;
   unsigned long long* amax;
   int* out_ids; int* n_committed; int* n_accepted;
@@ -151,7 +156,7 @@ cudaError_t launch_reset_seq(const StepState& st, int seq, cudaStream_t s);
 // ---- drafter update (update.cu)
 struct UpdateArgs {
   int cap, V, d, r, dtype, B, K;
-  const void* log_u; const float* log_logits; int* log_meta; int* log_step;
+  const void* log_u; size_t log_plane; const float* log_logits; int* log_meta; int* log_step;
   float* Z;                                     // [cap][V] drafter logits
   float* rowstat;                               // [cap][8]
   float* coef;                                  // [cap][4] + globals

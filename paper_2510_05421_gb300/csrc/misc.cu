@@ -4,7 +4,8 @@
 //
 // Every residual row these kernels write is written with its per-128-feature
 // sums of squares (the next RMSNorm's statistics) and with x * g, the next
-// projection's activation row (the norm gain folded in, model dtype).
+// projection's activation row (the norm gain folded in; bf16 as a hi/lo pair
+// of planes).
 //
 // finalize_verify is the accept/commit/rollback step of Sec. 3.3: with
 // y*_{n+i} the verifier's argmax at block row i-1 and t~_i the drafts,
@@ -25,8 +26,8 @@ constexpr int kMaxTiles = 64;   // d <= 8192
 // per-tile sums of squares.  All of the row's loads are issued before any is
 // used (one memory round trip), then a single block barrier.
 template <typename T>
-__device__ void embed_row_block(const T* table, int tok, int d, float* x, const float* g, T* xg, float* ss,
-                                int ss_ld, int row, float* red) {
+__device__ void embed_row_block(const T* table, int tok, int d, float* x, const float* g, T* xg, size_t plane,
+                                float* ss, int ss_ld, int row, float* red) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nt = d / kTileRows;
   const T* src = table + static_cast<size_t>(tok) * d;
@@ -43,7 +44,7 @@ __device__ void embed_row_block(const T* table, int tok, int d, float* x, const 
     if (t < nt) {
       const int c = t * kTileRows + tid;
       x[c] = v[t];
-      DT<T>::st(xg + c, v[t] * gv[t]);
+      Act<T>::st(xg + c, plane, v[t] * gv[t]);
       const float s = warp_sum(v[t] * v[t]);
       if (lane == 0) red[t * 4 + warp] = s;
     }
@@ -67,7 +68,8 @@ __global__ void __launch_bounds__(128) embed_kernel(const EmbedArgs a) {
     tok = 0;
   }
   embed_row_block<T>(static_cast<const T*>(a.table), tok, a.d, a.x + static_cast<size_t>(row) * a.ldx, a.g,
-                     static_cast<T*>(a.xg) + static_cast<size_t>(row) * a.ldxg, a.ss, a.ss_ld, row, red);
+                     static_cast<T*>(a.xg) + static_cast<size_t>(row) * a.ldxg, a.xg_plane, a.ss, a.ss_ld, row,
+                     red);
 }
 
 cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s) {
@@ -128,7 +130,7 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
     if (lu) {
 #pragma unroll
       for (int t = 0; t < kMaxTiles; ++t)
-        if (t < nt) DT<T>::st(lu + t * kTileRows + tid, xv[t] * rstd * gv[t]);
+        if (t < nt) Act<T>::st(lu + t * kTileRows + tid, a.log_plane, xv[t] * rstd * gv[t]);
     }
     if (a.x_copy) {
       const int crow = row * a.copy_row_stride + a.copy_row_off;
@@ -142,7 +144,7 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
       for (int t = 0; t < kMaxTiles; ++t)
         if (t < nt) {
           xc[t * kTileRows + tid] = xv[t];
-          DT<T>::st(xgc + t * kTileRows + tid, xv[t] * gc[t]);
+          Act<T>::st(xgc + t * kTileRows + tid, a.xg_copy_plane, xv[t] * gc[t]);
         }
       for (int t = tid; t < nt; t += 128)
         a.ss_copy[static_cast<size_t>(t) * a.ss_copy_ld + crow] =
@@ -195,8 +197,8 @@ template <typename T>
 __device__ void embed_rows(const StepState& st, const int* toks, float* red) {
   for (int b = 0; b < st.B; ++b)
     embed_row_block<T>(static_cast<const T*>(st.embed), toks[b], st.d, st.x_dr + static_cast<size_t>(b) * st.d,
-                       st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(b) * st.d, st.ss_dr, st.ss_dr_ld, b,
-                       red);
+                       st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(b) * st.d, st.xg_dr_plane, st.ss_dr,
+                       st.ss_dr_ld, b, red);
 }
 
 template <typename T>
@@ -302,8 +304,8 @@ __global__ void __launch_bounds__(128) finalize_prefill_kernel(const StepState s
   }
   __syncthreads();
   embed_row_block<T>(static_cast<const T*>(st.embed), tok, st.d, st.x_dr + static_cast<size_t>(seq) * st.d,
-                     st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(seq) * st.d, st.ss_dr, st.ss_dr_ld,
-                     seq, red);
+                     st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(seq) * st.d, st.xg_dr_plane, st.ss_dr,
+                     st.ss_dr_ld, seq, red);
 }
 
 __global__ void reset_seq_kernel(const StepState st, int seq) {

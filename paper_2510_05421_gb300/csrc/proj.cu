@@ -7,11 +7,15 @@
 // token rows sit on the MMA's N dimension ("swap AB").
 //
 // bf16 (tcgen05): warp 4 streams the 128x64 weight tile and the matching
-// n_pad x 64 activation tile of each K block by TMA (128-byte swizzle, the
-// K-major layout tcgen05 reads) into a ring of shared-memory stages; warp 5
-// issues tcgen05.mma (M=128, N=n_pad, K=16) into a TMEM accumulator and frees
+// activation tiles of each K block by TMA (128-byte swizzle, the K-major
+// layout tcgen05 reads) into a ring of shared-memory stages; warp 5 issues
+// tcgen05.mma (M=128, N=n_pad, K=16) into a TMEM accumulator and frees
 // stages with tcgen05.commit; warps 0-3 then read TMEM and run the fused
-// epilogue.  A gate/up tile holds 64 rows of W_gate and the same 64 rows of
+// epilogue.  Activations are bf16 pairs hi + lo (two planes of the
+// activation buffer) whose rows sit next to each other in a stage, so each
+// K step's MMA (N = 2 n_pad) writes W.hi to accumulator columns [0, n_pad)
+// and W.lo to [n_pad, 2 n_pad); the epilogue adds the two, and the product
+// carries the rounding of the weights only.  A gate/up tile holds 64 rows of W_gate and the same 64 rows of
 // W_up (two 64-row TMA boxes), so SwiGLU pairs rows r and r+64 of one tile.
 // The RMSNorm feeding a projection is split in two: its gain is folded into
 // the activation rows by the kernel that produced them, and its 1/rms (a
@@ -57,8 +61,9 @@ __device__ __forceinline__ void row_seq_pos(const ProjArgs& p, int n, int& seq, 
   pos = p.lens[seq] + p.pos_off + n % p.rows_per_seq;
 }
 
-// rstd[n] for the token rows of the launch (1 when there is no norm).
-__device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int tid, int nthreads) {
+// rstd[n] for the token rows of the launch (1 when there is no norm), and
+// for the QKV flavour the cache position of every row.
+__device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int* posn, int tid, int nthreads) {
   for (int n = tid; n < p.M; n += nthreads) {
     float r = 1.f;
     if (p.ss) {
@@ -67,6 +72,11 @@ __device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int
       r = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
     }
     rstd[n] = r;
+    if (p.flavor == EPI_QKV) {
+      int seq, pos;
+      row_seq_pos(p, n, seq, pos);
+      posn[n] = pos;
+    }
   }
 }
 
@@ -80,8 +90,8 @@ __device__ __forceinline__ uint32_t valid_cols(const ProjArgs& p, int c0) {
 // subset of the valid ones) of one 128-feature tile.  Called by the 128
 // epilogue threads together (row = feature within tile).
 template <typename T>
-__device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, float (&v)[kChunk],
-                               const float* rstd, EpiSmem& es, uint32_t own) {
+__device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, float (&v)[kChunk],
+                               const float* rstd, const int* posn, EpiSmem& es, uint32_t own) {
   const int warp = row >> 5, lane = row & 31;
   if (p.ss) {
 #pragma unroll
@@ -106,8 +116,8 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
     for (int j = 0; j < kChunk; ++j) {
       const int n = c0 + j;
       if ((own >> j) & 1u) {
-        int seq, pos;
-        row_seq_pos(p, n, seq, pos);
+        const int seq = p.seq0 + n / p.rows_per_seq;
+        const int pos = posn[n];
         if (pos >= p.max_len || pos < 0) {
           flag_status(p.status, DVI_DEV_KV_FULL);
         } else {
@@ -139,7 +149,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
         float* xp = p.x_res + static_cast<size_t>(n) * p.ld_res + f;
         xn = *xp + v[j];
         *xp = xn;
-        if (p.xg_out) DT<T>::st(static_cast<T*>(p.xg_out) + static_cast<size_t>(n) * p.ld_xg + f, xn * g);
+        if (p.xg_out) Act<T>::st(static_cast<T*>(p.xg_out) + static_cast<size_t>(n) * p.ld_xg + f, p.xg_plane, xn * g);
       }
       sq[j] = xn * xn;
     }
@@ -166,7 +176,7 @@ __device__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, flo
         if ((own >> j) & 1u) {
           const float gt = es.stage[row][j];
           const float h = gt / (1.f + expf(-gt)) * es.stage[row + kGuRows][j];
-          DT<T>::st(static_cast<T*>(p.h_out) + static_cast<size_t>(n) * p.ld_h + f, h);
+          Act<T>::st(static_cast<T*>(p.h_out) + static_cast<size_t>(n) * p.ld_h + f, p.h_plane, h);
         }
       }
     }
@@ -266,13 +276,14 @@ __device__ __forceinline__ uint32_t tmem_cols(int n) {
   return c;
 }
 
-// Writes one 64-wide K block of the B operand from float32 rows (B_SOFT_F32).
+// Writes one 64-wide K block of the B operand from float32 rows (B_SOFT_F32):
+// the hi rows, then n_pad rows further the lo rows.
 __device__ __forceinline__ void produce_b_f32(const ProjArgs& p, uint8_t* bs, int kb, int tid) {
   const int nslots = p.n_pad * 8;
   for (int slot = tid; slot < nslots; slot += kTileRows) {
     const int n = slot >> 3, c = slot & 7;
     const int k0 = kb * kKBlock + c * 8;
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
+    uint4 val = make_uint4(0u, 0u, 0u, 0u), lo = val;
     if (n < p.M && k0 < p.K) {
       const float* src = static_cast<const float*>(p.act) + static_cast<size_t>(p.act_row0 + n) * p.ld_act + k0;
       float f[8];
@@ -284,15 +295,19 @@ __device__ __forceinline__ void produce_b_f32(const ProjArgs& p, uint8_t* bs, in
 #pragma unroll
         for (int e = 0; e < 8; ++e) f[e] = (k0 + e < p.K) ? src[e] : 0.f;
       }
-      val = make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
-                       pack_bf16x2(f[6], f[7]));
+      split_bf16x2(f[0], f[1], val.x, lo.x);
+      split_bf16x2(f[2], f[3], val.y, lo.y);
+      split_bf16x2(f[4], f[5], val.z, lo.z);
+      split_bf16x2(f[6], f[7], val.w, lo.w);
     }
     *reinterpret_cast<uint4*>(bs + n * 128 + ((c ^ (n & 7)) << 4)) = val;
+    const int nl = n + p.n_pad;
+    *reinterpret_cast<uint4*>(bs + nl * 128 + ((c ^ (nl & 7)) << 4)) = lo;
   }
 }
 
 // ------------------------------------------------------------------ tcgen05
-__global__ void __launch_bounds__(192, 3)
+__global__ void __launch_bounds__(192, 2)
     proj_tc_kernel(const __grid_constant__ CUtensorMap m0, const __grid_constant__ CUtensorMap m1,
                    const __grid_constant__ CUtensorMap m2, const __grid_constant__ CUtensorMap mb,
                    const ProjArgs p, int stages) {
@@ -300,7 +315,7 @@ __global__ void __launch_bounds__(192, 3)
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
   constexpr int abytes = 16384;
-  const int bbytes = p.n_pad * 128;
+  const int bbytes = 2 * p.n_pad * 128;   // hi rows, then lo rows
   uint8_t* sA = base;
   uint8_t* sB = base + stages * abytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(sB + stages * bbytes);
@@ -308,6 +323,7 @@ __global__ void __launch_bounds__(192, 3)
   uint64_t* done = empty + stages;
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   float* rstd = reinterpret_cast<float*>(tmem_holder + 4);
+  int* posn = reinterpret_cast<int*>(rstd + kMaxTokens);
   // after `done` the A stages are free: epilogue scratch, then this split's
   // partial tile [n_pad][128] for the cluster reduction
   EpiSmem& es = *reinterpret_cast<EpiSmem*>(sA);
@@ -317,7 +333,7 @@ __global__ void __launch_bounds__(192, 3)
   const int tile = blockIdx.x / p.n_splits, split = blockIdx.x % p.n_splits;
   const int kb0 = split * p.kb_per_split;
   const int nkb = min(p.kb_per_split, p.kb_total - kb0);
-  const uint32_t ncols = tmem_cols(p.n_pad);
+  const uint32_t ncols = tmem_cols(2 * p.n_pad);
   const bool soft_b = p.b_mode == B_SOFT_F32;
   const bool gu = p.flavor == EPI_GATEUP;
 
@@ -372,8 +388,10 @@ __global__ void __launch_bounds__(192, 3)
         if (soft_b) return;
         const int s = i % stages;
         const int x = (kb0 + i) * kKBlock;
-        for (int b = 0; b < nbox; ++b)
+        for (int b = 0; b < nbox; ++b) {
           tma_load_2d(sB + s * bbytes + b * 2048, &mb, x, p.act_row0 + b * 16, &full[s], 0ull);
+          tma_load_2d(sB + s * bbytes + (nbox + b) * 2048, &mb, x, p.act_lo + p.act_row0 + b * 16, &full[s], 0ull);
+        }
       };
       // The first stages' weight tiles do not depend on earlier kernels.
       const int pre = p.prefetch_a ? min(stages, nkb) : 0;
@@ -401,7 +419,10 @@ __global__ void __launch_bounds__(192, 3)
   } else if (warp == 5) {
     // ---------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_m128(static_cast<uint32_t>(p.n_pad));
+      // hi and lo rows are adjacent in the stage: one MMA of N = 2 n_pad
+      // covers both while N <= 256, else one MMA each
+      const bool fused_lo = 2 * p.n_pad <= 256;
+      const uint32_t idesc = idesc_bf16_m128(static_cast<uint32_t>(fused_lo ? 2 * p.n_pad : p.n_pad));
       for (int i = 0; i < nkb; ++i) {
         const int s = i % stages;
         const uint32_t ph = (i / stages) & 1;
@@ -409,9 +430,15 @@ __global__ void __launch_bounds__(192, 3)
         tc_fence_after();
         const uint32_t a = smem_u32(sA + s * abytes);
         const uint32_t b = smem_u32(sB + s * bbytes);
+        const uint32_t blo = b + static_cast<uint32_t>(p.n_pad) * 128u;
 #pragma unroll
-        for (int kk = 0; kk < kKBlock / 16; ++kk)
-          tc_mma_bf16(tmem, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc, (i | kk) != 0);
+        for (int kk = 0; kk < kKBlock / 16; ++kk) {
+          const uint64_t ad = smem_desc_sw128(a + kk * 32);
+          tc_mma_bf16(tmem, ad, smem_desc_sw128(b + kk * 32), idesc, (i | kk) != 0);
+          if (!fused_lo)
+            tc_mma_bf16(tmem + static_cast<uint32_t>(p.n_pad), ad, smem_desc_sw128(blo + kk * 32), idesc,
+                        (i | kk) != 0);
+        }
         tc_commit(&empty[s]);
       }
       tc_commit(done);
@@ -432,7 +459,7 @@ __global__ void __launch_bounds__(192, 3)
         if (lane == 0) mbar_arrive(&full[s]);
       }
     }
-    compute_rstd(p, rstd, tid, kTileRows);
+    compute_rstd(p, rstd, posn, tid, kTileRows);
     named_bar(1, kTileRows);
     ok = mbar_wait(done, 0, p.status);
     tc_fence_after();
@@ -440,9 +467,14 @@ __global__ void __launch_bounds__(192, 3)
     const int nchunks = (p.M + kChunk - 1) / kChunk;
     float v[kChunk];
     for (int c = 0; c < nchunks; ++c) {
+      float vl[kChunk];
       tmem_ld16(lane_base + c * kChunk, v);
+      tmem_ld16(lane_base + p.n_pad + c * kChunk, vl);
+#pragma unroll
+      for (int j = 0; j < kChunk; ++j) v[j] += vl[j];
       if (p.n_splits == 1) {
-        if (ok) epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es, valid_cols(p, c * kChunk));
+        if (ok)
+          epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, valid_cols(p, c * kChunk));
       } else {
 #pragma unroll
         for (int j = 0; j < kChunk; ++j)
@@ -491,7 +523,7 @@ __global__ void __launch_bounds__(192, 3)
             v[j] = acc;
           }
         }
-        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, es, own);
+        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, own);
       }
     }
     cluster.sync();   // every rank keeps its shared memory until all have read it
@@ -503,6 +535,7 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
   __shared__ float Ws[kTileRows][kKBlockF32 + 1];
   __shared__ float Bs[kChunk][kKBlockF32];
   __shared__ float rstd[kChunk];
+  __shared__ int posn[kChunk];
   __shared__ EpiSmem es;
   griddep_launch();
   griddep_wait();
@@ -540,6 +573,11 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
       r = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
     }
     rstd[tid] = r;
+    if (p.flavor == EPI_QKV && n < p.M) {
+      int seq, pos;
+      row_seq_pos(p, n, seq, pos);
+      posn[tid] = pos;
+    }
   }
   __syncthreads();
   float acc[kChunk];
@@ -568,10 +606,12 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
     __syncthreads();
   }
   const int row = tid;
-  // epilogue_chunk indexes rstd by token; shift so rstd[c0 + j] is this tile's
+  // epilogue_chunk indexes rstd and positions by token; shift so that
+  // rstd[c0 + j] is this tile's
   float* rs = rstd - c0;
+  const int* ps = posn - c0;
   if (p.n_splits == 1) {
-    epilogue_chunk<float>(p, tile, row, c0, acc, rs, es, valid_cols(p, c0));
+    epilogue_chunk<float>(p, tile, row, c0, acc, rs, ps, es, valid_cols(p, c0));
     return;
   }
   const size_t reg = static_cast<size_t>(kTileRows) * kChunk;
@@ -583,15 +623,14 @@ __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
   const float* all = p.part + static_cast<size_t>(ci) * p.n_splits * reg;
 #pragma unroll
   for (int j = 0; j < kChunk; ++j) acc[j] = sum_splits(all + j * kTileRows + row, reg, p.n_splits);
-  epilogue_chunk<float>(p, tile, row, c0, acc, rs, es, valid_cols(p, c0));
+  epilogue_chunk<float>(p, tile, row, c0, acc, rs, ps, es, valid_cols(p, c0));
 }
 
 // ------------------------------------------------------------------ host
 // Work per launch: n_tiles output tiles x n_splits K ranges.  bf16: one wave
-// of at most two CTAs per SM (a third fits, which lets the next kernel's CTAs
-// start streaming weights under programmatic dependent launch), splits only
-// while tiles are too few, at most 8 (a portable cluster) and at least 4 K
-// blocks each.  f32: balanced waves of the FFMA kernel.
+// of at most two CTAs per SM (the shared-memory ring of four stages admits
+// two), splits only while tiles are too few, at most 8 (a portable cluster)
+// and at least 4 K blocks each.  f32: balanced waves of the FFMA kernel.
 void plan_splits(ProjArgs& a, int n_sms, bool tc) {
   if (a.flavor == EPI_QKV)
     a.n_tiles = a.rows_q / kTileRows + a.rows_k / kTileRows + a.rows_v / kTileRows;
@@ -632,9 +671,10 @@ size_t proj_partial_floats(const ProjArgs& a, bool tc) {
 }
 
 static int tc_stages(int n_pad, size_t* smem_bytes) {
-  const int per = 16384 + n_pad * 128;
-  const int fixed = 1024 /*align*/ + 1024 /*barriers, tmem slot*/ + 4 * kMaxTokens /*rstd*/;
-  int stages = n_pad <= 64 ? 4 : std::max(2, std::min(8, (112 * 1024 - fixed) / per));
+  const int per = 16384 + 2 * n_pad * 128;   // weight tile + hi and lo activation rows
+  const int fixed = 1024 /*align*/ + 1024 /*barriers, tmem slot*/ + 8 * kMaxTokens /*rstd, positions*/;
+  // two CTAs per SM while the ring keeps at least three stages
+  int stages = std::max(2, std::min(4, (112 * 1024 - fixed) / per));
   *smem_bytes = static_cast<size_t>(fixed) + static_cast<size_t>(stages) * per;
   return stages;
 }

@@ -58,7 +58,7 @@ __global__ void __launch_bounds__(128) update_prep_kernel(const UpdateArgs a) {
   for (int j = warp; j < a.r; j += 4) {
     const float* br = a.lora_b + static_cast<size_t>(j) * a.d;
     float acc = 0.f;
-    for (int c = lane; c < a.d; c += 32) acc = fmaf(br[c], DT<T>::ld(u + c), acc);
+    for (int c = lane; c < a.d; c += 32) acc = fmaf(br[c], Act<T>::ld(u + c, a.log_plane), acc);
     acc = warp_sum(acc);
     if (lane == 0) a.ub[n * a.r + j] = acc;
   }
@@ -321,8 +321,8 @@ __global__ void __launch_bounds__(128) update_grad_b_kernel(const UpdateArgs a) 
     float acc = 0.f;
     for (int n = 0; n < a.cap; ++n) {
       if (!row_valid(a, n)) continue;
-      acc = fmaf(a.ga[n * a.r + j], DT<T>::ld(static_cast<const T*>(a.log_u) + static_cast<size_t>(n) * a.d + c),
-                 acc);
+      acc = fmaf(a.ga[n * a.r + j],
+                 Act<T>::ld(static_cast<const T*>(a.log_u) + static_cast<size_t>(n) * a.d + c, a.log_plane), acc);
     }
     const float g = a.gamma * acc;
     const size_t i = static_cast<size_t>(j) * a.d + c;
@@ -376,7 +376,9 @@ __global__ void __launch_bounds__(128) update_gw_kernel(const UpdateArgs a) {
       float4 u = make_float4(0.f, 0.f, 0.f, 0.f);
       if (n < a.cap && col < a.d && row_valid(a, n)) {
         const T* src = U + static_cast<size_t>(n) * a.d + col;
-        u = make_float4(DT<T>::ld(src), DT<T>::ld(src + 1), DT<T>::ld(src + 2), DT<T>::ld(src + 3));
+        const size_t pl = a.log_plane;
+        u = make_float4(Act<T>::ld(src, pl), Act<T>::ld(src + 1, pl), Act<T>::ld(src + 2, pl),
+                        Act<T>::ld(src + 3, pl));
       }
       us[row][i % (kGwCols / 4)] = u;
     }

@@ -217,6 +217,9 @@ class DVIEngine:
         self.n_accepted = torch.zeros(batch, dtype=torch.int32, device=self.device)
         self.ar_ids = torch.zeros(batch, dtype=torch.int32, device=self.device)
         self.first = torch.zeros(batch, dtype=torch.int32, device=self.device)
+        self.log_steps = log_steps
+        self._logging = True        # the library logs by default
+        self._logged = 0            # decode steps logged since the last update
 
     # -- calls ------------------------------------------------------------
     def _check(self, rc, what):
@@ -239,14 +242,18 @@ class DVIEngine:
         rc = lib().dvi_draft_verify_commit(self.ctx, _ptr(self.out_ids), _ptr(self.n_committed),
                                            _ptr(self.n_accepted))
         self._check(rc, "dvi_draft_verify_commit")
+        if self._logging:
+            self._logged += 1
         return self.out_ids, self.n_committed, self.n_accepted
 
     def update(self, hyper, keep_grad_w: bool = False):
         c = hyper if isinstance(hyper, UpdateConfigC) else update_config(hyper, keep_grad_w)
         self._check(lib().dvi_update_drafter(self.ctx, ctypes.byref(c)), "dvi_update_drafter")
+        self._logged = 0
 
     def log(self, enable: bool):
         self._check(lib().dvi_log(self.ctx, 1 if enable else 0), "dvi_log")
+        self._logging = bool(enable)
 
     def ar_step(self) -> torch.Tensor:
         self._check(lib().dvi_ar_step(self.ctx, _ptr(self.ar_ids)), "dvi_ar_step")
@@ -308,7 +315,8 @@ class DVIEngine:
 
         Each prompt is copied from pinned host memory, prefilled, then steps
         run until every sequence has n_gen tokens; an update of the drafter
-        runs every `update_every` steps.  Replay-buffer logging is on when
+        runs after every `update_every` logged steps of the engine (counted
+        across calls, so a later call continues the drafter's schedule).  Replay-buffer logging is on when
         updates are requested (or when `log` says so).  Returns (tokens per
         sequence, per-step accept lengths [steps, B], bytes h2d, bytes d2h).
         """
@@ -348,7 +356,7 @@ class DVIEngine:
                 toks[b].extend(out_h[b, :int(cnt_h[b])].tolist())
             mats.append(acc_h.tolist())
             step += 1
-            if update_every and hyper is not None and step % update_every == 0:
+            if update_every and hyper is not None and self._logged >= update_every:
                 self.update(hyper)
         return [t[:n_gen] for t in toks], np.array(mats), h2d, d2h
 

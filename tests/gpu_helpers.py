@@ -21,6 +21,15 @@ def engine_for(w, W=None, dtype=None, use_graphs=True, max_seq_len=None, batch=N
     return eng, W, dw
 
 
+def logged_u(eng, w):
+    """The replay buffer's head inputs u as float64 [cap][d] (bf16: hi + lo planes)."""
+    d = w.shape.d_model
+    if eng.dtype == "bf16":
+        lu = eng.buffer("LOG_U", torch.bfloat16).view(2, -1, d).double()
+        return (lu[0] + lu[1]).cpu().numpy()
+    return eng.buffer("LOG_U", torch.float32).view(-1, d).double().cpu().numpy()
+
+
 def rounded_weights(W):
     """The bf16-rounded weights promoted back to float32 (the oracle's view of a bf16 run)."""
     return W.map(bf16_round)

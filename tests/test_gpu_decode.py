@@ -5,7 +5,8 @@
   gradients within 1e-3 relative (Sec. 3.3, Sec. 3.4).
 * bf16: the GPU's DVI stream equals the GPU's own greedy AR stream bit for
   bit (lossless), and the logged verifier logits are within 3e-2 of the
-  oracle's teacher-forced logits on the bf16-rounded weights.
+  oracle's teacher-forced logits on the bf16-rounded weights with a bf16 KV
+  cache (the workloads' storage types).
 * Batch of ragged prompts, CUDA-graph vs eager launch, and the full-acceptance
   case (drafter = the whole model).
 """
@@ -125,7 +126,7 @@ def test_bf16_dvi_equals_gpu_ar_and_oracle_teacher_forced(graphs):
     assert all(0 <= x <= w.k_spec for x in mats[:, 0])
     eng.close()
     # teacher-forced verifier logits of the oracle on the bf16-rounded weights
-    model = OracleModel(rounded_weights(W), w.shape, w.lora_gamma)
+    model = OracleModel(rounded_weights(W), w.shape, w.lora_gamma, kv_dtype="bf16")
     seq = np.concatenate([P[0], np.array(toks[0], dtype=np.int32)])
     ref = teacher_forced_logits(model, seq)
     plen = len(P[0])

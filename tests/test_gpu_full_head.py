@@ -18,7 +18,7 @@ import torch
 from oracle import OracleModel, dvi_generate
 from oracle.update import AdamState, adam_step, grad_logits, head_logits, objective_weights, param_grads
 from workloads import workload, make_weights, make_prompts, UpdateHyper
-from gpu_helpers import engine_for, rounded_weights
+from gpu_helpers import engine_for, logged_u, rounded_weights
 from test_gpu_decode import Recorder, _bf16_case
 
 pytestmark = pytest.mark.gpu
@@ -101,7 +101,7 @@ def test_bf16_full_head_lossless_and_gradient():
     V, d = w.shape.vocab, w.shape.d_model
     meta = eng.buffer("LOG_META", torch.int32).view(-1, 6).cpu().numpy()
     lg = eng.buffer("LOG_LOGITS", torch.float32).view(-1, V).cpu().numpy().astype(np.float64)
-    lu = eng.buffer("LOG_U", torch.bfloat16).view(-1, d).float().cpu().numpy().astype(np.float64)
+    lu = logged_u(eng, w)
     w_s = dw.draft_head.float().cpu().numpy().astype(np.float64)
     eng.update(hyper, keep_grad_w=True)
     eng.sync()

@@ -1,0 +1,132 @@
+"""The decode path at the full sizes of the measured workloads.
+
+Shapes, split points, K, prompt lengths and launch configuration (CUDA
+graphs, KV capacity as the benchmark sizes it) are the workloads' own; only
+the number of generated tokens is cut.  At these sizes the oracle is used on
+sampled outputs, and the rest is checked through properties that hold at any
+size:
+
+* losslessness (Sec. 3.3): the committed DVI stream equals the GPU's own
+  greedy autoregressive stream bit for bit, with the drafter training online;
+* teacher-forced verifier logits of the first step's verify rows against the
+  oracle (float32 arithmetic on the bf16-rounded weights, bf16 KV cache),
+  within 3e-2 (1B and 7B);
+* the 8-sequence ragged batch over two prompt waves whose drafter state
+  carries over, and the 16K-token prompt with K = 8.
+"""
+import functools
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import OracleModel
+from workloads import workload, make_weights, make_prompts
+from gpu_helpers import rounded_weights, teacher_forced_logits
+
+pytestmark = pytest.mark.gpu
+GEN = 24
+
+
+@functools.lru_cache(maxsize=1)
+def _weights(name):
+    from paper_2510_05421_gb300 import DeviceWeights
+    w = workload(name)
+    W = make_weights(w)
+    return W, DeviceWeights.from_host(W, w.dtype)
+
+
+def _engine(w, dw, max_seq_len):
+    from paper_2510_05421_gb300 import DVIEngine
+    return DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=w.k_spec, split_k=w.split_k,
+                     lora_rank=w.lora_rank, lora_gamma=w.lora_gamma, max_seq_len=max_seq_len,
+                     log_steps=w.update_every)
+
+
+def _capacity(w, P):
+    # as the benchmark sizes the KV cache: prompt + K per generated token + slack
+    return max(len(p) for p in P) + w.gen_tokens * w.k_spec + 64
+
+
+def _lossless(w, dw, P, n_gen=GEN):
+    eng = _engine(w, dw, _capacity(w, P))
+    ar = eng.generate_ar(P, n_gen)
+    eng.close()
+    eng = _engine(w, dw, _capacity(w, P))
+    toks, mats, _, _ = eng.generate(P, n_gen, update_every=w.update_every, hyper=w.update)
+    st = eng.stats()
+    eng.close()
+    assert st["device_status"] == 0, st["device_flags"]
+    for b in range(len(P)):
+        assert toks[b] == list(ar[b]), b
+    assert ((mats >= 0) & (mats <= w.k_spec)).all()
+    return toks, mats
+
+
+def _first_step_logits(w, dw, W, P):
+    """Verify-row logits of the first decode step: GPU log against the oracle."""
+    eng = _engine(w, dw, _capacity(w, P))
+    toks, _, _, _ = eng.generate(P, 10 ** 6, max_steps=1, log=True)
+    eng.sync()
+    meta = eng.buffer("LOG_META", torch.int32).view(-1, 6).cpu().numpy()
+    lg = eng.buffer("LOG_LOGITS", torch.float32).view(-1, w.shape.vocab).cpu().numpy()
+    eng.close()
+    rows = [i for i in range(w.k_spec) if meta[i, 0]]
+    assert rows and rows == list(range(len(rows)))
+    model = OracleModel(rounded_weights(W), w.shape, w.lora_gamma, dtype=np.float32, kv_dtype="bf16")
+    seq = np.concatenate([P[0], np.array(toks[0][:len(rows)], dtype=np.int32)])
+    ref = teacher_forced_logits(model, seq)
+    n0 = len(P[0])
+    for i in rows:
+        err = np.abs(lg[i] - ref[n0 + i]).max()
+        assert err < 3e-2, (i, err)
+        assert int(np.argmax(lg[i])) == int(meta[i, 5])
+
+
+def test_1b_gqa_lossless_and_teacher_forced():
+    w = workload("1b")
+    W, dw = _weights("1b")
+    P = make_prompts(w)
+    _lossless(w, dw, P)
+    _first_step_logits(w, dw, W, P)
+
+
+def test_7b_lossless_and_teacher_forced():
+    w = workload("7b")
+    W, dw = _weights("7b")
+    P = make_prompts(w)
+    _lossless(w, dw, P)
+    _first_step_logits(w, dw, W, P)
+
+
+def test_7b_batch8_ragged_two_waves():
+    w = workload("7b-b8")
+    _, dw = _weights("7b")
+    waves = [make_prompts(w, wave) for wave in range(2)]
+    for P in waves:
+        assert len({len(p) for p in P}) > 1
+    cap = max(_capacity(w, P) for P in waves)
+    ar = []
+    eng = _engine(w, dw, cap)
+    for P in waves:
+        ar.append(eng.generate_ar(P, GEN))
+    eng.close()
+    # one context for both waves: the drafter's training carries over
+    eng = _engine(w, dw, cap)
+    for P, ref in zip(waves, ar):
+        toks, mats, _, _ = eng.generate(P, GEN, update_every=w.update_every, hyper=w.update)
+        for b in range(w.batch):
+            assert toks[b] == list(ref[b]), b
+        assert ((mats >= 0) & (mats <= w.k_spec)).all()
+    st = eng.stats()
+    eng.close()
+    assert st["device_status"] == 0, st["device_flags"]
+    assert st["updates"] >= 2
+
+
+def test_7b_16k_prompt_lossless():
+    w = workload("7b-16k")
+    _, dw = _weights("7b")
+    P = make_prompts(w)
+    assert len(P[0]) == 16384
+    _lossless(w, dw, P, n_gen=16)

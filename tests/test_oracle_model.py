@@ -153,3 +153,36 @@ def test_heads_match_definitions():
     Weff = m.w_s + 0.7 * m.lora_a @ m.lora_b
     np.testing.assert_allclose(m.drafter_logits(h), u @ Weff.T, rtol=1e-10, atol=1e-12)
     np.testing.assert_allclose(m.verifier_logits(h), u @ m.w_v.T, rtol=1e-10, atol=1e-12)
+
+
+def test_to_bf16_matches_torch_rounding():
+    """to_bf16 == torch's float32 -> bfloat16 conversion (round to nearest even), ties included."""
+    from oracle.model import to_bf16
+    r = _rng(21)
+    x = np.concatenate([r.standard_normal(4096) * 10.0 ** r.integers(-6, 6, 4096),
+                        -r.standard_normal(512) * 1e-3]).astype(np.float32)
+    # exact ties: low 16 bits 0x8000 on both even and odd kept parts
+    ties = (r.integers(0x3F000000, 0x40800000, 256, dtype=np.uint32) & np.uint32(0xFFFF0000)) | np.uint32(0x8000)
+    x = np.concatenate([x, ties.view(np.float32), -ties.view(np.float32)])
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float32).numpy()
+    np.testing.assert_array_equal(to_bf16(x), ref)
+
+
+def test_bf16_kv_cache_rows_and_incremental_decode():
+    """kv_dtype='bf16': cached rows are bfloat16 values, cached decode == full recompute,
+    and the logits move by no more than bf16 storage noise."""
+    from oracle.model import to_bf16
+    m, w = _model()
+    mb = OracleModel(make_weights(w), w.shape, w.lora_gamma, kv_dtype="bf16")
+    L = w.shape.n_layers
+    toks = _rng(7).integers(0, w.shape.vocab, 20)
+    cf = mb.new_cache(32)
+    full = mb.layers_range(0, L, mb.embed(toks), 0, cf)
+    assert np.array_equal(to_bf16(cf.k[:, :20]).astype(np.float64), cf.k[:, :20])
+    assert np.array_equal(to_bf16(cf.v[:, :20]).astype(np.float64), cf.v[:, :20])
+    c = mb.new_cache(32)
+    rows = [mb.layers_range(0, L, mb.embed(toks[i:i + 1]), i, c)[0] for i in range(20)]
+    np.testing.assert_allclose(np.stack(rows), full, rtol=1e-12, atol=1e-12)
+    ref = m.verifier_logits(m.layers_range(0, L, m.embed(toks), 0, m.new_cache(32)))
+    diff = np.abs(mb.verifier_logits(full) - ref).max()
+    assert 0.0 < diff < 2.0 ** -8 * np.abs(ref).max()
