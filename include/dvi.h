@@ -91,6 +91,11 @@ typedef struct {
                            bf16, and the gradient buffer: 12 (f32) or 16 (bf16) B per entry) */
   int max_prefill_chunk;/* rows per prefill pass, 16..128 (multiple of 16); 0 = 128 */
   int use_graphs;       /* capture the decode step in a CUDA graph on first use */
+  int bonus;            /* 0: verify the K drafted rows and commit min(m+1, K) tokens (Sec. 3.3
+                           emits y*_{n+m+1}, which the K verify rows hold only for m < K);
+                           1: one more shallow pass on t~_K and a (K+1)-th verify row, so the
+                           correction y*_{n+K+1} exists at m = K and every step commits m+1
+                           tokens.  K + bonus <= 16. */
 } dvi_runtime_config;
 
 typedef struct {
@@ -174,12 +179,12 @@ dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tok
                        int32_t* d_first_token);
 
 /* One DVI step for all B sequences (Sec. 3.3): K greedy draft passes through
- * layers 1..k and the drafter head, one verify pass of the K rows through
- * layers k+1..L and the LM head, accept length m, commit and rollback, and
- * (when logging is on) the replay-buffer tuples of positions 1..min(m+1, K).
- * Outputs (device, may be null): d_out_ids [B][K] committed ids (the first
- * d_n_committed[b] = min(m+1, K) entries of row b are valid), d_n_accepted
- * [B] = m. */
+ * layers 1..k and the drafter head, one verify pass of the K (K+1 with the
+ * bonus row) rows through layers k+1..L and the LM head, accept length m,
+ * commit and rollback, and (when logging is on) the replay-buffer tuples of
+ * positions 1..min(m+1, K).  Outputs (device, may be null): d_out_ids
+ * [B][K + bonus] committed ids (the first d_n_committed[b] entries of row b
+ * are valid: min(m+1, K), or m+1 with the bonus row), d_n_accepted [B] = m. */
 dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids,
                                    int32_t* d_n_committed, int32_t* d_n_accepted);
 

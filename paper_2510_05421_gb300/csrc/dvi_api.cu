@@ -60,6 +60,7 @@ struct dvi_ctx {
   bool tc = false;
   size_t esz = 4;
   int L, d, Hq, Hkv, hd, F, V, k, r, B, K, max_len, cap_steps, cap_rows, chunk, M_max, nq, nkv;
+  int Kv;   // verify rows per sequence: K, or K + 1 with the bonus row
   // device state
   int *lens, *pending, *draft_ids, *status, *log_step, *log_meta;
   long long* counters;
@@ -142,13 +143,15 @@ bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::
   if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f)) return bad("bad rms_eps / rope_theta");
   if (rt->batch < 1 || rt->batch > 64) return bad("batch must be in [1, 64]");
   if (rt->k_spec < 1 || rt->k_spec > 16) return bad("k_spec must be in [1, 16]");
+  if (rt->bonus != 0 && rt->bonus != 1) return bad("bonus must be 0 or 1");
+  if (rt->k_spec + rt->bonus > 16) return bad("k_spec + bonus must be <= 16");
   if (rt->max_seq_len < rt->k_spec + 2) return bad("max_seq_len too small");
   if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
     return bad("log_steps * batch * k_spec must be in [1, 256]");
   if (rt->head_mode != 0 && rt->head_mode != 1) return bad("head_mode must be 0 (LoRA) or 1 (full W^S)");
   if (rt->max_prefill_chunk && (rt->max_prefill_chunk < 16 || rt->max_prefill_chunk > 128 || rt->max_prefill_chunk % 16))
     return bad("max_prefill_chunk must be 16..128, a multiple of 16");
-  if (rt->batch * rt->k_spec > kMaxTokens) return bad("batch * k_spec > 256");
+  if (rt->batch * (rt->k_spec + rt->bonus) > kMaxTokens) return bad("batch * (k_spec + bonus) > 256");
   return true;
 }
 
@@ -175,14 +178,14 @@ size_t layout(dvi_ctx* c, char* base) {
   c->dev_state = reinterpret_cast<float*>(take(sizeof(float) * 16));
   c->x_dr = reinterpret_cast<float*>(take(sizeof(float) * B * d));
   c->ss_dr = reinterpret_cast<float*>(take(sizeof(float) * st * B));
-  c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * K * d));
-  c->ss_ver = reinterpret_cast<float*>(take(sizeof(float) * st * B * K));
+  c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * c->Kv * d));
+  c->ss_ver = reinterpret_cast<float*>(take(sizeof(float) * st * B * c->Kv));
   c->x_pf = reinterpret_cast<float*>(take(sizeof(float) * c->chunk * d));
   c->ss_pf = reinterpret_cast<float*>(take(sizeof(float) * st * c->chunk));
   // activation rows feeding matrix products: bf16 keeps a hi and a lo plane
   const size_t pl = c->tc ? 2 : 1;
   c->xg_dr = take(pl * e * B * d);
-  c->xg_ver = take(pl * e * B * K * d);
+  c->xg_ver = take(pl * e * B * c->Kv * d);
   c->xg_pf = take(pl * e * c->chunk * d);
   c->q = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * c->nq));
   c->bu = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * (r > 0 ? r : 1)));
@@ -221,7 +224,7 @@ size_t layout(dvi_ctx* c, char* base) {
     c->grad_w = reinterpret_cast<float*>(take(sizeof(float) * vd));
     c->G = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
   }
-  c->out_ids = reinterpret_cast<int*>(take(sizeof(int) * B * K));
+  c->out_ids = reinterpret_cast<int*>(take(sizeof(int) * B * c->Kv));
   c->n_committed = reinterpret_cast<int*>(take(sizeof(int) * B));
   c->n_accepted = reinterpret_cast<int*>(take(sizeof(int) * B));
   c->ar_out = reinterpret_cast<int*>(take(sizeof(int) * B));
@@ -313,7 +316,8 @@ bool init_dims(dvi_ctx* c, const dvi_model_config* cfg, const dvi_runtime_config
   c->cap_steps = rt->log_steps;
   c->cap_rows = rt->log_steps * rt->batch * rt->k_spec;
   c->chunk = rt->max_prefill_chunk ? rt->max_prefill_chunk : 128;
-  c->M_max = std::max(std::max(c->B * c->K, c->chunk), std::max(c->cap_rows, c->B));
+  c->Kv = c->K + (rt->bonus ? 1 : 0);
+  c->M_max = std::max(std::max(c->B * c->Kv, c->chunk), std::max(c->cap_rows, c->B));
   c->nq = c->Hq * c->hd;
   c->nkv = c->Hkv * c->hd;
   c->tc = cfg->dtype == DVI_BF16;
@@ -372,7 +376,7 @@ ProjMaps with_act(const ProjMaps& w, const CUtensorMap* act) {
 // after its hi plane.
 int act_rows(const dvi_ctx* c, const void* buf) {
   if (buf == c->xg_dr) return c->B;
-  if (buf == c->xg_ver) return c->B * c->K;
+  if (buf == c->xg_ver) return c->B * c->Kv;
   if (buf == c->xg_pf) return c->chunk;
   if (buf == c->attn_o || buf == c->ffn_h) return c->M_max;
   if (buf == c->log_u) return c->cap_rows;
@@ -382,9 +386,8 @@ size_t act_plane(const dvi_ctx* c, const void* buf, int ld) {
   return c->tc ? static_cast<size_t>(act_rows(c, buf)) * ld : 0;
 }
 
-// launch_proj with the plane offsets of the context's activation buffers.
+// launch_proj with the plane strides of the context's activation buffers.
 cudaError_t launch_proj_ctx(const dvi_ctx* c, ProjArgs a, const ProjMaps* m, cudaStream_t s) {
-  if (c->tc && a.b_mode == B_ACT) a.act_lo = act_rows(c, a.act);
   if (a.xg_out) a.xg_plane = act_plane(c, a.xg_out, a.ld_xg);
   if (a.h_out) a.h_plane = act_plane(c, a.h_out, a.ld_h);
   return launch_proj(a, m, s);
@@ -525,6 +528,8 @@ StepState step_state(dvi_ctx* c) {
   StepState st{};
   st.B = c->B;
   st.K = c->K;
+  st.Kv = c->Kv;
+  st.bonus = c->Kv > c->K ? 1 : 0;
   st.d = c->d;
   st.vocab = c->V;
   st.max_len = c->max_len;
@@ -580,6 +585,8 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
     a.log_step = ctx->log_step;
     a.log_cap_steps = ctx->cap_steps;
     a.log_rows_per_step = ctx->B * ctx->K;
+    a.log_src_rows = ctx->Kv;   // verify rows per sequence; the log keeps the first K
+    a.log_dst_rows = ctx->K;
   }
   ProjMaps pm{};
   if (ctx->tc) pm = with_act(draft ? ctx->head_s : ctx->head_v, act_map);
@@ -592,7 +599,10 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   dvi_status rc;
-  for (int j = 0; j < ctx->K; ++j) {
+  // passes j = 0..K-1 draft t~_{j+1}; with the bonus row, pass K only hands
+  // h_{k,n+K} (of t~_K) to the verify rows
+  for (int j = 0; j < ctx->Kv; ++j) {
+    const bool drafts = j < ctx->K;
     Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, j, ctx->xg_dr, &ctx->map_xg_dr};
     if ((rc = enqueue_layers(ctx, 0, ctx->k, ps)) != DVI_OK) return rc;
     // u = RMSNorm_final(h_k) into the replay buffer, B u, and h_k to the verify rows
@@ -606,10 +616,10 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
     h.dtype = ctx->cfg.dtype;
     h.x_copy = ctx->x_ver;
     h.ld_copy = ctx->d;
-    h.copy_row_stride = ctx->K;
+    h.copy_row_stride = ctx->Kv;
     h.copy_row_off = j;
     h.ss_copy = ctx->ss_ver;
-    h.ss_copy_ld = ctx->B * ctx->K;
+    h.ss_copy_ld = ctx->B * ctx->Kv;
     h.g_copy = norm_gain_before(ctx, ctx->k);
     h.xg_copy = ctx->xg_ver;
     h.xg_copy_plane = act_plane(ctx, ctx->xg_ver, ctx->d);
@@ -620,17 +630,19 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
     h.log_rows_per_step = ctx->B * ctx->K;
     h.log_row_stride = ctx->K;
     h.log_row_off = j;
-    h.log_enabled = ctx->log_enabled;
-    if (ctx->r > 0) {
+    h.log_enabled = drafts ? ctx->log_enabled : 0;
+    if (ctx->r > 0 && drafts) {
       h.lora_b = ctx->w.lora_b;
       h.bu = ctx->bu;
       h.r = ctx->r;
     }
     DVI_CUDA(launch_head_prep(h, s));
+    ctx->launches += 1;
+    if (!drafts) continue;
     if ((rc = enqueue_head(ctx, true, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
       return rc;
     DVI_CUDA(launch_finalize_draft(st, j, s));
-    ctx->launches += 2;
+    ctx->launches += 1;
   }
   return DVI_OK;
 }
@@ -639,8 +651,8 @@ dvi_status enqueue_verify(dvi_ctx* ctx) {
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   dvi_status rc;
-  const int M = ctx->B * ctx->K;
-  Pass pv{ctx->x_ver, ctx->ss_ver, M, M, ctx->K, 0, ctx->B, 0, ctx->xg_ver, &ctx->map_xg_ver};
+  const int M = ctx->B * ctx->Kv;
+  Pass pv{ctx->x_ver, ctx->ss_ver, M, M, ctx->Kv, 0, ctx->B, 0, ctx->xg_ver, &ctx->map_xg_ver};
   if ((rc = enqueue_layers(ctx, ctx->k, ctx->L, pv)) != DVI_OK) return rc;
   if ((rc = enqueue_head(ctx, false, M, ctx->log_enabled ? 2 : 0, ctx->xg_ver, &ctx->map_xg_ver, 0, ctx->ss_ver,
                          M)) != DVI_OK)
@@ -785,13 +797,13 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
     }
     ok = ok && mk(&ctx->head_v.m0, weights->lm_head, ctx->V, ctx->d) &&
          mk(&ctx->head_s.m0, weights->draft_head, ctx->V, ctx->d);
-    // each map covers both planes: rows [0, R) hi, [R, 2R) lo
-    ok = ok && make_act_map(&ctx->map_xg_dr, ctx->xg_dr, 2 * ctx->B, ctx->d) &&
-         make_act_map(&ctx->map_xg_ver, ctx->xg_ver, 2 * ctx->B * ctx->K, ctx->d) &&
-         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, 2 * ctx->chunk, ctx->d) &&
-         make_act_map(&ctx->map_attn_o, ctx->attn_o, 2 * ctx->M_max, ctx->nq) &&
-         make_act_map(&ctx->map_ffn_h, ctx->ffn_h, 2 * ctx->M_max, ctx->F) &&
-         make_act_map(&ctx->map_log_u, ctx->log_u, 2 * ctx->cap_rows, ctx->d);
+    // each map covers both planes of its buffer: [2][R][cols]
+    ok = ok && make_act_map(&ctx->map_xg_dr, ctx->xg_dr, ctx->B, ctx->d) &&
+         make_act_map(&ctx->map_xg_ver, ctx->xg_ver, ctx->B * ctx->Kv, ctx->d) &&
+         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, ctx->chunk, ctx->d) &&
+         make_act_map(&ctx->map_attn_o, ctx->attn_o, ctx->M_max, ctx->nq) &&
+         make_act_map(&ctx->map_ffn_h, ctx->ffn_h, ctx->M_max, ctx->F) &&
+         make_act_map(&ctx->map_log_u, ctx->log_u, ctx->cap_rows, ctx->d);
     const long long kv_rows = static_cast<long long>(ctx->L) * ctx->B * ctx->Hkv * ctx->max_len;
     ok = ok && make_kv_map(&ctx->map_kc, ctx->kcache, kv_rows, ctx->hd) &&
          make_kv_map(&ctx->map_vc, ctx->vcache, kv_rows, ctx->hd);
@@ -820,7 +832,7 @@ dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tok
   if (!ctx) return DVI_ERR_INVALID_ARG;
   if (seq < 0 || seq >= ctx->B || !d_tokens || n_tokens < 1)
     return fail(ctx, DVI_ERR_INVALID_ARG, "prefill: bad sequence, tokens or length");
-  if (n_tokens + ctx->K + 1 > ctx->max_len) return fail(ctx, DVI_ERR_CAPACITY, "prefill: prompt exceeds max_seq_len");
+  if (n_tokens + ctx->Kv + 1 > ctx->max_len) return fail(ctx, DVI_ERR_CAPACITY, "prefill: prompt exceeds max_seq_len");
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   DVI_CUDA(launch_reset_seq(st, seq, s));
@@ -877,7 +889,7 @@ dvi_status dvi_draft_verify_commit(dvi_ctx* ctx, int32_t* d_out_ids, int32_t* d_
   if (rc != DVI_OK) return rc;
   mark_end(ctx, 1, t1);
   if (d_out_ids)
-    DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->out_ids, sizeof(int) * ctx->B * ctx->K, cudaMemcpyDeviceToDevice, s));
+    DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->out_ids, sizeof(int) * ctx->B * ctx->Kv, cudaMemcpyDeviceToDevice, s));
   if (d_n_committed)
     DVI_CUDA(cudaMemcpyAsync(d_n_committed, ctx->n_committed, sizeof(int) * ctx->B, cudaMemcpyDeviceToDevice, s));
   if (d_n_accepted)
@@ -1051,7 +1063,7 @@ dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes)
     case DVI_BUF_GRAD_A: *dptr = ctx->grad_a; *bytes = sizeof(float) * static_cast<size_t>(ctx->V) * rr; break;
     case DVI_BUF_GRAD_B: *dptr = ctx->grad_b; *bytes = sizeof(float) * static_cast<size_t>(rr) * ctx->d; break;
     case DVI_BUF_X_DRAFT: *dptr = ctx->x_dr; *bytes = sizeof(float) * ctx->B * ctx->d; break;
-    case DVI_BUF_X_VERIFY: *dptr = ctx->x_ver; *bytes = sizeof(float) * ctx->B * ctx->K * ctx->d; break;
+    case DVI_BUF_X_VERIFY: *dptr = ctx->x_ver; *bytes = sizeof(float) * ctx->B * ctx->Kv * ctx->d; break;
     case DVI_BUF_K_CACHE: *dptr = ctx->kcache; *bytes = kv; break;
     case DVI_BUF_V_CACHE: *dptr = ctx->vcache; *bytes = kv; break;
     case DVI_BUF_STATUS: *dptr = ctx->status; *bytes = sizeof(int); break;

@@ -35,9 +35,9 @@ struct ProjArgs {
   const void* w2;
   int rows_q, rows_k, rows_v;
   // B operand: rows act_row0 .. act_row0+M-1 of act[.][ld_act]; bf16
-  // activations hold a hi plane and, act_lo rows further, a lo plane
-  // (value = hi + lo), so the MMA runs over 2 n_pad columns
-  const void* act; int ld_act; int act_row0; int act_lo;
+  // activations hold a hi plane and a lo plane (value = hi + lo; the TMA
+  // map `mb` is [2][rows][ld_act]), so the MMA runs over 2 n_pad columns
+  const void* act; int ld_act; int act_row0;
   // Optional RMSNorm scale applied to every accumulator in the epilogue:
   // rstd[n] = rsqrt(sum_t ss[t*ss_ld + n] / d_norm + eps) (the norm gain is
   // already folded into the activation rows).
@@ -63,6 +63,7 @@ struct ProjArgs {
   float* logits_out; int ld_logits;
   int logits_mode;            // 0 none, 1 row n -> logits_out[n], 2 replay-buffer slot
   const int* log_step; int log_cap_steps; int log_rows_per_step;
+  int log_src_rows, log_dst_rows;   // mode 2: launch rows per sequence, of which the log keeps the first
   const float* lora_a; const float* lora_bu; int lora_r; float gamma;
   unsigned long long* amax;   // [M] argmax keys, or null
 };
@@ -79,7 +80,7 @@ size_t proj_partial_floats(const ProjArgs& a, bool tc);
 cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s);
 bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols);   // 64-row boxes (gate/up)
-bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);
+bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);   // [2 planes][rows][cols]
 
 struct AttnArgs {
   const float* q; int ld_q;          // rotated queries [M][H_q*hd]
@@ -135,6 +136,7 @@ cudaError_t launch_head_prep(const HeadPrepArgs& a, cudaStream_t s);
 
 struct StepState {
   int B, K, d, vocab, max_len, dtype;
+  int Kv, bonus;                                // verify rows per sequence (K + bonus)
   int* lens; int* pending; int* draft_ids;      // [B][K+1]
   float* x_dr; float* ss_dr; int ss_dr_ld;
   const float* g0; void* xg_dr;                 // first layer's attention-norm gain, x * g0

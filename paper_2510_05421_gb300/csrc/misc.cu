@@ -13,6 +13,8 @@
 // t~_1..t~_m and, when m < K, the correction y*_{n+m+1} -- min(m+1, K)
 // tokens -- and the cache length advances by the same count, which discards
 // the KV rows of rejected drafts (they are overwritten later; no data moves).
+// With the bonus row (verify rows for t~_1..t~_K and one more for t~_K's
+// successor) y*_{n+K+1} exists too, and every step commits m + 1 tokens.
 // The replay-buffer tuples of rows 1..min(m+1, K) get r = 1 up to m and r = 0
 // at the first reject (Sec. 3.3); later rows stay invalid (counterfactual).
 #include "common.cuh"
@@ -213,7 +215,7 @@ __global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st,
     tok_s[b] = t;
   }
   __syncthreads();
-  if (j + 1 < st.K) embed_rows<T>(st, tok_s, red);
+  if (j + 1 < st.Kv) embed_rows<T>(st, tok_s, red);   // the next pass's token (t~_K feeds the bonus row)
 }
 
 template <typename T>
@@ -222,19 +224,20 @@ __global__ void __launch_bounds__(128) finalize_verify_kernel(const StepState st
   __shared__ float red[kMaxTiles * 4];
   griddep_launch();
   griddep_wait();
-  const int K = st.K;
+  const int K = st.K, Kv = st.Kv;
   const int ls = *st.log_step;
   const bool log_ok = st.log_enabled && ls < st.log_cap_steps;
   for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
     int y[16];
-    for (int i = 0; i < K; ++i) y[i] = take_argmax(st.amax + b * K + i, st.status);
+    for (int i = 0; i < Kv; ++i) y[i] = take_argmax(st.amax + b * Kv + i, st.status);
     int* dr = st.draft_ids + b * (K + 1);
     int m = 0;
     while (m < K && dr[m + 1] == y[m]) ++m;
-    const int c = m < K ? m + 1 : K;
-    for (int i = 0; i < K; ++i) {
+    // the correction y*_{n+m+1} exists for m < K, and for m = K with the bonus row
+    const int c = m < Kv ? m + 1 : K;
+    for (int i = 0; i < Kv; ++i) {
       const int id = i < m ? dr[i + 1] : (i == m ? y[m] : -1);
-      st.out_ids[b * K + i] = id;
+      st.out_ids[b * Kv + i] = id;
     }
     st.n_committed[b] = c;
     st.n_accepted[b] = m;
@@ -249,7 +252,7 @@ __global__ void __launch_bounds__(128) finalize_verify_kernel(const StepState st
         meta[5] = y[i];
       }
     }
-    const int newtok = st.out_ids[b * K + c - 1];
+    const int newtok = st.out_ids[b * Kv + c - 1];
     st.lens[b] += c;
     st.pending[b] = newtok;
     dr[0] = newtok;

@@ -210,8 +210,14 @@ __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int 
       }
       if (dst) {
 #pragma unroll
-        for (int j = 0; j < kChunk; ++j)
-          if ((own >> j) & 1u) dst[static_cast<size_t>(c0 + j) * p.ld_logits + f] = z[j];
+        for (int j = 0; j < kChunk; ++j) {
+          int row = c0 + j;
+          if (p.logits_mode == 2) {   // replay-buffer slot of (sequence, block row)
+            const int i = row % p.log_src_rows;
+            row = i < p.log_dst_rows ? row / p.log_src_rows * p.log_dst_rows + i : -1;
+          }
+          if (((own >> j) & 1u) && row >= 0) dst[static_cast<size_t>(row) * p.ld_logits + f] = z[j];
+        }
       }
     }
     if (p.amax) {
@@ -388,9 +394,11 @@ __global__ void __launch_bounds__(192, 2)
         if (soft_b) return;
         const int s = i % stages;
         const int x = (kb0 + i) * kKBlock;
+        // the activation map is [plane][rows][cols]: rows past the buffer's
+        // are out of bounds (zero fill, no traffic) in either plane
         for (int b = 0; b < nbox; ++b) {
-          tma_load_2d(sB + s * bbytes + b * 2048, &mb, x, p.act_row0 + b * 16, &full[s], 0ull);
-          tma_load_2d(sB + s * bbytes + (nbox + b) * 2048, &mb, x, p.act_lo + p.act_row0 + b * 16, &full[s], 0ull);
+          tma_load_3d(sB + s * bbytes + b * 2048, &mb, x, p.act_row0 + b * 16, 0, &full[s], 0ull);
+          tma_load_3d(sB + s * bbytes + (nbox + b) * 2048, &mb, x, p.act_row0 + b * 16, 1, &full[s], 0ull);
         }
       };
       // The first stages' weight tiles do not depend on earlier kernels.
@@ -752,7 +760,17 @@ bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
   return make_map(map, w, rows, cols, kGuRows);
 }
 bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols) {
-  return make_map(map, act, rows, cols, 16);
+  // two planes (hi, lo) of [rows][cols] bf16, boxes of 16 rows x 64 columns
+  auto encode = encoder();
+  if (!encode) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows), 2};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2, static_cast<cuuint64_t>(rows) * cols * 2};
+  cuuint32_t box[3] = {kKBlock, 16, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(act), dims, strides, box,
+                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
 }
 bool make_kv_map(CUtensorMap* map, const void* cache, long long rows, int hd) {
   auto encode = encoder();

@@ -39,7 +39,7 @@ class ModelConfig(ctypes.Structure):
 class RuntimeConfig(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int), ("k_spec", ctypes.c_int), ("max_seq_len", ctypes.c_int),
                 ("log_steps", ctypes.c_int), ("head_mode", ctypes.c_int), ("max_prefill_chunk", ctypes.c_int),
-                ("use_graphs", ctypes.c_int)]
+                ("use_graphs", ctypes.c_int), ("bonus", ctypes.c_int)]
 
 
 class LayerWeightsC(ctypes.Structure):
@@ -181,16 +181,18 @@ class DVIEngine:
 
     def __init__(self, shape, dtype: str, weights: DeviceWeights, *, batch: int, k_spec: int, split_k: int,
                  lora_rank: int, lora_gamma: float = 1.0, max_seq_len: int, log_steps: int,
-                 prefill_chunk: int = 128, use_graphs: bool = True, device: int = 0, head_mode: int = 0):
+                 prefill_chunk: int = 128, use_graphs: bool = True, device: int = 0, head_mode: int = 0,
+                 bonus: bool = False):
         L = lib()
         self.shape, self.dtype, self.w = shape, dtype, weights
         self.B, self.K = batch, k_spec
+        self.Kv = k_spec + (1 if bonus else 0)      # verify rows (and committed ids) per sequence
         self.device = torch.device("cuda", device)
         self.cfg = ModelConfig(shape.n_layers, shape.d_model, shape.n_heads, shape.n_kv_heads, shape.head_dim,
                                shape.d_ffn, shape.vocab, split_k, lora_rank, lora_gamma, shape.rms_eps,
                                shape.rope_theta, DVI_BF16 if dtype == "bf16" else DVI_F32)
         self.rt = RuntimeConfig(batch, k_spec, max_seq_len, log_steps, head_mode, prefill_chunk,
-                                1 if use_graphs else 0)
+                                1 if use_graphs else 0, 1 if bonus else 0)
         nbytes = L.dvi_workspace_bytes(ctypes.byref(self.cfg), ctypes.byref(self.rt))
         if nbytes == 0:
             raise DVIError("invalid configuration")
@@ -212,7 +214,7 @@ class DVIEngine:
                           ctypes.c_void_p(self.stream.cuda_stream), ctypes.byref(self.ctx))
         if rc != 0:
             raise DVIError(f"dvi_create failed: {STATUS.get(rc, rc)}")
-        self.out_ids = torch.zeros(batch, k_spec, dtype=torch.int32, device=self.device)
+        self.out_ids = torch.zeros(batch, self.Kv, dtype=torch.int32, device=self.device)
         self.n_committed = torch.zeros(batch, dtype=torch.int32, device=self.device)
         self.n_accepted = torch.zeros(batch, dtype=torch.int32, device=self.device)
         self.ar_ids = torch.zeros(batch, dtype=torch.int32, device=self.device)
@@ -238,7 +240,7 @@ class DVIEngine:
         return self.first
 
     def step(self):
-        """One draft -> verify -> commit step; device tensors (ids [B,K], n_committed [B], m [B])."""
+        """One draft -> verify -> commit step; device tensors (ids [B,K(+1)], n_committed [B], m [B])."""
         rc = lib().dvi_draft_verify_commit(self.ctx, _ptr(self.out_ids), _ptr(self.n_committed),
                                            _ptr(self.n_accepted))
         self._check(rc, "dvi_draft_verify_commit")
@@ -333,7 +335,7 @@ class DVIEngine:
         with torch.cuda.stream(self.stream):
             first.copy_(self.first, non_blocking=True)
         d2h += self.B * 4
-        out_h = torch.empty(self.B, self.K, dtype=torch.int32).pin_memory()
+        out_h = torch.empty(self.B, self.Kv, dtype=torch.int32).pin_memory()
         cnt_h = torch.empty(self.B, dtype=torch.int32).pin_memory()
         acc_h = torch.empty(self.B, dtype=torch.int32).pin_memory()
         toks: List[List[int]] = [[] for _ in range(self.B)]
@@ -350,7 +352,7 @@ class DVIEngine:
                 out_h.copy_(ids, non_blocking=True)
                 cnt_h.copy_(cnt, non_blocking=True)
                 acc_h.copy_(acc, non_blocking=True)
-            d2h += (self.B * self.K + 2 * self.B) * 4
+            d2h += (self.B * self.Kv + 2 * self.B) * 4
             self.stream.synchronize()
             for b in range(self.B):
                 toks[b].extend(out_h[b, :int(cnt_h[b])].tolist())
