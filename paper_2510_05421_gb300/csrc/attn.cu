@@ -15,6 +15,9 @@
 // rule, and positions a row must not see contribute exact zeros, so a row's
 // output does not depend on how many rows share the launch.
 //
+// The bf16 tensor-core decode kernel (attn_mma_kernel) instead splits each
+// row's own positions evenly: see the rule at its split set-up.
+//
 // Decode (<= 16 rows per sequence): attn_dec_kernel streams the split's K/V
 // through a shared-memory ring by bulk copies and keeps a query group's
 // vectors, scores and accumulators in registers; each warp walks its
@@ -382,15 +385,21 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   const int nrows = min(RQ, a.rows_per_seq - i0);
   const int Q = nrows * G;
   const int base = a.lens[seq] + a.pos_off;
-  const int t_cta = min(base + i0 + nrows, a.max_len);
-  const int p0 = split * a.split_len;
-  const int p1 = max(p0, min(p0 + a.split_len, t_cta));
-  const int nch = (p1 - p0 + kChunkPos - 1) / kChunkPos;   // 0 for a split past the rows' positions
+  // Split `split` of a row at position p covers the 64-position chunks
+  // [split*C/S, (split+1)*C/S) of the C = p/64 + 1 chunks that hold positions
+  // 0..p: a function of p alone, so a row's result is the same whichever
+  // rows share the CTA, and every split gets the same number of chunks (to
+  // within one).  The CTA runs the union of its rows' chunk ranges; a chunk
+  // outside a row's range is masked for that row and leaves its state exact.
+  const int p_min = min(base + i0, a.max_len - 1);
+  const int p_max = min(base + i0 + nrows - 1, a.max_len - 1);
+  const int c0 = split * (p_min / kChunkPos + 1) / S;
+  const int nch = max(0, (split + 1) * (p_max / kChunkPos + 1) / S - c0);
   const int row0 = static_cast<int>(a.kv_row0 + (static_cast<long long>(seq) * a.n_kv_heads + g) * a.max_len);
 
   auto issue = [&](int ch) {
     const int st = ch % kDecStages;
-    const int y = row0 + p0 + ch * kChunkPos;
+    const int y = row0 + (c0 + ch) * kChunkPos;
     mbar_arrive_expect_tx(&full[st], kStage);
     for (int b = 0; b < kBoxes; ++b) {
       tma_load_2d(ring + st * kStage + b * kBoxBytes, &mk, b * 64, y, &full[st], 0ull);
@@ -410,7 +419,7 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   // Q fragments (rows gq and gq+8), scaled by 1/sqrt(hd) * log2(e), as a
   // bf16 pair hi + lo (two products per K fragment keep 16 bits of q)
   uint32_t qa[HD / 16][4], qb[HD / 16][4];
-  int lim0 = -1, lim1 = -1;
+  int lim0 = -1, lim1 = -1, lo0 = 0, hi0 = 0, lo1 = 0, hi1 = 0;
   {
     const float sc = a.scale * kLog2e;
     const float* qrow[2] = {nullptr, nullptr};
@@ -424,6 +433,13 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
         else lim1 = base + i0 + ii;
       }
     }
+    // this split's positions of each row: [lo, hi)
+    const int C0 = min(max(lim0, 0), a.max_len - 1) / kChunkPos + 1;
+    const int C1 = min(max(lim1, 0), a.max_len - 1) / kChunkPos + 1;
+    lo0 = split * C0 / S * kChunkPos;
+    hi0 = (split + 1) * C0 / S * kChunkPos;
+    lo1 = split * C1 / S * kChunkPos;
+    hi1 = (split + 1) * C1 / S * kChunkPos;
 #pragma unroll
     for (int kk = 0; kk < HD / 16; ++kk) {
 #pragma unroll
@@ -432,7 +448,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
         const int col = kk * 16 + (r >> 1) * 8 + 2 * tq;
         qa[kk][r] = 0u;
         qb[kk][r] = 0u;
-        if (qr) split_bf16x2(qr[col] * sc, qr[col + 1] * sc, qa[kk][r], qb[kk][r]);
+        if (qr) {
+          const float2 v = *reinterpret_cast<const float2*>(qr + col);
+          split_bf16x2(v.x * sc, v.y * sc, qa[kk][r], qb[kk][r]);
+        }
       }
     }
   }
@@ -448,7 +467,7 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
     mbar_wait(&full[st], (ch / kDecStages) & 1, a.status);
     const uint8_t* ks = ring + st * kStage;
     const uint8_t* vs = ks + kBoxes * kBoxBytes;
-    const int pc = p0 + ch * kChunkPos;
+    const int pc = (c0 + ch) * kChunkPos;
     // S = Q K^T for this warp's 16 positions (two n-tiles of 8)
     float sacc[2][4], slo[2][4];   // q_hi K^T and q_lo K^T: independent MMA chains
 #pragma unroll
@@ -479,8 +498,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const int pos = pc + warp * 16 + nt * 8 + 2 * tq + e;
-        if (!(pos < p1 && pos <= lim0)) sacc[nt][e] = -INFINITY;
-        if (!(pos < p1 && pos <= lim1)) sacc[nt][2 + e] = -INFINITY;
+        if (!(pos >= lo0 && pos < hi0 && pos <= lim0)) sacc[nt][e] = -INFINITY;
+        if (!(pos >= lo1 && pos < hi1 && pos <= lim1)) sacc[nt][2 + e] = -INFINITY;
         mx0 = fmaxf(mx0, sacc[nt][e]);
         mx1 = fmaxf(mx1, sacc[nt][2 + e]);
       }

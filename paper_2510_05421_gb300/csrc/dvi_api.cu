@@ -79,7 +79,7 @@ struct dvi_ctx {
   int* attn_ctr;
   int n_attn_ctr;
   int attn_split_len, attn_nsplits;
-  int dec_split_len, dec_nsplits;   // bf16 decode attention: splits of one cluster
+  int dec_nsplits;                  // bf16 decode attention: splits (one cluster) per KV head
   void* log_u;
   float* log_logits;
   float *Z, *rowstat, *coef, *ub, *ga, *ga_part;
@@ -273,12 +273,9 @@ void size_scratch(dvi_ctx* c) {
   sl = std::max(kAttnBlk, (sl + kAttnBlk - 1) / kAttnBlk * kAttnBlk);
   c->attn_split_len = sl;
   c->attn_nsplits = (c->max_len + sl - 1) / sl;
-  // bf16 decode: the splits of a KV head form one cluster of at most 8
-  const int dsplits = std::max(1, std::min(8, target / std::max(1, c->B * c->Hkv)));
-  int dsl = (c->max_len + dsplits - 1) / dsplits;
-  dsl = std::max(kAttnBlk, (dsl + kAttnBlk - 1) / kAttnBlk * kAttnBlk);
-  c->dec_split_len = dsl;
-  c->dec_nsplits = (c->max_len + dsl - 1) / dsl;
+  // bf16 decode: the splits of a KV head form one cluster of at most 8; each
+  // split takes an even share of every row's own positions
+  c->dec_nsplits = std::max(1, std::min(8, target / std::max(1, c->B * c->Hkv)));
   AttnArgs at{};
   at.n_heads = c->Hq;
   at.n_kv_heads = c->Hkv;
@@ -446,7 +443,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   t.n_seqs = ps.n_seqs;
   t.pos_off = ps.pos_off;
   const bool dec_cluster = ctx->tc && ps.rows_per_seq <= 16 && ctx->Hq / ctx->Hkv <= 8;
-  t.split_len = dec_cluster ? ctx->dec_split_len : ctx->attn_split_len;
+  t.split_len = dec_cluster ? 0 : ctx->attn_split_len;
   t.n_splits_max = dec_cluster ? ctx->dec_nsplits : ctx->attn_nsplits;
   t.part = ctx->attn_part;
   t.counters = ctx->attn_ctr;
