@@ -37,15 +37,12 @@
 // them in split order.  Both are deterministic, and the split plan depends on
 // the weight shape only (never on the number of decode rows).
 #include <algorithm>
-#include <cooperative_groups.h>
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
 #include "kernels.h"
 
 namespace dvi {
-
-namespace cg = cooperative_groups;
 
 constexpr int kGuRows = 64;   // features per gate/up tile (64 gate rows + 64 up rows)
 
@@ -313,6 +310,9 @@ __device__ __forceinline__ void produce_b_f32(const ProjArgs& p, uint8_t* bs, in
 }
 
 // ------------------------------------------------------------------ tcgen05
+// kSplit: the launch splits K over a cluster (n_splits > 1); the unsplit
+// instantiation carries no cluster code.
+template <bool kSplit>
 __global__ void __launch_bounds__(192, 2)
     proj_tc_kernel(const __grid_constant__ CUtensorMap m0, const __grid_constant__ CUtensorMap m1,
                    const __grid_constant__ CUtensorMap m2, const __grid_constant__ CUtensorMap mb,
@@ -330,6 +330,7 @@ __global__ void __launch_bounds__(192, 2)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   float* rstd = reinterpret_cast<float*>(tmem_holder + 4);
   int* posn = reinterpret_cast<int*>(rstd + kMaxTokens);
+
   // after `done` the A stages are free: epilogue scratch, then this split's
   // partial tile [n_pad][128] for the cluster reduction
   EpiSmem& es = *reinterpret_cast<EpiSmem*>(sA);
@@ -342,6 +343,7 @@ __global__ void __launch_bounds__(192, 2)
   const uint32_t ncols = tmem_cols(2 * p.n_pad);
   const bool soft_b = p.b_mode == B_SOFT_F32;
   const bool gu = p.flavor == EPI_GATEUP;
+  const int S = kSplit ? p.n_splits : 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -474,19 +476,24 @@ __global__ void __launch_bounds__(192, 2)
     const uint32_t lane_base = tmem + ((static_cast<uint32_t>(warp) * 32u) << 16);
     const int nchunks = (p.M + kChunk - 1) / kChunk;
     float v[kChunk];
-    for (int c = 0; c < nchunks; ++c) {
-      float vl[kChunk];
-      tmem_ld16(lane_base + c * kChunk, v);
-      tmem_ld16(lane_base + p.n_pad + c * kChunk, vl);
+    if (!kSplit) {
+      for (int c = 0; c < nchunks; ++c) {
+        float vl[kChunk];
+        tmem_ld16(lane_base + c * kChunk, v);
+        tmem_ld16(lane_base + p.n_pad + c * kChunk, vl);
 #pragma unroll
-      for (int j = 0; j < kChunk; ++j) v[j] += vl[j];
-      if (p.n_splits == 1) {
+        for (int j = 0; j < kChunk; ++j) v[j] += vl[j];
         if (ok)
           epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, valid_cols(p, c * kChunk));
-      } else {
+      }
+    } else {
+      for (int c = 0; c < nchunks; ++c) {
+        float vl[kChunk];
+        tmem_ld16(lane_base + c * kChunk, v);
+        tmem_ld16(lane_base + p.n_pad + c * kChunk, vl);
 #pragma unroll
         for (int j = 0; j < kChunk; ++j)
-          if (c * kChunk + j < p.M) part[(c * kChunk + j) * kTileRows + tid] = v[j];
+          if (c * kChunk + j < p.M) part[(c * kChunk + j) * kTileRows + tid] = v[j] + vl[j];
       }
     }
     tc_fence_before();
@@ -496,18 +503,18 @@ __global__ void __launch_bounds__(192, 2)
       tmem_dealloc(tmem, ncols);
     }
   }
-  if (p.n_splits > 1) {
+  if (kSplit) {
     // ---------------- split-K across the cluster: rank r finishes the token
-    // columns n with n % n_splits == r, summing every rank's partial in rank
-    // order (all of a column's loads are issued before the sum)
-    cg::cluster_group cluster = cg::this_cluster();
-    cluster.sync();
+    // columns n with n % S == r, summing every rank's partial in rank order
+    // (all of a column's loads from the peers are issued before the sum)
+    cluster_arrive_release();
+    cluster_wait_acquire();
     if (warp < 4) {
       const int tid = threadIdx.x;
-      const int S = p.n_splits;
-      const float* peer[8];
+      uint32_t peer[8];
+      const uint32_t mine = smem_u32(part) + static_cast<uint32_t>(tid) * 4u;
 #pragma unroll
-      for (int r = 0; r < 8; ++r) peer[r] = r < S ? cluster.map_shared_rank(part, r) : part;
+      for (int r = 0; r < 8; ++r) peer[r] = r < S ? mapa_shared(mine, r) : 0u;
       const int nchunks = (p.M + kChunk - 1) / kChunk;
       for (int c = 0; c < nchunks; ++c) {
         uint32_t own = 0;
@@ -520,10 +527,10 @@ __global__ void __launch_bounds__(192, 2)
         for (int j = 0; j < kChunk; ++j) {
           v[j] = 0.f;
           if ((own >> j) & 1u) {
+            const uint32_t off = static_cast<uint32_t>((c * kChunk + j) * kTileRows) * 4u;
             float t[8];
-            const int off = (c * kChunk + j) * kTileRows + tid;
 #pragma unroll
-            for (int r = 0; r < 8; ++r) t[r] = r < S ? peer[r][off] : 0.f;
+            for (int r = 0; r < 8; ++r) t[r] = r < S ? ld_cluster_f32(peer[r] + off) : 0.f;
             float acc = t[0];
 #pragma unroll
             for (int r = 1; r < 8; ++r)
@@ -534,7 +541,9 @@ __global__ void __launch_bounds__(192, 2)
         epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, own);
       }
     }
-    cluster.sync();   // every rank keeps its shared memory until all have read it
+    // every rank keeps its shared memory until all have read it
+    cluster_arrive_release();
+    cluster_wait_acquire();
   }
 }
 
@@ -692,7 +701,8 @@ cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s
   if (a0.dtype == DVI_BF16) {
     static bool attr = false;
     if (!attr) {
-      cudaFuncSetAttribute(proj_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      cudaFuncSetAttribute(proj_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      cudaFuncSetAttribute(proj_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
       attr = true;
     }
     ProjArgs a = a0;
@@ -717,7 +727,9 @@ cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s
     at[1].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = a.n_splits > 1 ? 2 : 1;
-    e = cudaLaunchKernelEx(&cfg, proj_tc_kernel, maps->m0, maps->m1, maps->m2, maps->mb, a, stages);
+    e = a.n_splits > 1
+            ? cudaLaunchKernelEx(&cfg, proj_tc_kernel<true>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages)
+            : cudaLaunchKernelEx(&cfg, proj_tc_kernel<false>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages);
   } else {
     ProjArgs b = a0;
     b.n_ttiles = (a0.M + kChunk - 1) / kChunk;
