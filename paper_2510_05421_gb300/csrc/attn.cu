@@ -365,6 +365,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   __shared__ __align__(8) uint64_t full[kDecStages];
   __shared__ float wm[4][kMmaQ], wl[4][kMmaQ];
   __shared__ float cm[kMmaQ], cl[kMmaQ];             // this split's merged max / sum
+  __shared__ float ww[4][kMmaQ];                     // per-warp merge weights
+  __shared__ float rw[8][kMmaQ], rinv[kMmaQ];        // per-rank combine weights, 1 / sum
   const uint32_t raw = smem_u32(dsm_raw);
   uint8_t* ring = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
   float* wO = reinterpret_cast<float*>(ring);                       // [4][16][HD], after the loop
@@ -560,7 +562,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  // merge the four warps into this split's (m, l, O) (the ring is free now)
+  // merge the four warps into this split's (m, l, O) (the ring is free now);
+  // only the Q live query rows are merged
   if (tq == 0) {
     wm[warp][gq] = m0;
     wm[warp][gq + 8] = m1;
@@ -570,70 +573,79 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
 #pragma unroll
   for (int nt = 0; nt < kNT; ++nt) {
     const int d = nt * 8 + 2 * tq;
-    wO[(warp * kMmaQ + gq) * HD + d] = o[nt][0];
-    wO[(warp * kMmaQ + gq) * HD + d + 1] = o[nt][1];
-    wO[(warp * kMmaQ + gq + 8) * HD + d] = o[nt][2];
-    wO[(warp * kMmaQ + gq + 8) * HD + d + 1] = o[nt][3];
+    if (gq < Q) {
+      wO[(warp * kMmaQ + gq) * HD + d] = o[nt][0];
+      wO[(warp * kMmaQ + gq) * HD + d + 1] = o[nt][1];
+    }
+    if (gq + 8 < Q) {
+      wO[(warp * kMmaQ + gq + 8) * HD + d] = o[nt][2];
+      wO[(warp * kMmaQ + gq + 8) * HD + d + 1] = o[nt][3];
+    }
   }
   __syncthreads();
-  if (tid < kMmaQ) {
+  if (tid < Q) {
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w][tid]);
     float Ls = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) Ls = fmaf(wl[w][tid], (wm[w][tid] == -INFINITY) ? 0.f : exp2f(wm[w][tid] - M), Ls);
+    for (int w = 0; w < 4; ++w) {
+      const float wt = (wm[w][tid] == -INFINITY) ? 0.f : exp2f(wm[w][tid] - M);
+      ww[w][tid] = wt;
+      Ls = fmaf(wl[w][tid], wt, Ls);
+    }
     cm[tid] = M;
     cl[tid] = Ls;
   }
-  for (int idx = tid; idx < kMmaQ * HD; idx += 128) {
+  __syncthreads();
+  for (int idx = tid; idx < Q * HD; idx += 128) {
     const int qi = idx / HD, d = idx % HD;
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w][qi]);
     float O = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w)
-      O = fmaf(wO[(w * kMmaQ + qi) * HD + d], (wm[w][qi] == -INFINITY) ? 0.f : exp2f(wm[w][qi] - M), O);
+    for (int w = 0; w < 4; ++w) O = fmaf(wO[(w * kMmaQ + qi) * HD + d], ww[w][qi], O);
     cO[idx] = O;
   }
-  // combine the splits of the cluster: rank r finishes output elements
-  // r*128 + tid, (r + S)*128 + tid, ...
+  // combine the splits of the cluster: per query row, the rank weights
+  // 2^(m_r - M) and 1 / sum_r l_r 2^(m_r - M) once; then rank r finishes
+  // output elements r*128 + tid, (r + S)*128 + tid, ...
   cluster.sync();
-  const float* pm[8];
-  const float* pl[8];
   const float* pO[8];
 #pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    const int rr = r < S ? r : 0;
-    pm[r] = cluster.map_shared_rank(cm, rr);
-    pl[r] = cluster.map_shared_rank(cl, rr);
-    pO[r] = cluster.map_shared_rank(cO, rr);
-  }
-  const int hq_base = g * G;
-  for (int idx = split * 128 + tid; idx < Q * HD; idx += S * 128) {
-    const int qi = idx / HD, d = idx % HD;
-    float ms[8], ls[8], os[8];
+  for (int r = 0; r < 8; ++r) pO[r] = cluster.map_shared_rank(cO, r < S ? r : 0);
+  if (tid < Q) {
+    float ms[8], ls[8];
 #pragma unroll
     for (int r = 0; r < 8; ++r) {
-      ms[r] = r < S ? pm[r][qi] : -INFINITY;
-      ls[r] = r < S ? pl[r][qi] : 0.f;
-      os[r] = r < S ? pO[r][idx] : 0.f;
+      ms[r] = r < S ? cluster.map_shared_rank(cm, r)[tid] : -INFINITY;
+      ls[r] = r < S ? cluster.map_shared_rank(cl, r)[tid] : 0.f;
     }
     float M = ms[0];
 #pragma unroll
     for (int r = 1; r < 8; ++r) M = fmaxf(M, ms[r]);
-    float Ls = 0.f, O = 0.f;
+    float Ls = 0.f;
 #pragma unroll
     for (int r = 0; r < 8; ++r) {
       const float w = (ms[r] == -INFINITY) ? 0.f : exp2f(ms[r] - M);
+      rw[r][tid] = w;
       Ls = fmaf(ls[r], w, Ls);
-      O = fmaf(os[r], w, O);
     }
+    rinv[tid] = 1.f / Ls;
+  }
+  __syncthreads();
+  const int hq_base = g * G;
+  for (int idx = split * 128 + tid; idx < Q * HD; idx += S * 128) {
+    const int qi = idx / HD, d = idx % HD;
+    float os[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) os[r] = r < S ? pO[r][idx] : 0.f;
+    float O = 0.f;
+#pragma unroll
+    for (int r = 0; r < 8; ++r)
+      if (r < S) O = fmaf(os[r], rw[r][qi], O);
     const int ii = qi / G, hh = qi % G;
     const int n = sl * a.rows_per_seq + i0 + ii;
     Act<__nv_bfloat16>::st(static_cast<__nv_bfloat16*>(a.o) + static_cast<size_t>(n) * a.ld_o + (hq_base + hh) * HD + d,
-                           a.o_plane, O / Ls);
+                           a.o_plane, O * rinv[qi]);
   }
   cluster.sync();   // every rank keeps its shared memory until all have read it
 }
