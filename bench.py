@@ -179,6 +179,20 @@ def cpu_baseline_dict(res, w, cores):
 
 
 # ---------------------------------------------------------------- main
+def combine_ranks(ms, committed, world):
+    """Whole-job figures over replica ranks: the slowest rank's time and the
+    tokens every rank committed (max and sum over the process group)."""
+    if world <= 1:
+        return ms, float(committed)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms, float(committed)], dtype=torch.float64)
+    tmax = t.clone()
+    dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(tmax[0]), float(t[1])
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -286,14 +300,7 @@ def main():
     dsteps = st1["steps"] - st0["steps"]
     mat = (st1["accepted"] - st0["accepted"]) / max(1, dsteps * w.batch)
     launches = st1["kernel_launches"] - st0["kernel_launches"]
-    if world > 1:
-        t = torch.tensor([ms, float(committed)], dtype=torch.float64)
-        tmax = t.clone()
-        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        ms_all, committed_all = float(tmax[0]), float(t[1])
-    else:
-        ms_all, committed_all = ms, float(committed)
+    ms_all, committed_all = combine_ranks(ms, committed, world)
     value = committed_all / (ms_all / 1e3)
 
     # roofline of the verify pass (and the draft pass), from the phase timing
