@@ -15,8 +15,9 @@
 // rule, and positions a row must not see contribute exact zeros, so a row's
 // output does not depend on how many rows share the launch.
 //
-// The bf16 tensor-core decode kernel (attn_mma_kernel) instead splits each
-// row's own positions evenly: see the rule at its split set-up.
+// The bf16 tensor-core kernel (attn_mma_kernel; decode passes and prefill
+// chunks) instead splits each row's own positions evenly: see the rule at
+// its split set-up.
 //
 // Decode (<= 16 rows per sequence): attn_dec_kernel streams the split's K/V
 // through a shared-memory ring by bulk copies and keeps a query group's
@@ -839,8 +840,9 @@ template <typename T>
 static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
   const bool bf16 = sizeof(T) == 2;
   dim3 grid(a.n_splits_max, a.n_kv_heads, a.n_seqs * n_qgroups(a, bf16));
-  if (bf16 && use_reg_kernel(a.rows_per_seq, a.n_heads / a.n_kv_heads)) {
-    // one cluster of n_splits_max (<= 8) CTAs per (sequence, query group, KV head)
+  if (bf16 && a.n_heads / a.n_kv_heads <= kRegQ) {
+    // one cluster of n_splits_max (<= 8) CTAs per (sequence, query group, KV
+    // head); decode and prefill chunks alike (16 / G query rows per group)
     const size_t smem = 1024 + static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * 2;
     static bool mma_attr = false;
     if (!mma_attr) {

@@ -442,7 +442,7 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   t.seq0 = ps.seq0;
   t.n_seqs = ps.n_seqs;
   t.pos_off = ps.pos_off;
-  const bool dec_cluster = ctx->tc && ps.rows_per_seq <= 16 && ctx->Hq / ctx->Hkv <= 8;
+  const bool dec_cluster = ctx->tc && ctx->Hq / ctx->Hkv <= 8;   // the tensor-core kernel
   t.split_len = dec_cluster ? 0 : ctx->attn_split_len;
   t.n_splits_max = dec_cluster ? ctx->dec_nsplits : ctx->attn_nsplits;
   t.part = ctx->attn_part;
