@@ -7,8 +7,8 @@
 //
 //  update_prep      UB[n] = B u_n                               (LoRA down)
 //  (projection)     Z = U W^S^T + gamma UB A^T                  (EPI_HEAD)
-//  update_rowstats  per row: log-normalisers of z, l/tau, l; KL(p||q),
-//                   KL(p||q1), H[p], -log p(a), -log p(y*)
+//  update_rowstats  per row: log-normalisers of z, l/tau, l (one online
+//                   pass); KL(p||q), KL(p||q1), H[p], -log p(a), -log p(y*)
 //  update_coef      the schedule's term weights at update t, the means that
 //                   form the loss, per-row gradient coefficients; the EMA
 //                   baseline b moves after the loss is formed
@@ -44,81 +44,145 @@ enum { DS_T = 0, DS_B, DS_LOSS, DS_KL, DS_PG, DS_CE, DS_ENT, DS_RL, DS_KL1, DS_A
 
 __device__ __forceinline__ bool row_valid(const UpdateArgs& a, int n) { return a.log_meta[n * 6] != 0; }
 
+// grid (cap, ceil(r/4)); warp w of CTA (n, y) forms UB[n][4y + w] = B_j . u_n
+// (lanes take 4 consecutive features per step, eight steps in flight).
 template <typename T>
 __global__ void __launch_bounds__(128) update_prep_kernel(const UpdateArgs a) {
   griddep_launch();
   griddep_wait();
   const int n = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = blockIdx.y * 4 + warp;
+  if (j >= a.r) return;
   if (!row_valid(a, n)) {
-    for (int j = threadIdx.x; j < a.r; j += 128) a.ub[n * a.r + j] = 0.f;
+    if (lane == 0) a.ub[n * a.r + j] = 0.f;
     return;
   }
   const T* u = static_cast<const T*>(a.log_u) + static_cast<size_t>(n) * a.d;
-  for (int j = warp; j < a.r; j += 4) {
-    const float* br = a.lora_b + static_cast<size_t>(j) * a.d;
-    float acc = 0.f;
-    for (int c = lane; c < a.d; c += 32) acc = fmaf(br[c], Act<T>::ld(u + c, a.log_plane), acc);
-    acc = warp_sum(acc);
-    if (lane == 0) a.ub[n * a.r + j] = acc;
+  const float4* br = reinterpret_cast<const float4*>(a.lora_b + static_cast<size_t>(j) * a.d);
+  float acc = 0.f;
+#pragma unroll 8
+  for (int c4 = lane; c4 < a.d / 4; c4 += 32) {
+    const float4 b4 = br[c4];
+    const T* uc = u + c4 * 4;
+    acc = fmaf(b4.x, Act<T>::ld(uc, a.log_plane), acc);
+    acc = fmaf(b4.y, Act<T>::ld(uc + 1, a.log_plane), acc);
+    acc = fmaf(b4.z, Act<T>::ld(uc + 2, a.log_plane), acc);
+    acc = fmaf(b4.w, Act<T>::ld(uc + 3, a.log_plane), acc);
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) a.ub[n * a.r + j] = acc;
+}
+
+// (m, s) pairs of log-sum-exp: merge of two partial maxima and sums.
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  const float M = fmaxf(m, m2);
+  if (M == -INFINITY) return;
+  s = (m == -INFINITY ? 0.f : s * expf(m - M)) + (m2 == -INFINITY ? 0.f : s2 * expf(m2 - M));
+  m = M;
+}
+__device__ __forceinline__ void lse_add(float& m, float& s, float x) {
+  if (x == -INFINITY) return;
+  if (x > m) {
+    s = (m == -INFINITY ? 0.f : s * expf(m - x)) + 1.f;
+    m = x;
+  } else {
+    s += expf(x - m);
   }
 }
 
-__device__ float block_reduce(float v, float* red, bool is_max) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  v = is_max ? warp_max(v) : warp_sum(v);
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  float r = red[0];
-  for (int w = 1; w < nw; ++w) r = is_max ? fmaxf(r, red[w]) : r + red[w];
-  return r;
-}
-
-__global__ void __launch_bounds__(256) update_rowstats_kernel(const UpdateArgs a) {
+// One CTA of 512 threads per buffer row: a single pass for the three
+// log-normalisers (online max / sum of exponentials), then one for KL(p||q),
+// KL(p||q1) and H[p]; float4 loads when V is a multiple of 4.
+__global__ void __launch_bounds__(512) update_rowstats_kernel(const UpdateArgs a) {
   griddep_launch();
   griddep_wait();
-  __shared__ float red[8];
+  __shared__ float red[16][6];
   const int n = blockIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
   float* rs = a.rowstat + n * RS_N;
   if (!row_valid(a, n)) {
-    if (threadIdx.x < RS_N) rs[threadIdx.x] = 0.f;
+    if (tid < RS_N) rs[tid] = 0.f;
     return;
   }
   const float* z = a.Z + static_cast<size_t>(n) * a.V;
   const float* l = a.log_logits + static_cast<size_t>(n) * a.V;
   const float it = 1.f / a.cfg.tau;
-  float mz = -INFINITY, mq = -INFINITY, mq1 = -INFINITY;
-  for (int v = threadIdx.x; v < a.V; v += blockDim.x) {
-    mz = fmaxf(mz, z[v]);
-    mq = fmaxf(mq, l[v] * it);
-    mq1 = fmaxf(mq1, l[v]);
+  const bool vec = (a.V & 3) == 0;
+  const int nv = vec ? a.V / 4 : a.V;
+  float mz = -INFINITY, sz = 0.f, mq = -INFINITY, sq = 0.f, mq1 = -INFINITY, sq1 = 0.f;
+  for (int i = tid; i < nv; i += blockDim.x) {
+    if (vec) {
+      const float4 z4 = reinterpret_cast<const float4*>(z)[i];
+      const float4 l4 = reinterpret_cast<const float4*>(l)[i];
+      const float zz[4] = {z4.x, z4.y, z4.z, z4.w}, ll[4] = {l4.x, l4.y, l4.z, l4.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        lse_add(mz, sz, zz[e]);
+        lse_add(mq, sq, ll[e] * it);
+        lse_add(mq1, sq1, ll[e]);
+      }
+    } else {
+      lse_add(mz, sz, z[i]);
+      lse_add(mq, sq, l[i] * it);
+      lse_add(mq1, sq1, l[i]);
+    }
   }
-  mz = block_reduce(mz, red, true);
-  mq = block_reduce(mq, red, true);
-  mq1 = block_reduce(mq1, red, true);
-  float sz = 0.f, sq = 0.f, sq1 = 0.f;
-  for (int v = threadIdx.x; v < a.V; v += blockDim.x) {
-    sz += expf(z[v] - mz);
-    sq += expf(l[v] * it - mq);
-    sq1 += expf(l[v] - mq1);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lse_merge(mz, sz, __shfl_xor_sync(0xffffffffu, mz, o), __shfl_xor_sync(0xffffffffu, sz, o));
+    lse_merge(mq, sq, __shfl_xor_sync(0xffffffffu, mq, o), __shfl_xor_sync(0xffffffffu, sq, o));
+    lse_merge(mq1, sq1, __shfl_xor_sync(0xffffffffu, mq1, o), __shfl_xor_sync(0xffffffffu, sq1, o));
   }
-  sz = block_reduce(sz, red, false);
-  sq = block_reduce(sq, red, false);
-  sq1 = block_reduce(sq1, red, false);
+  if (lane == 0) {
+    red[warp][0] = mz; red[warp][1] = sz; red[warp][2] = mq; red[warp][3] = sq; red[warp][4] = mq1; red[warp][5] = sq1;
+  }
+  __syncthreads();
+  mz = red[0][0]; sz = red[0][1]; mq = red[0][2]; sq = red[0][3]; mq1 = red[0][4]; sq1 = red[0][5];
+  for (int w = 1; w < nw; ++w) {
+    lse_merge(mz, sz, red[w][0], red[w][1]);
+    lse_merge(mq, sq, red[w][2], red[w][3]);
+    lse_merge(mq1, sq1, red[w][4], red[w][5]);
+  }
+  __syncthreads();
   const float lz = mz + logf(sz), lq = mq + logf(sq), lq1 = mq1 + logf(sq1);
   float kl = 0.f, kl1 = 0.f, ent = 0.f;
-  for (int v = threadIdx.x; v < a.V; v += blockDim.x) {
-    const float lp = z[v] - lz;
-    const float p = expf(lp);
-    kl = fmaf(p, lp - (l[v] * it - lq), kl);
-    kl1 = fmaf(p, lp - (l[v] - lq1), kl1);
-    ent = fmaf(-p, lp, ent);
+  for (int i = tid; i < nv; i += blockDim.x) {
+    float zz[4], ll[4];
+    int ne = 1;
+    if (vec) {
+      const float4 z4 = reinterpret_cast<const float4*>(z)[i];
+      const float4 l4 = reinterpret_cast<const float4*>(l)[i];
+      zz[0] = z4.x; zz[1] = z4.y; zz[2] = z4.z; zz[3] = z4.w;
+      ll[0] = l4.x; ll[1] = l4.y; ll[2] = l4.z; ll[3] = l4.w;
+      ne = 4;
+    } else {
+      zz[0] = z[i];
+      ll[0] = l[i];
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      if (e < ne) {
+        const float lp = zz[e] - lz;
+        const float p = expf(lp);
+        kl = fmaf(p, lp - (ll[e] * it - lq), kl);
+        kl1 = fmaf(p, lp - (ll[e] - lq1), kl1);
+        ent = fmaf(-p, lp, ent);
+      }
+    }
   }
-  kl = block_reduce(kl, red, false);
-  kl1 = block_reduce(kl1, red, false);
-  ent = block_reduce(ent, red, false);
-  if (threadIdx.x == 0) {
+  kl = warp_sum(kl);
+  kl1 = warp_sum(kl1);
+  ent = warp_sum(ent);
+  if (lane == 0) {
+    red[warp][0] = kl; red[warp][1] = kl1; red[warp][2] = ent;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    kl = 0.f; kl1 = 0.f; ent = 0.f;
+    for (int w = 0; w < nw; ++w) {
+      kl += red[w][0]; kl1 += red[w][1]; ent += red[w][2];
+    }
     const int* meta = a.log_meta + n * 6;
     rs[RS_LSEZ] = lz;
     rs[RS_LSEQ] = lq;
@@ -298,33 +362,56 @@ __global__ void __launch_bounds__(128) update_grad_a_kernel(const UpdateArgs a) 
   }
 }
 
-__global__ void update_ga_reduce_kernel(const UpdateArgs a) {
+// GA[n][j] = sum over vocabulary tiles of the partials: 256 threads per row,
+// thread (part, j) sums tiles t = part (mod parts), then the parts in order.
+__global__ void __launch_bounds__(256) update_ga_reduce_kernel(const UpdateArgs a) {
   griddep_launch();
   griddep_wait();
+  __shared__ float ps[256];
   if (a.dev_state[DS_SKIP] != 0.f) return;
-  const int n = blockIdx.x, j = threadIdx.x;
-  if (j >= a.r) return;
+  const int n = blockIdx.x, tid = threadIdx.x;
+  const int parts = 256 / a.r;
+  const int j = tid % a.r, part = tid / a.r;
   float acc = 0.f;
-  for (int t = 0; t < a.n_vtiles; ++t) acc += a.ga_part[(static_cast<size_t>(t) * a.cap + n) * a.r + j];
-  a.ga[n * a.r + j] = acc;
+  if (part < parts) {
+#pragma unroll 4
+    for (int t = part; t < a.n_vtiles; t += parts) acc += a.ga_part[(static_cast<size_t>(t) * a.cap + n) * a.r + j];
+  }
+  ps[tid] = acc;
+  __syncthreads();
+  if (tid < a.r) {
+    float s = 0.f;
+    for (int q = 0; q < parts; ++q) s += ps[q * a.r + tid];
+    a.ga[n * a.r + tid] = s;
+  }
 }
 
+// grid (ceil(d/128), ceil(r/4)): thread c of CTA (x, y) forms dB[j][c] for
+// the four j = 4y.. of the CTA (one pass over the buffer rows) and steps them.
 template <typename T>
 __global__ void __launch_bounds__(128) update_grad_b_kernel(const UpdateArgs a) {
   griddep_launch();
   griddep_wait();
   if (a.dev_state[DS_SKIP] != 0.f) return;
   const int c = blockIdx.x * 128 + threadIdx.x;
+  const int j0 = blockIdx.y * 4;
   if (c >= a.d) return;
   const float step = a.dev_state[DS_ADAM];
-  for (int j = 0; j < a.r; ++j) {
-    float acc = 0.f;
-    for (int n = 0; n < a.cap; ++n) {
-      if (!row_valid(a, n)) continue;
-      acc = fmaf(a.ga[n * a.r + j],
-                 Act<T>::ld(static_cast<const T*>(a.log_u) + static_cast<size_t>(n) * a.d + c, a.log_plane), acc);
-    }
-    const float g = a.gamma * acc;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  const T* u = static_cast<const T*>(a.log_u) + c;
+#pragma unroll 4
+  for (int n = 0; n < a.cap; ++n) {
+    if (!row_valid(a, n)) continue;
+    const float un = Act<T>::ld(u + static_cast<size_t>(n) * a.d, a.log_plane);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (j0 + q < a.r) acc[q] = fmaf(a.ga[n * a.r + j0 + q], un, acc[q]);
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int j = j0 + q;
+    if (j >= a.r) break;
+    const float g = a.gamma * acc[q];
     const size_t i = static_cast<size_t>(j) * a.d + c;
     a.grad_b[i] = g;
     opt_step(a.cfg, step, g, a.lora_b + i, a.m_b + i, a.v_b + i);
@@ -476,13 +563,14 @@ __global__ void update_finish_kernel(const UpdateArgs a) {
 
 cudaError_t launch_update_prep(const UpdateArgs& a, cudaStream_t s) {
   if (a.r == 0) return cudaSuccess;
-  const cudaError_t e = a.dtype == DVI_BF16 ? launch_pdl(update_prep_kernel<__nv_bfloat16>, dim3(a.cap), dim3(128), 0, s, a)
-                                            : launch_pdl(update_prep_kernel<float>, dim3(a.cap), dim3(128), 0, s, a);
+  const dim3 grid(a.cap, (a.r + 3) / 4);
+  const cudaError_t e = a.dtype == DVI_BF16 ? launch_pdl(update_prep_kernel<__nv_bfloat16>, grid, dim3(128), 0, s, a)
+                                            : launch_pdl(update_prep_kernel<float>, grid, dim3(128), 0, s, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 cudaError_t launch_update_rowstats(const UpdateArgs& a, cudaStream_t s) {
-  const cudaError_t e = launch_pdl(update_rowstats_kernel, dim3(a.cap), dim3(256), 0, s, a);
+  const cudaError_t e = launch_pdl(update_rowstats_kernel, dim3(a.cap), dim3(512), 0, s, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -505,10 +593,11 @@ cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s) {
 }
 cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s) {
   if (a.r == 0) return cudaSuccess;
-  cudaError_t e = launch_pdl(update_ga_reduce_kernel, dim3(a.cap), dim3(64), 0, s, a);
+  cudaError_t e = launch_pdl(update_ga_reduce_kernel, dim3(a.cap), dim3(256), 0, s, a);
   if (e != cudaSuccess) return e;
-  e = a.dtype == DVI_BF16 ? launch_pdl(update_grad_b_kernel<__nv_bfloat16>, dim3((a.d + 127) / 128), dim3(128), 0, s, a)
-                          : launch_pdl(update_grad_b_kernel<float>, dim3((a.d + 127) / 128), dim3(128), 0, s, a);
+  const dim3 grid((a.d + 127) / 128, (a.r + 3) / 4);
+  e = a.dtype == DVI_BF16 ? launch_pdl(update_grad_b_kernel<__nv_bfloat16>, grid, dim3(128), 0, s, a)
+                          : launch_pdl(update_grad_b_kernel<float>, grid, dim3(128), 0, s, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
