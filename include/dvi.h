@@ -82,7 +82,7 @@ typedef struct {
 
 typedef struct {
   int batch;            /* B sequences decoded together */
-  int k_spec;           /* K: drafted tokens per step, 1 <= K <= 16 / (H_q / H_kv) */
+  int k_spec;           /* K: drafted tokens per step, 1 <= K <= 16 (K + bonus <= 16) */
   int max_seq_len;      /* KV rows per sequence: prompt + generated + K */
   int log_steps;        /* decode steps the replay buffer holds between updates (U) */
   int head_mode;        /* 0: train LoRA A_s, B_s on the frozen W^(S); 1: train W^(S) itself
