@@ -318,8 +318,9 @@ class DVIEngine:
         Each prompt is copied from pinned host memory, prefilled, then steps
         run until every sequence has n_gen tokens; an update of the drafter
         runs after every `update_every` logged steps of the engine (counted
-        across calls, so a later call continues the drafter's schedule).  Replay-buffer logging is on when
-        updates are requested (or when `log` says so).  Returns (tokens per
+        across calls, so a later call continues the drafter's schedule).
+        Replay-buffer logging is on when updates are requested (or when
+        `log` says so).  Returns (tokens per
         sequence, per-step accept lengths [steps, B], bytes h2d, bytes d2h).
         """
         self.log(bool(update_every and hyper is not None) if log is None else log)
