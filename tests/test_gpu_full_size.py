@@ -12,7 +12,9 @@ size:
   oracle (float32 arithmetic on the bf16-rounded weights, bf16 KV cache),
   within 3e-2 (1B and 7B);
 * the 8-sequence ragged batch over two prompt waves whose drafter state
-  carries over, and the 16K-token prompt with K = 8.
+  carries over, and the 16K-token prompt with K = 8;
+* one LoRA update at the 7B shape: dA, dB against the oracle's closed-form
+  gradients on the GPU's own logged tuples, within 1e-3.
 """
 import functools
 
@@ -130,3 +132,49 @@ def test_7b_16k_prompt_lossless():
     P = make_prompts(w)
     assert len(P[0]) == 16384
     _lossless(w, dw, P, n_gen=16)
+
+
+def test_7b_update_gradients_on_logged_tuples():
+    """One LoRA update at the 7B shape: dA, dB against the oracle's closed-form
+    gradients on the GPU's own logged tuples (Sec. 3.4), within 1e-3 of the
+    largest entry."""
+    from oracle.update import grad_logits, head_logits, objective_weights, param_grads
+    from workloads import UpdateHyper
+    from gpu_helpers import logged_u
+    from workloads.gen import bf16_round
+    w = workload("7b")
+    W, dw = _weights("7b")
+    rng = np.random.default_rng(5)
+    a0 = (rng.standard_normal(W.lora_a.shape) * 0.05).astype(np.float32)
+    b_saved = dw.lora_b.clone()
+    dw.lora_a.copy_(torch.from_numpy(a0))
+    hyper = UpdateHyper(objective="dvi", lr=1e-3, t_warmup=0, t_ramp=0, w_ent=0.01, w_ce=0.05)
+    P = make_prompts(w)
+    eng = _engine(w, dw, _capacity(w, P))
+    eng.generate(P, 10 ** 6, max_steps=w.update_every, log=True)
+    eng.sync()
+    V, d = w.shape.vocab, w.shape.d_model
+    meta = eng.buffer("LOG_META", torch.int32).view(-1, 6).cpu().numpy()
+    lg = eng.buffer("LOG_LOGITS", torch.float32).view(-1, V).cpu().numpy().astype(np.float64)
+    lu = logged_u(eng, w)
+    b0 = dw.lora_b.cpu().numpy().astype(np.float64)
+    eng.update(hyper)
+    eng.sync()
+    ga = eng.buffer("GRAD_A", torch.float32).view(V, -1).cpu().numpy()
+    gb = eng.buffer("GRAD_B", torch.float32).view(w.lora_rank, -1).cpu().numpy()
+    st = eng.stats()
+    eng.close()
+    dw.lora_a.zero_()                 # the cached weights serve the other tests
+    dw.lora_b.copy_(b_saved)
+    assert st["device_status"] == 0, st["device_flags"]
+    rows = np.nonzero(meta[:, 0])[0]
+    assert len(rows) > 0
+    w_s = bf16_round(W.draft_head).astype(np.float64)
+    A = a0.astype(np.float64)
+    Z = head_logits(lu[rows], w_s, A, b0, w.lora_gamma)
+    G = grad_logits(Z, lg[rows], meta[rows, 1], meta[rows, 5], meta[rows, 2].astype(np.float64),
+                    objective_weights(0, hyper), 0.0)
+    ref = param_grads(G, lu[rows], A, b0, w.lora_gamma)
+    for name, got in (("A", ga), ("B", gb)):
+        rel = np.abs(got - ref[name]).max() / np.abs(ref[name]).max()
+        assert rel < 1e-3, (name, rel)
