@@ -96,6 +96,12 @@ typedef struct {
                            1: one more shallow pass on t~_K and a (K+1)-th verify row, so the
                            correction y*_{n+K+1} exists at m = K and every step commits m+1
                            tokens.  K + bonus <= 16. */
+  int persistent;       /* 0: one kernel per projection.  1: bf16 decode passes of up to 64
+                           rows run each layer's O, gate/up and down projections and the next
+                           layer's QKV as one persistent launch (attention stays a launch of
+                           its own); the context then needs every CTA of that launch resident
+                           at once (two per SM) and ignores the flag when they do not fit.
+                           Results differ from mode 0 in summation order only. */
 } dvi_runtime_config;
 
 typedef struct {
@@ -157,6 +163,8 @@ typedef struct {
   float baseline_b;       /* EMA reward baseline after the last update */
   int update_t;           /* completed updates t (the schedule's clock) */
   int device_status;      /* DVI_DEV_* bits */
+  int persistent_ctas;    /* grid of the persistent projection launch (runtime option
+                             persistent = 1 in effect), else 0 */
 } dvi_stats;
 
 /* Bytes of device workspace a context needs (KV caches, residual streams,

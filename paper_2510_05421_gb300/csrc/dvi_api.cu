@@ -80,6 +80,10 @@ struct dvi_ctx {
   int n_attn_ctr;
   int attn_split_len, attn_nsplits;
   int dec_nsplits;                  // bf16 decode attention: splits (one cluster) per KV head
+  int chain_ctas = 0;               // persistent projection chain: grid size (0: not used)
+  float* chain_part = nullptr;
+  size_t chain_part_floats = 0;
+  int* chain_ctr = nullptr;
   void* log_u;
   float* log_logits;
   float *Z, *rowstat, *coef, *ub, *ga, *ga_part;
@@ -144,6 +148,7 @@ bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::
   if (rt->batch < 1 || rt->batch > 64) return bad("batch must be in [1, 64]");
   if (rt->k_spec < 1 || rt->k_spec > 16) return bad("k_spec must be in [1, 16]");
   if (rt->bonus != 0 && rt->bonus != 1) return bad("bonus must be 0 or 1");
+  if (rt->persistent != 0 && rt->persistent != 1) return bad("persistent must be 0 or 1");
   if (rt->k_spec + rt->bonus > 16) return bad("k_spec + bonus must be <= 16");
   if (rt->max_seq_len < rt->k_spec + 2) return bad("max_seq_len too small");
   if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
@@ -200,6 +205,8 @@ size_t layout(dvi_ctx* c, char* base) {
   c->proj_counters = reinterpret_cast<int*>(take(sizeof(int) * c->n_proj_counters));
   c->attn_part = reinterpret_cast<float*>(take(sizeof(float) * c->attn_part_floats));
   c->attn_ctr = reinterpret_cast<int*>(take(sizeof(int) * c->n_attn_ctr));
+  c->chain_part = reinterpret_cast<float*>(take(sizeof(float) * c->chain_part_floats));
+  c->chain_ctr = reinterpret_cast<int*>(take(sizeof(int) * (kChainMax + kChainMax * kChainTiles + 4)));
   c->log_u = take(pl * e * c->cap_rows * d);
   c->log_logits = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
   c->Z = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
@@ -293,6 +300,20 @@ void size_scratch(dvi_ctx* c) {
   }
   c->attn_part_floats = ap;
   c->n_attn_ctr = ac;
+  // persistent projection chain (runtime option; bf16 passes of up to
+  // kChainMaxPad rows): as many CTAs as the SMs keep resident at every n_pad
+  c->chain_ctas = 0;
+  c->chain_part_floats = 0;
+  if (c->tc && c->rt.persistent) {
+    int per_sm = 2;
+    for (int np = 16; np <= kChainMaxPad; np += 16) per_sm = std::min(per_sm, chain_ctas_per_sm(np));
+    const int max_tiles =
+        std::max(std::max(c->p_qkv.n_tiles, c->p_o.n_tiles), std::max(c->p_gu.n_tiles, c->p_down.n_tiles));
+    if (per_sm > 0 && max_tiles <= kChainTiles) {
+      c->chain_ctas = per_sm * c->n_sms;
+      c->chain_part_floats = chain_partial_floats(max_tiles, c->chain_ctas, kChainMaxPad);
+    }
+  }
 }
 
 bool init_dims(dvi_ctx* c, const dvi_model_config* cfg, const dvi_runtime_config* rt) {
@@ -390,17 +411,18 @@ cudaError_t launch_proj_ctx(const dvi_ctx* c, ProjArgs a, const ProjMaps* m, cud
   return launch_proj(a, m, s);
 }
 
-// One decoder layer on the pass's rows.  `g_last` is the gain of whatever
-// consumes the pass's residual after this layer (the next layer's attention
-// norm, or the final norm before a head).
-dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last) {
+struct ProjLaunch {
+  ProjArgs a;
+  ProjMaps m;
+};
+
+// q, k, v of RMSNorm(x) (gain folded into xg, 1/rms in the epilogue), RoPE,
+// k/v rows into the cache
+ProjLaunch qkv_launch(dvi_ctx* ctx, int l, const Pass& ps) {
   const dvi_layer_weights& lw = ctx->layers[l];
-  const bool tc = ctx->tc;
-  cudaStream_t s = ctx->stream;
-  ProjMaps pm{};
-  // q, k, v of RMSNorm(x) (gain folded into xg, 1/rms in the epilogue), RoPE,
-  // k/v rows into the cache
-  ProjArgs a = base_args(ctx, EPI_QKV, ctx->p_qkv, ps);
+  ProjLaunch r{};
+  ProjArgs& a = r.a;
+  a = base_args(ctx, EPI_QKV, ctx->p_qkv, ps);
   a.act = ps.xg;
   a.ld_act = ctx->d;
   a.ss = ps.ss;
@@ -421,14 +443,17 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.head_dim = ctx->hd;
   a.n_kv_heads = ctx->Hkv;
   a.rope = ctx->rope;
-  if (tc) pm = with_act(ctx->maps[l].qkv, ps.xg_map);
-  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
-  // block-causal multi-query attention
+  if (ctx->tc) r.m = with_act(ctx->maps[l].qkv, ps.xg_map);
+  return r;
+}
+
+// block-causal multi-query attention of layer l
+AttnArgs attn_args(dvi_ctx* ctx, int l, const Pass& ps) {
   AttnArgs t{};
   t.q = ctx->q;
   t.ld_q = ctx->nq;
-  t.kc = a.kc;
-  t.vc = a.vc;
+  t.kc = static_cast<char*>(ctx->kcache) + layer_kv_offset(ctx, l);
+  t.vc = static_cast<char*>(ctx->vcache) + layer_kv_offset(ctx, l);
   t.o = ctx->attn_o;
   t.ld_o = ctx->nq;
   t.o_dtype = ctx->cfg.dtype;
@@ -453,8 +478,14 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   t.kmap = &ctx->map_kc;
   t.vmap = &ctx->map_vc;
   t.o_plane = act_plane(ctx, ctx->attn_o, ctx->nq);
-  DVI_CUDA(launch_attn(t, s));
-  // x += W_o . attn, then xg = x * ffn_norm for the FFN
+  return t;
+}
+
+// x += W_o . attn, then xg = x * ffn_norm for the FFN
+ProjLaunch o_launch(dvi_ctx* ctx, int l, const Pass& ps) {
+  const dvi_layer_weights& lw = ctx->layers[l];
+  ProjLaunch r{};
+  ProjArgs& a = r.a;
   a = base_args(ctx, EPI_RESID, ctx->p_o, ps);
   a.act = ctx->attn_o;
   a.ld_act = ctx->nq;
@@ -468,9 +499,15 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.g_next = static_cast<const float*>(lw.ffn_norm);
   a.xg_out = ps.xg;
   a.ld_xg = ctx->d;
-  if (tc) pm = with_act(ctx->maps[l].o, &ctx->map_attn_o);
-  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
-  // h = SiLU(W_gate n) * (W_up n) with n = RMSNorm(x)
+  if (ctx->tc) r.m = with_act(ctx->maps[l].o, &ctx->map_attn_o);
+  return r;
+}
+
+// h = SiLU(W_gate n) * (W_up n) with n = RMSNorm(x)
+ProjLaunch gu_launch(dvi_ctx* ctx, int l, const Pass& ps) {
+  const dvi_layer_weights& lw = ctx->layers[l];
+  ProjLaunch r{};
+  ProjArgs& a = r.a;
   a = base_args(ctx, EPI_GATEUP, ctx->p_gu, ps);
   a.act = ps.xg;
   a.ld_act = ctx->d;
@@ -482,9 +519,15 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.w1 = lw.w_up;
   a.h_out = ctx->ffn_h;
   a.ld_h = ctx->F;
-  if (tc) pm = with_act(ctx->maps[l].gu, ps.xg_map);
-  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
-  // x += W_down . h, then xg = x * (next norm's gain)
+  if (ctx->tc) r.m = with_act(ctx->maps[l].gu, ps.xg_map);
+  return r;
+}
+
+// x += W_down . h, then xg = x * g_last (the gain of the norm after the layer)
+ProjLaunch down_launch(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last) {
+  const dvi_layer_weights& lw = ctx->layers[l];
+  ProjLaunch r{};
+  ProjArgs& a = r.a;
   a = base_args(ctx, EPI_RESID, ctx->p_down, ps);
   a.act = ctx->ffn_h;
   a.ld_act = ctx->F;
@@ -498,10 +541,66 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   a.g_next = g_last;
   a.xg_out = ps.xg;
   a.ld_xg = ctx->d;
-  if (tc) pm = with_act(ctx->maps[l].down, &ctx->map_ffn_h);
-  DVI_CUDA(launch_proj_ctx(ctx, a, tc ? &pm : nullptr, s));
-  ctx->launches += 5;
+  if (ctx->tc) r.m = with_act(ctx->maps[l].down, &ctx->map_ffn_h);
+  return r;
+}
+
+dvi_status run_proj(dvi_ctx* ctx, const ProjLaunch& pl) {
+  DVI_CUDA(launch_proj_ctx(ctx, pl.a, ctx->tc ? &pl.m : nullptr, ctx->stream));
+  ++ctx->launches;
   return DVI_OK;
+}
+
+// Projections gathered for one persistent chain launch.
+struct ChainBuilder {
+  ChainArgs a;
+};
+
+void chain_reset(dvi_ctx* ctx, ChainBuilder& cb) {
+  memset(&cb.a, 0, sizeof(cb.a));
+  cb.a.n_ctas = ctx->chain_ctas;
+  cb.a.phase_done = ctx->chain_ctr;
+  cb.a.tile_ctr = ctx->chain_ctr + kChainMax;
+  cb.a.exit_ctr = ctx->chain_ctr + kChainMax + kChainMax * kChainTiles;
+  cb.a.part = ctx->chain_part;
+}
+
+void chain_add(dvi_ctx* ctx, ChainBuilder& cb, const ProjLaunch& pl) {
+  ProjArgs a = pl.a;
+  if (a.xg_out) a.xg_plane = act_plane(ctx, a.xg_out, a.ld_xg);
+  if (a.h_out) a.h_plane = act_plane(ctx, a.h_out, a.ld_h);
+  const int n = cb.a.n_phases++;
+  cb.a.p[n] = a;
+  cb.a.maps[n][0] = pl.m.m0;
+  cb.a.maps[n][1] = pl.m.m1;
+  cb.a.maps[n][2] = pl.m.m2;
+  cb.a.maps[n][3] = pl.m.mb;
+}
+
+dvi_status chain_flush(dvi_ctx* ctx, ChainBuilder& cb) {
+  if (cb.a.n_phases == 0) return DVI_OK;
+  DVI_CUDA(launch_chain(cb.a, ctx->stream));
+  ++ctx->launches;
+  chain_reset(ctx, cb);
+  return DVI_OK;
+}
+
+// The persistent chain serves bf16 passes of up to kChainMaxPad rows.
+bool use_chain(const dvi_ctx* ctx, const Pass& ps) {
+  return ctx->tc && ctx->chain_ctas > 0 && (ps.M + 15) / 16 * 16 <= kChainMaxPad;
+}
+
+// One decoder layer on the pass's rows, one kernel per projection.  `g_last`
+// is the gain of whatever consumes the pass's residual after this layer (the
+// next layer's attention norm, or the final norm before a head).
+dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last) {
+  dvi_status st;
+  if ((st = run_proj(ctx, qkv_launch(ctx, l, ps))) != DVI_OK) return st;
+  DVI_CUDA(launch_attn(attn_args(ctx, l, ps), ctx->stream));
+  ++ctx->launches;
+  if ((st = run_proj(ctx, o_launch(ctx, l, ps))) != DVI_OK) return st;
+  if ((st = run_proj(ctx, gu_launch(ctx, l, ps))) != DVI_OK) return st;
+  return run_proj(ctx, down_launch(ctx, l, ps, g_last));
 }
 
 // Gain of the RMSNorm that reads the residual after layer l-1: layer l's
@@ -512,13 +611,32 @@ const float* norm_gain_before(dvi_ctx* ctx, int l) {
 }
 
 // Layers lo..hi-1; after the last one xg holds x * final_norm for a head.
+// With the chain: QKV(lo), then per layer the attention kernel and one chain
+// of O, gate/up, down and the next layer's QKV.
 dvi_status enqueue_layers(dvi_ctx* ctx, int lo, int hi, const Pass& ps) {
-  for (int l = lo; l < hi; ++l) {
-    const float* g_last = l + 1 < hi ? norm_gain_before(ctx, l + 1) : static_cast<const float*>(ctx->w.final_norm);
-    dvi_status st = enqueue_layer(ctx, l, ps, g_last);
-    if (st != DVI_OK) return st;
+  if (!use_chain(ctx, ps)) {
+    for (int l = lo; l < hi; ++l) {
+      const float* g_last = l + 1 < hi ? norm_gain_before(ctx, l + 1) : static_cast<const float*>(ctx->w.final_norm);
+      dvi_status st = enqueue_layer(ctx, l, ps, g_last);
+      if (st != DVI_OK) return st;
+    }
+    return DVI_OK;
   }
-  return DVI_OK;
+  ChainBuilder cb;
+  chain_reset(ctx, cb);
+  dvi_status st;
+  for (int l = lo; l < hi; ++l) {
+    if (l == lo) chain_add(ctx, cb, qkv_launch(ctx, l, ps));
+    if ((st = chain_flush(ctx, cb)) != DVI_OK) return st;
+    DVI_CUDA(launch_attn(attn_args(ctx, l, ps), ctx->stream));
+    ++ctx->launches;
+    const float* g_last = l + 1 < hi ? norm_gain_before(ctx, l + 1) : static_cast<const float*>(ctx->w.final_norm);
+    chain_add(ctx, cb, o_launch(ctx, l, ps));
+    chain_add(ctx, cb, gu_launch(ctx, l, ps));
+    chain_add(ctx, cb, down_launch(ctx, l, ps, g_last));
+    if (l + 1 < hi) chain_add(ctx, cb, qkv_launch(ctx, l + 1, ps));
+  }
+  return chain_flush(ctx, cb);
 }
 
 StepState step_state(dvi_ctx* c) {
@@ -1028,6 +1146,7 @@ dvi_status dvi_get_stats(dvi_ctx* ctx, dvi_stats* out) {
   out->last_kl1 = ds[8];
   out->last_accept_rate = ds[9];
   out->device_status = status;
+  out->persistent_ctas = ctx->chain_ctas;
   return DVI_OK;
 }
 

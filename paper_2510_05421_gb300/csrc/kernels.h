@@ -82,6 +82,32 @@ bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols);   // 64-row boxes (gate/up)
 bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);   // [2 planes][rows][cols]
 
+// Persistent projection chain (bf16): up to kChainMax projections of one
+// pass in a single launch, each phase's output feeding the next phase's B
+// operand (O, gate/up, down, next layer's QKV).  Every CTA takes an equal
+// contiguous range of the phase's (tile, K block) sequence; a range that
+// covers only part of a tile leaves its partial sum in `part`, and the last
+// of the tile's CTAs to arrive sums the partials in K order and runs the
+// epilogue.  A phase's activation loads wait for every tile of the phase
+// before it (`phase_done`); its weight loads do not.
+constexpr int kChainMax = 4;
+constexpr int kChainTiles = 1024;   // tile counters per phase
+constexpr int kChainMaxPad = 64;    // largest n_pad (two TMEM accumulators of 2 n_pad columns)
+struct ChainArgs {
+  CUtensorMap maps[kChainMax][4];   // per phase: m0, m1, m2, mb
+  ProjArgs p[kChainMax];
+  int n_phases;
+  int n_ctas;             // grid size; fixed per context so the K ranges depend on the weight shape only
+  int* phase_done;        // [kChainMax] finished tiles per phase (reset by the last CTA to leave)
+  int* tile_ctr;          // [kChainMax][kChainTiles] arrivals per tile (reset by the tile's finisher)
+  int* exit_ctr;
+  float* part;            // [n_tiles + n_ctas][n_pad][128] partial slots (slot = tile + CTA)
+};
+// CTAs per SM the chain kernel keeps resident at n_pad (0 if it cannot run).
+int chain_ctas_per_sm(int n_pad);
+size_t chain_partial_floats(int max_tiles, int n_ctas, int n_pad);
+cudaError_t launch_chain(const ChainArgs& a, cudaStream_t s);
+
 struct AttnArgs {
   const float* q; int ld_q;          // rotated queries [M][H_q*hd]
   const void* kc; const void* vc;    // layer base of the caches [B][H_kv][max_len][hd]

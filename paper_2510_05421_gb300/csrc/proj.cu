@@ -36,6 +36,16 @@
 // global scratch and the last CTA to arrive (an atomic counter per tile) sums
 // them in split order.  Both are deterministic, and the split plan depends on
 // the weight shape only (never on the number of decode rows).
+//
+// Persistent chain (bf16, opt-in): one launch runs several projections of
+// a pass in order (a layer's O, gate/up, down and the next layer's QKV).
+// Each phase's (tile, K block) sequence is cut into equal contiguous ranges,
+// one per CTA (stream-K); a tile covered by several CTAs is summed in K
+// order by the CTA holding its first K block, from the others' partials in
+// global scratch.  A phase's activation loads wait on a release/acquire
+// counter of the previous phase's finished tiles (bounded polls); its weight
+// loads do not, so the ring fills across the boundary.  Every CTA must be
+// resident at once: the grid is the number of CTAs the SMs hold.
 #include <algorithm>
 #include <cudaTypedefs.h>
 
@@ -64,8 +74,17 @@ __device__ __forceinline__ void compute_rstd(const ProjArgs& p, float* rstd, int
   for (int n = tid; n < p.M; n += nthreads) {
     float r = 1.f;
     if (p.ss) {
+      // loads in batches of eight, summed in tile order
       float s = 0.f;
-      for (int t = 0; t < p.ss_tiles; ++t) s += p.ss[static_cast<size_t>(t) * p.ss_ld + n];
+      int t = 0;
+      for (; t + 8 <= p.ss_tiles; t += 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = __ldcg(p.ss + static_cast<size_t>(t + u) * p.ss_ld + n);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) s += x[u];
+      }
+      for (; t < p.ss_tiles; ++t) s += __ldcg(p.ss + static_cast<size_t>(t) * p.ss_ld + n);
       r = rsqrtf(s / static_cast<float>(p.d_norm) + p.eps);
     }
     rstd[n] = r;
@@ -144,7 +163,7 @@ __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int 
       float xn = 0.f;
       if (((own >> j) & 1u) && f < p.n_out) {
         float* xp = p.x_res + static_cast<size_t>(n) * p.ld_res + f;
-        xn = *xp + v[j];
+        xn = __ldcg(xp) + v[j];
         *xp = xn;
         if (p.xg_out) Act<T>::st(static_cast<T*>(p.xg_out) + static_cast<size_t>(n) * p.ld_xg + f, p.xg_plane, xn * g);
       }
@@ -547,6 +566,428 @@ __global__ void __launch_bounds__(192, 2)
   }
 }
 
+// ------------------------------------------------------------------ chain
+__device__ __forceinline__ int ld_acquire_gpu(const int* ptr) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_gpu_add(int* ptr, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
+}
+// Orders this thread's generic-proxy global accesses with its later (or
+// earlier) TMA accesses.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// CTAs that take part in a phase of `all` blocks: every one of them gets at
+// least one block, so a tile's contributors are consecutive CTAs.
+__device__ __forceinline__ int chain_width(long long all, int n_ctas) {
+  return static_cast<int>(all < n_ctas ? all : n_ctas);
+}
+// The CTA's share of one phase: K blocks [k0, k1) of the phase's sequence of
+// n_tiles x kb_total (tile-major) blocks.
+struct ChainRange {
+  long long k0[kChainMax];
+  int n[kChainMax];
+  int total;
+};
+__device__ __forceinline__ void chain_range(const ChainArgs& a, int cta, ChainRange& r) {
+  r.total = 0;
+#pragma unroll
+  for (int ph = 0; ph < kChainMax; ++ph) {
+    r.k0[ph] = 0;
+    r.n[ph] = 0;
+    if (ph < a.n_phases) {
+      const long long all = static_cast<long long>(a.p[ph].n_tiles) * a.p[ph].kb_total;
+      const int g = chain_width(all, a.n_ctas);
+      if (cta < g) {
+        r.k0[ph] = all * cta / g;
+        r.n[ph] = static_cast<int>(all * (cta + 1) / g - r.k0[ph]);
+        r.total += r.n[ph];
+      }
+    }
+  }
+}
+// Sequential walk over the CTA's blocks: phase, tile, K block within the tile.
+struct ChainCursor {
+  int ph, tile, kb, kbt, left;
+};
+__device__ __forceinline__ void cursor_settle(const ChainArgs& a, const ChainRange& r, ChainCursor& c) {
+  while (c.left == 0 && c.ph + 1 < a.n_phases) {
+    ++c.ph;
+    c.left = r.n[c.ph];
+    c.kbt = a.p[c.ph].kb_total;
+    c.tile = static_cast<int>(r.k0[c.ph] / c.kbt);
+    c.kb = static_cast<int>(r.k0[c.ph] - static_cast<long long>(c.tile) * c.kbt);
+  }
+}
+__device__ __forceinline__ void cursor_init(const ChainArgs& a, const ChainRange& r, ChainCursor& c) {
+  c.ph = -1;
+  c.left = 0;
+  cursor_settle(a, r, c);
+}
+__device__ __forceinline__ void cursor_next(const ChainArgs& a, const ChainRange& r, ChainCursor& c) {
+  --c.left;
+  if (++c.kb == c.kbt) {
+    c.kb = 0;
+    ++c.tile;
+  }
+  if (c.left == 0) cursor_settle(a, r, c);
+}
+// CTA whose range holds block k of a phase with `all` blocks.
+__device__ __forceinline__ int chain_owner(long long k, long long all, int n_ctas) {
+  const long long g = chain_width(all, n_ctas);
+  return static_cast<int>(((k + 1) * g + all - 1) / all) - 1;
+}
+
+constexpr uint32_t kChainPollLimit = 1u << 21;   // polls of another CTA's counter before giving up
+
+__global__ void __launch_bounds__(192, 2) proj_chain_kernel(const __grid_constant__ ChainArgs a, int stages) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  constexpr int abytes = 16384;
+  const int n_pad = a.p[0].n_pad;
+  const int bbytes = 2 * n_pad * 128;
+  uint8_t* sA = base;
+  uint8_t* sB = base + stages * abytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + stages * bbytes);
+  uint64_t* empty = full + stages;
+  uint64_t* accf = empty + stages;   // [2] accumulator b holds a finished segment
+  uint64_t* acce = accf + 2;         // [2] accumulator b has been read
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(acce + 2);
+  float* rstd = reinterpret_cast<float*>(tmem_holder + 4);
+  int* posn = reinterpret_cast<int*>(rstd + kMaxTokens);
+  EpiSmem& es = *reinterpret_cast<EpiSmem*>(posn + kMaxTokens);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cta = blockIdx.x;
+  const uint32_t bufcols = tmem_cols(2 * n_pad);
+  int* status = a.p[0].status;
+  ChainRange rg;
+  chain_range(a, cta, rg);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf[b], 1);
+      mbar_init(&acce[b], 1);
+    }
+    mbar_fence_init();
+  }
+  if (warp == 0) tmem_alloc(tmem_holder, 2 * bufcols);
+  if (warp == 4 && lane == 0) {
+    for (int ph = 0; ph < a.n_phases; ++ph) {
+      const int f = a.p[ph].flavor;
+      tma_prefetch_desc(&a.maps[ph][0]);
+      if (f == EPI_GATEUP || f == EPI_QKV) tma_prefetch_desc(&a.maps[ph][1]);
+      if (f == EPI_QKV) tma_prefetch_desc(&a.maps[ph][2]);
+      tma_prefetch_desc(&a.maps[ph][3]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  griddep_launch();
+  const uint32_t tmem = *tmem_holder;
+
+  if (warp == 4) {
+    // ---------------- TMA producer.  Weight loads run up to the ring's depth
+    // ahead of the activation loads, which wait for the previous phase.
+    if (lane == 0 && rg.total > 0) {
+      const uint64_t pol = l2_evict_first_policy();
+      const uint32_t tx = abytes + static_cast<uint32_t>(bbytes);
+      const int nbox = n_pad / 16;
+      auto load_a = [&](int j, const ChainCursor& c) {
+        const ProjArgs& p = a.p[c.ph];
+        const int x = c.kb * kKBlock;
+        uint8_t* dst = sA + (j % stages) * abytes;
+        uint64_t* bar = &full[j % stages];
+        if (p.flavor == EPI_GATEUP) {
+          tma_load_2d(dst, &a.maps[c.ph][0], x, c.tile * kGuRows, bar, pol);
+          tma_load_2d(dst + abytes / 2, &a.maps[c.ph][1], x, c.tile * kGuRows, bar, pol);
+        } else {
+          int m = 0, y = c.tile * kTileRows;
+          if (p.flavor == EPI_QKV) {
+            const int tq = p.rows_q / kTileRows, tk = p.rows_k / kTileRows;
+            if (c.tile >= tq + tk) { m = 2; y = (c.tile - tq - tk) * kTileRows; }
+            else if (c.tile >= tq) { m = 1; y = (c.tile - tq) * kTileRows; }
+          }
+          tma_load_2d(dst, &a.maps[c.ph][m], x, y, bar, pol);
+        }
+      };
+      auto load_b = [&](int j, const ChainCursor& c) {
+        const int x = c.kb * kKBlock;
+        const int row0 = a.p[c.ph].act_row0;
+        uint8_t* dst = sB + (j % stages) * bbytes;
+        uint64_t* bar = &full[j % stages];
+        for (int b = 0; b < nbox; ++b) {
+          tma_load_3d(dst + b * 2048, &a.maps[c.ph][3], x, row0 + b * 16, 0, bar, 0ull);
+          tma_load_3d(dst + (nbox + b) * 2048, &a.maps[c.ph][3], x, row0 + b * 16, 1, bar, 0ull);
+        }
+      };
+      int ia = 0, ib = 0;
+      ChainCursor ca, cb;
+      cursor_init(a, rg, ca);
+      cursor_init(a, rg, cb);
+      for (; ia < min(stages, rg.total); ++ia) {
+        mbar_arrive_expect_tx(&full[ia], tx);
+        load_a(ia, ca);
+        cursor_next(a, rg, ca);
+      }
+      griddep_wait();
+      int ready = 0;          // phases 0..ready may load activations
+      uint32_t idle = 0;
+      bool ok = true;
+      while (ib < rg.total) {
+        bool prog = false;
+        if (ib < ia) {
+          const int ph = cb.ph;
+          if (ph > ready && ld_acquire_gpu(a.phase_done + ph - 1) >= a.p[ph - 1].n_tiles) {
+            fence_proxy_async_global();
+            ready = ph;
+          }
+          if (ph <= ready) {
+            load_b(ib, cb);
+            cursor_next(a, rg, cb);
+            ++ib;
+            prog = true;
+          }
+        }
+        if (ia < rg.total && mbar_test_wait(&empty[ia % stages], ((ia / stages) & 1) ^ 1)) {
+          mbar_arrive_expect_tx(&full[ia % stages], tx);
+          load_a(ia, ca);
+          cursor_next(a, rg, ca);
+          ++ia;
+          prog = true;
+        }
+        if (prog) {
+          idle = 0;
+        } else if (++idle > kChainPollLimit) {
+          flag_status(status, DVI_DEV_TIMEOUT);
+          ok = false;
+          break;
+        } else if (idle > 16) {
+          __nanosleep(64);
+        }
+      }
+      if (!ok) {
+        // copies in flight land within microseconds; wait (bounded) for the
+        // stages whose activation loads were issued
+        for (int j = max(0, ib - stages); j < ib; ++j) mbar_wait(&full[j % stages], (j / stages) & 1, status);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 5) {
+    // ---------------- MMA issuer: one accumulator per segment (a run of
+    // blocks of one tile), alternating between two TMEM buffers
+    if (lane == 0 && rg.total > 0) {
+      const bool fused_lo = 2 * n_pad <= 256;
+      const uint32_t idesc = idesc_bf16_m128(static_cast<uint32_t>(fused_lo ? 2 * n_pad : n_pad));
+      int seg = -1, cur_ph = -1, cur_tile = -1;
+      uint32_t acc = tmem;
+      ChainCursor cm;
+      cursor_init(a, rg, cm);
+      for (int j = 0; j < rg.total; ++j, cursor_next(a, rg, cm)) {
+        const bool first = cm.ph != cur_ph || cm.tile != cur_tile;
+        if (first) {
+          if (seg >= 0) tc_commit(&accf[seg & 1]);
+          ++seg;
+          cur_ph = cm.ph;
+          cur_tile = cm.tile;
+          if (seg >= 2 && !mbar_wait(&acce[seg & 1], ((seg >> 1) - 1) & 1, status)) break;
+          tc_fence_after();
+          acc = tmem + static_cast<uint32_t>(seg & 1) * bufcols;
+        }
+        const int s = j % stages;
+        if (!mbar_wait(&full[s], (j / stages) & 1, status)) break;
+        tc_fence_after();
+        const uint32_t ab = smem_u32(sA + s * abytes);
+        const uint32_t bb = smem_u32(sB + s * bbytes);
+        const uint32_t blo = bb + static_cast<uint32_t>(n_pad) * 128u;
+#pragma unroll
+        for (int kk = 0; kk < kKBlock / 16; ++kk) {
+          const uint64_t ad = smem_desc_sw128(ab + kk * 32);
+          const uint32_t accum = (first && kk == 0) ? 0u : 1u;
+          tc_mma_bf16(acc, ad, smem_desc_sw128(bb + kk * 32), idesc, accum);
+          if (!fused_lo)
+            tc_mma_bf16(acc + static_cast<uint32_t>(n_pad), ad, smem_desc_sw128(blo + kk * 32), idesc, accum);
+        }
+        tc_commit(&empty[s]);
+      }
+      if (seg >= 0) tc_commit(&accf[seg & 1]);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- warps 0-3: partial tiles, reductions, epilogues
+    const int tid = threadIdx.x;
+    griddep_wait();
+    int seg = 0;
+    bool ok = true;
+    for (int ph = 0; ph < a.n_phases && ok; ++ph) {
+      const ProjArgs& p = a.p[ph];
+      const long long all = static_cast<long long>(p.n_tiles) * p.kb_total;
+      const int nchunks = (p.M + kChunk - 1) / kChunk;
+      const size_t slot = static_cast<size_t>(n_pad) * kTileRows;
+      if (rg.n[ph] > 0) {
+        // 1/rms of this phase's rows as soon as the previous phase is done
+        // (overlapping this phase's weight stream)
+        if (ph > 0) {
+          if (tid == 0) {
+            uint32_t i = 0;
+            while (ld_acquire_gpu(a.phase_done + ph - 1) < a.p[ph - 1].n_tiles) {
+              if (++i > kChainPollLimit) {
+                flag_status(status, DVI_DEV_TIMEOUT);
+                break;
+              }
+              if (i > 16) __nanosleep(64);
+            }
+          }
+          named_bar(1, kTileRows);
+          ld_acquire_gpu(a.phase_done + ph - 1);
+        }
+        compute_rstd(p, rstd, posn, tid, kTileRows);
+        named_bar(1, kTileRows);
+      }
+      auto finish_tile = [&]() {
+        __threadfence();
+        fence_proxy_async_global();
+        named_bar(1, kTileRows);
+        if (tid == 0) red_release_gpu_add(a.phase_done + ph, 1);
+      };
+      long long k = rg.k0[ph];
+      const long long kend = k + rg.n[ph];
+      while (k < kend) {
+        const int tile = static_cast<int>(k / p.kb_total);
+        const long long tend = min(kend, static_cast<long long>(tile + 1) * p.kb_total);
+        const bool whole = tend - k == p.kb_total;
+        const int b = seg & 1;
+        ok = mbar_wait(&accf[b], (seg >> 1) & 1, status);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t lane_base = tmem + ((static_cast<uint32_t>(warp) * 32u) << 16) + static_cast<uint32_t>(b) * bufcols;
+        float v[kChunk], vl[kChunk];
+        if (whole) {
+          for (int c = 0; c < nchunks; ++c) {
+            tmem_ld16(lane_base + c * kChunk, v);
+            tmem_ld16(lane_base + n_pad + c * kChunk, vl);
+#pragma unroll
+            for (int j = 0; j < kChunk; ++j) v[j] += vl[j];
+            epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, valid_cols(p, c * kChunk));
+          }
+          tc_fence_before();
+          named_bar(1, kTileRows);
+          if (tid == 0) mbar_arrive(&acce[b]);
+          finish_tile();
+        } else {
+          const long long t0 = static_cast<long long>(tile) * p.kb_total;
+          const int first = chain_owner(t0, all, a.n_ctas);
+          const int last = chain_owner(t0 + p.kb_total - 1, all, a.n_ctas);
+          int* ctr = a.tile_ctr + ph * kChainTiles + tile;
+          if (cta != first) {
+            // contributor: partial into the slot, then a release increment
+            // of the tile's counter; nothing to wait for
+            float* mine = a.part + (static_cast<size_t>(tile) + cta) * slot;
+            for (int c = 0; c < nchunks; ++c) {
+              tmem_ld16(lane_base + c * kChunk, v);
+              tmem_ld16(lane_base + n_pad + c * kChunk, vl);
+#pragma unroll
+              for (int j = 0; j < kChunk; ++j)
+                if (c * kChunk + j < p.M) __stcg(mine + (c * kChunk + j) * kTileRows + tid, v[j] + vl[j]);
+            }
+            tc_fence_before();
+            __threadfence();
+            named_bar(1, kTileRows);
+            if (tid == 0) {
+              mbar_arrive(&acce[b]);
+              red_release_gpu_add(ctr, 1);
+            }
+          } else {
+            // finisher (the CTA holding the tile's first K block, whose last
+            // segment of the phase this is): wait for the other contributors,
+            // then sum its own accumulator and their partials in K order
+            if (tid == 0) {
+              uint32_t i = 0;
+              while (ld_acquire_gpu(ctr) < last - first) {
+                if (++i > kChainPollLimit) {
+                  flag_status(status, DVI_DEV_TIMEOUT);
+                  break;
+                }
+                if (i > 16) __nanosleep(32);
+              }
+            }
+            named_bar(1, kTileRows);
+            const float* src = a.part + (static_cast<size_t>(tile) + first) * slot + tid;
+            const int nc = last - first + 1;
+            for (int c = 0; c < nchunks; ++c) {
+              const uint32_t own = valid_cols(p, c * kChunk);
+              const float* col = src + static_cast<size_t>(c) * kChunk * kTileRows;
+              tmem_ld16(lane_base + c * kChunk, v);
+              tmem_ld16(lane_base + n_pad + c * kChunk, vl);
+#pragma unroll
+              for (int j = 0; j < kChunk; ++j) v[j] += vl[j];
+              // the other contributors' partials: four contributors' loads of
+              // all 16 columns in flight at a time (columns past M are in
+              // the slot and ignored)
+              int cc = 1;
+              for (; cc + 4 <= nc; cc += 4) {
+                float t[4][kChunk];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                  for (int j = 0; j < kChunk; ++j) t[u][j] = __ldcg(col + (cc + u) * slot + j * kTileRows);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                  for (int j = 0; j < kChunk; ++j) v[j] += t[u][j];
+              }
+              for (; cc < nc; ++cc) {
+                float t[kChunk];
+#pragma unroll
+                for (int j = 0; j < kChunk; ++j) t[j] = __ldcg(col + cc * slot + j * kTileRows);
+#pragma unroll
+                for (int j = 0; j < kChunk; ++j) v[j] += t[j];
+              }
+#pragma unroll
+              for (int j = 0; j < kChunk; ++j) v[j] = ((own >> j) & 1u) ? v[j] : 0.f;
+              epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, own);
+            }
+            tc_fence_before();
+            named_bar(1, kTileRows);
+            if (tid == 0) {
+              mbar_arrive(&acce[b]);
+              *ctr = 0;
+            }
+            finish_tile();
+          }
+        }
+        ++seg;
+        k = tend;
+      }
+    }
+  }
+  // ---------------- teardown; the last CTA to leave resets the phase counters
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * bufcols);
+  }
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(a.exit_ctr, 1) == a.n_ctas - 1) {
+      for (int ph = 0; ph < kChainMax; ++ph) a.phase_done[ph] = 0;
+      *a.exit_ctr = 0;
+      __threadfence();
+    }
+  }
+}
+
 // ------------------------------------------------------------------ FP32 FMA
 __global__ void __launch_bounds__(128) proj_f32_kernel(const ProjArgs p) {
   __shared__ float Ws[kTileRows][kKBlockF32 + 1];
@@ -735,6 +1176,72 @@ cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s
     b.n_ttiles = (a0.M + kChunk - 1) / kChunk;
     e = launch_pdl(proj_f32_kernel, dim3(a0.n_tiles * a0.n_splits, b.n_ttiles), dim3(128), 0, s, b);
   }
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Chain kernel: ring depth for two CTAs per SM at n_pad.
+static int chain_stages(int n_pad, size_t* smem_bytes) {
+  const int per = 16384 + 2 * n_pad * 128;
+  const int fixed = 1024 /*align*/ + 16 * 8 + 16 /*barriers, tmem slot*/ + 8 * kMaxTokens /*rstd, positions*/ +
+                    static_cast<int>(sizeof(EpiSmem));
+  const int budget = 113 * 1024;   // two CTAs per SM
+  int stages = std::max(2, std::min(6, (budget - fixed) / per));
+  *smem_bytes = static_cast<size_t>(fixed) + static_cast<size_t>(stages) * per;
+  return stages;
+}
+
+static void chain_attr() {
+  static bool done = false;
+  if (!done) {
+    cudaFuncSetAttribute(proj_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    cudaFuncSetAttribute(proj_chain_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                         cudaSharedmemCarveoutMaxShared);
+    done = true;
+  }
+}
+
+int chain_ctas_per_sm(int n_pad) {
+  if (n_pad < 16 || n_pad > kChainMaxPad || n_pad % 16) return 0;
+  chain_attr();
+  size_t smem = 0;
+  chain_stages(n_pad, &smem);
+  // from the device limits: shared memory (with the per-block reservation)
+  // and registers (allocated per warp in units of 256)
+  int dev = 0, smem_sm = 0, reserved = 0, regs_sm = 0;
+  cudaFuncAttributes fa{};
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaFuncGetAttributes(&fa, proj_chain_kernel) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  const size_t per_cta = smem + fa.sharedSizeBytes + static_cast<size_t>(reserved);
+  const int by_smem = static_cast<int>(static_cast<size_t>(smem_sm) / per_cta);
+  const int regs_warp = (fa.numRegs * 32 + 255) / 256 * 256;
+  const int by_regs = regs_sm / (regs_warp * 6);
+  return std::max(0, std::min(2, std::min(by_smem, by_regs)));
+}
+
+size_t chain_partial_floats(int max_tiles, int n_ctas, int n_pad) {
+  return static_cast<size_t>(max_tiles + n_ctas) * n_pad * kTileRows;
+}
+
+cudaError_t launch_chain(const ChainArgs& a, cudaStream_t s) {
+  chain_attr();
+  size_t smem = 0;
+  const int stages = chain_stages(a.p[0].n_pad, &smem);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.n_ctas);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, proj_chain_kernel, a, stages);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
