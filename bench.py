@@ -72,20 +72,22 @@ def step_bytes(w, n_ctx):
     return draft, verify
 
 
-def measured_traffic(w, n_attended):
+def measured_traffic(w, n_attended, persistent=False):
     """Per-launch DRAM traffic of the verify pass from the committed ncu summary.
 
-    The summary holds the bytes ncu counted per deep layer's projections, the
-    LM head, and one deep layer's attention at a given number of 64-position
-    chunks; the pass's traffic is scaled to this workload's layer count and
-    context.  Returns None when no capture matches the workload.
+    The summary holds the bytes ncu counted per deep layer's projections (or,
+    for the persistent chain, per chain launch), the LM head, and one deep
+    layer's attention at a given number of 64-position chunks; the pass's
+    traffic is scaled to this workload's layer count and context.  Returns
+    None when no capture matches the workload.
     """
     p = os.path.join(ROOT, "profiles", "verify_pass_dram_7b_width.md")
     if not os.path.exists(p):
         return None
     m = None
+    key = "traffic-model-persistent:" if persistent else "traffic-model:"
     for ln in open(p):
-        if ln.startswith("traffic-model:"):
+        if ln.startswith(key):
             m = json.loads(ln.split(":", 1)[1])
     s = w.shape
     if m is None or (m["d_model"], m["n_heads"], m["d_ffn"], m["vocab"]) != (s.d_model, s.n_heads, s.d_ffn,
@@ -94,8 +96,11 @@ def measured_traffic(w, n_attended):
         return None
     deep = w.shape.n_layers - w.split_k
     chunks = float(np.mean([-(-int(round(n + w.k_spec)) // 64) * 64 for n in n_attended]))
-    return deep * (m["proj_bytes_per_deep_layer"] + m["attn_bytes_per_deep_layer"] * chunks
-                   / m["attn_chunk_positions"]) + m["head_bytes"]
+    attn = deep * m["attn_bytes_per_deep_layer"] * chunks / m["attn_chunk_positions"]
+    if persistent:
+        return (m["qkv_first_bytes"] + (deep - 1) * m["chain_bytes_per_deep_layer"] + m["chain_last_bytes"]
+                + m["head_bytes"] + attn)
+    return deep * m["proj_bytes_per_deep_layer"] + attn + m["head_bytes"]
 
 
 # ---------------------------------------------------------------- clocks
@@ -315,8 +320,7 @@ def main():
     u_ms = phases["update"][0] / max(1, phases["update"][1])
     hbm = pk["hbm_gbs"]
     v_gbs = verify_b / (v_ms / 1e3) / 1e9
-    # the ncu counters were taken on the per-kernel path
-    v_traffic = None if args.persistent else measured_traffic(w, n_mid)
+    v_traffic = measured_traffic(w, n_mid, args.persistent)
     d_gbs = draft_b / (d_ms / 1e3) / 1e9
 
     e2e = None
