@@ -72,6 +72,20 @@ def step_bytes(w, n_ctx):
     return draft, verify
 
 
+def prefill_bytes(w, n, chunk):
+    """Algorithmic HBM bytes of prefilling one n-token prompt in chunks of
+    `chunk` rows: every chunk streams all L layers' weights once, reads the
+    K/V rows of its prefix (its own included) once per layer and writes its
+    own; the LM head runs on the last row only."""
+    s, esz = w.shape, (2 if w.dtype == "bf16" else 4)
+    lb, kvb = layer_bytes(s, esz), kv_row_bytes(s, esz)
+    total = s.vocab * s.d_model * esz
+    for c0 in range(0, n, chunk):
+        rows = min(chunk, n - c0)
+        total += s.n_layers * (lb + (c0 + rows) * kvb + rows * kvb)
+    return total
+
+
 def measured_traffic(w, n_attended, persistent=False):
     """Per-launch DRAM traffic of the verify pass from the committed ncu summary.
 
@@ -269,8 +283,20 @@ def main():
                     lora_gamma=w.lora_gamma, max_seq_len=max_len, log_steps=U, device=local,
                     persistent=args.persistent)
     hyper = update_config(w.update)
-    for b, p in enumerate(P):
-        eng.prefill(b, torch.from_numpy(p).to(dev))
+    # prefill: sequence 0's prompt once to warm up, then every prompt timed
+    # with CUDA events on the engine's stream (prompts already on the device)
+    dP = [torch.from_numpy(p).to(dev) for p in P]
+    eng.prefill(0, dP[0])
+    pf0, pf1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    pf0.record(eng.stream)
+    for b, p in enumerate(dP):
+        eng.prefill(b, p)
+    pf1.record(eng.stream)
+    torch.cuda.synchronize(dev)
+    pf_ms = pf0.elapsed_time(pf1)
+    pf_tokens = sum(len(p) for p in P)
+    pf_bytes = sum(prefill_bytes(w, len(p), eng.rt.max_prefill_chunk or 128) for p in P)
     eng.log(True)
 
     def one_step():
@@ -356,6 +382,11 @@ def main():
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "projections": "persistent chain" if args.persistent else "one kernel each"},
         "mean_accepted_length": mat,
+        "prefill": {"tokens": pf_tokens, "ms": pf_ms, "tokens_per_s": pf_tokens / (pf_ms / 1e3),
+                    "chunk": eng.rt.max_prefill_chunk or 128,
+                    "roofline": {"bound": "hbm", "achieved": pf_bytes / (pf_ms / 1e3) / 1e9, "peak": hbm,
+                                 "unit": "GB/s", "frac": pf_bytes / (pf_ms / 1e3) / 1e9 / hbm,
+                                 "bytes": pf_bytes}},
         "roofline": {"bound": "hbm", "achieved": v_gbs, "peak": hbm, "unit": "GB/s", "frac": v_gbs / hbm,
                      "traffic": v_traffic, "kernel": "verify pass (layers k+1..L + LM head, CUDA-graph replay)",
                      "traffic_source": "profiles/verify_pass_dram_7b_width.md (ncu, 4-layer case scaled)"

@@ -350,8 +350,10 @@ __global__ void __launch_bounds__(192, 2)
   float* rstd = reinterpret_cast<float*>(tmem_holder + 4);
   int* posn = reinterpret_cast<int*>(rstd + kMaxTokens);
 
-  // after `done` the A stages are free: epilogue scratch, then this split's
-  // partial tile [n_pad][128] for the cluster reduction
+  // after `done` every stage is free: epilogue scratch in the first A
+  // stage, then this split's partial tile [n_pad][128] (n_pad * 512 bytes,
+  // which the remaining A stages and the B stages always hold: at least two
+  // stages of 16 KB + n_pad * 256 bytes)
   EpiSmem& es = *reinterpret_cast<EpiSmem*>(sA);
   float* part = reinterpret_cast<float*>(sA + abytes);
 
@@ -1147,11 +1149,6 @@ cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s
       attr = true;
     }
     ProjArgs a = a0;
-    // the cluster reduction keeps a [n_pad][128] partial in the A stages
-    if (a.n_pad > 64 && a.n_splits > 1) {
-      a.n_splits = 1;
-      a.kb_per_split = a.kb_total;
-    }
     size_t smem = 0;
     const int stages = tc_stages(a.n_pad, &smem);
     cudaLaunchConfig_t cfg = {};
