@@ -22,9 +22,6 @@ constexpr int kChunk = 16;           // token columns per epilogue chunk
 constexpr int kMaxTokens = 256;      // rows of one projection launch (tcgen05 N <= 256)
 constexpr int kAttnQ = 16;           // query vectors per attention CTA
 constexpr int kAttnBlk = 64;         // KV positions per attention sub-block
-// A bounded wait gives up after this many polls (each sleeps ~0.2 us), i.e.
-// after roughly a second, sets DVI_DEV_TIMEOUT and lets the kernel exit.
-constexpr uint32_t kSpinLimit = 1u << 22;
 
 // ---------------------------------------------------------------- dtype
 template <typename T> struct DT;
@@ -156,13 +153,36 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return done != 0;
 }
-// Bounded wait for the phase with the given parity to complete: polls with a
-// short sleep, and after kSpinLimit polls (about a second) flags
-// DVI_DEV_TIMEOUT and returns false so the caller can wind down.
+// Potentially blocking test: the thread may be suspended until the phase
+// completes or a hardware time limit passes, and resumes as soon as the
+// phase completes.
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+constexpr uint64_t kWaitLimitNs = 1000000000ull;   // a bounded wait gives up after one second
+// Bounded wait for the phase with the given parity to complete: hardware
+// try_wait (no sleep quantum between polls), and after kWaitLimitNs of
+// global time flags DVI_DEV_TIMEOUT and returns false so the caller can
+// wind down.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_test_wait(bar, parity)) return true;
-    if (i >= 32) __nanosleep(200);
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > kWaitLimitNs) break;
   }
   flag_status(status, DVI_DEV_TIMEOUT);
   return false;
