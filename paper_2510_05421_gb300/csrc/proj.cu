@@ -543,22 +543,25 @@ __global__ void __launch_bounds__(192, 2)
         for (int j = 0; j < kChunk; ++j)
           if (c * kChunk + j < p.M && (c * kChunk + j) % S == split) own |= 1u << j;
         if (!own) continue;
+        // one compact loop over the owned columns: the sum of every rank's
+        // partial (in rank order) replaces this rank's own partial, which
+        // only this rank reads for the columns it owns
+#pragma unroll 1
+        for (int j = 0; j < kChunk; ++j) {
+          if (!((own >> j) & 1u)) continue;
+          const uint32_t off = static_cast<uint32_t>((c * kChunk + j) * kTileRows) * 4u;
+          float t[8];
+#pragma unroll
+          for (int r = 0; r < 8; ++r) t[r] = r < S ? ld_cluster_f32(peer[r] + off) : 0.f;
+          float acc = t[0];
+#pragma unroll
+          for (int r = 1; r < 8; ++r)
+            if (r < S) acc += t[r];
+          part[(c * kChunk + j) * kTileRows + tid] = acc;
+        }
         float v[kChunk];
 #pragma unroll
-        for (int j = 0; j < kChunk; ++j) {
-          v[j] = 0.f;
-          if ((own >> j) & 1u) {
-            const uint32_t off = static_cast<uint32_t>((c * kChunk + j) * kTileRows) * 4u;
-            float t[8];
-#pragma unroll
-            for (int r = 0; r < 8; ++r) t[r] = r < S ? ld_cluster_f32(peer[r] + off) : 0.f;
-            float acc = t[0];
-#pragma unroll
-            for (int r = 1; r < 8; ++r)
-              if (r < S) acc += t[r];
-            v[j] = acc;
-          }
-        }
+        for (int j = 0; j < kChunk; ++j) v[j] = ((own >> j) & 1u) ? part[(c * kChunk + j) * kTileRows + tid] : 0.f;
         epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, own);
       }
     }
