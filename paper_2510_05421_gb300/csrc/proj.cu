@@ -128,11 +128,13 @@ __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int 
       named_bar(1, kTileRows);
     }
     const int prow = row + (dim < half ? half : -half);
+    // sequence of column c0 + j, advanced column by column (no division in
+    // the unrolled loop)
+    int seq = p.seq0 + c0 / p.rows_per_seq, in_seq = c0 % p.rows_per_seq;
 #pragma unroll
-    for (int j = 0; j < kChunk; ++j) {
+    for (int j = 0; j < kChunk; ++j, seq += (++in_seq == p.rows_per_seq), in_seq = in_seq == p.rows_per_seq ? 0 : in_seq) {
       const int n = c0 + j;
       if ((own >> j) & 1u) {
-        const int seq = p.seq0 + n / p.rows_per_seq;
         const int pos = posn[n];
         if (pos >= p.max_len || pos < 0) {
           flag_status(p.status, DVI_DEV_KV_FULL);
@@ -538,10 +540,10 @@ __global__ void __launch_bounds__(192, 2)
       for (int r = 0; r < 8; ++r) peer[r] = r < S ? mapa_shared(mine, r) : 0u;
       const int nchunks = (p.M + kChunk - 1) / kChunk;
       for (int c = 0; c < nchunks; ++c) {
+        // columns n of [c0, c0 + 16) with n = split (mod S)
+        const int c0 = c * kChunk, c1 = min(p.M, c0 + kChunk);
         uint32_t own = 0;
-#pragma unroll
-        for (int j = 0; j < kChunk; ++j)
-          if (c * kChunk + j < p.M && (c * kChunk + j) % S == split) own |= 1u << j;
+        for (int n = c0 + (split - c0 % S + S) % S; n < c1; n += S) own |= 1u << (n - c0);
         if (!own) continue;
         // one compact loop over the owned columns: the sum of every rank's
         // partial (in rank order) replaces this rank's own partial, which
