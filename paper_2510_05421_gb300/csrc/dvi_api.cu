@@ -674,8 +674,10 @@ StepState step_state(dvi_ctx* c) {
 
 // Head projection over `rows` activation rows xg (x * final_norm) starting
 // at row `row0` of `act`; 1/rms from `ss`.  W^S (+ LoRA) when `draft`.
+// With `bu_inline` (bf16 drafter head) the kernel computes B u itself from
+// the draft residual rows instead of reading it from `bu`.
 dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, const void* act,
-                        const CUtensorMap* act_map, int row0, const float* ss, int ss_ld) {
+                        const CUtensorMap* act_map, int row0, const float* ss, int ss_ld, bool bu_inline = false) {
   Pass ps{nullptr, nullptr, 0, rows, 1, 0, 1, 0, nullptr, nullptr};
   ProjArgs a = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
   a.act = act;
@@ -692,6 +694,12 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
     a.lora_bu = ctx->bu;
     a.lora_r = ctx->r;
     a.gamma = ctx->cfg.lora_gamma;
+    if (bu_inline) {
+      a.lora_bmat = ctx->w.lora_b;
+      a.bu_x = ctx->x_dr;
+      a.bu_ldx = ctx->d;
+      a.bu_g = static_cast<const float*>(ctx->w.final_norm);
+    }
   }
   if (logits_mode == 2) {
     a.logits_mode = 2;
@@ -708,6 +716,12 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
   DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &pm : nullptr, ctx->stream));
   ctx->launches += 1;
   return DVI_OK;
+}
+
+// The drafter head can compute B u in-kernel: bf16, a LoRA term of rank
+// <= kBuRank, at most kBuRows sequences, and a d the float4 loop covers.
+bool bu_inline_ok(const dvi_ctx* ctx) {
+  return ctx->tc && ctx->r > 0 && ctx->r <= kBuRank && ctx->B <= kBuRows && ctx->d % 128 == 0;
 }
 
 dvi_status enqueue_draft(dvi_ctx* ctx) {
@@ -746,17 +760,23 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
     h.log_row_stride = ctx->K;
     h.log_row_off = j;
     h.log_enabled = drafts ? ctx->log_enabled : 0;
-    if (ctx->r > 0 && drafts) {
+    // bf16: the head computes B u while its weights stream, and the logged u
+    // and the hand-off run in the finalize kernel after it (one launch less)
+    const bool fused = drafts && bu_inline_ok(ctx);
+    if (ctx->r > 0 && drafts && !fused) {
       h.lora_b = ctx->w.lora_b;
       h.bu = ctx->bu;
       h.r = ctx->r;
     }
-    DVI_CUDA(launch_head_prep(h, s));
-    ctx->launches += 1;
+    if (!fused) {
+      DVI_CUDA(launch_head_prep(h, s));
+      ctx->launches += 1;
+    }
     if (!drafts) continue;
-    if ((rc = enqueue_head(ctx, true, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
+    if ((rc = enqueue_head(ctx, true, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B, fused)) !=
+        DVI_OK)
       return rc;
-    DVI_CUDA(launch_finalize_draft(st, j, s));
+    DVI_CUDA(launch_finalize_draft(st, j, fused ? &h : nullptr, s));
     ctx->launches += 1;
   }
   return DVI_OK;

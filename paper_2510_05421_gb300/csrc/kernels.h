@@ -22,6 +22,9 @@ enum BMode : int {
   B_SOFT_F32 = 1   // bf16 path: float32 rows converted by warps 0-3 (dvi_linear)
 };
 
+constexpr int kBuRows = 16;   // rows of an in-kernel B u (the drafter head's batch)
+constexpr int kBuRank = 16;   // LoRA rank of an in-kernel B u
+
 struct ProjArgs {
   int flavor, b_mode, dtype;
   int M;              // token rows
@@ -65,6 +68,10 @@ struct ProjArgs {
   const int* log_step; int log_cap_steps; int log_rows_per_step;
   int log_src_rows, log_dst_rows;   // mode 2: launch rows per sequence, of which the log keeps the first
   const float* lora_a; const float* lora_bu; int lora_r; float gamma;
+  // bf16 drafter head, M <= kBuRows and lora_r <= kBuRank: B u computed by
+  // the kernel itself (lora_bu unused), u = (x * rstd) * g from the f32
+  // residual rows bu_x and the final-norm gain bu_g
+  const float* lora_bmat; const float* bu_x; int bu_ldx; const float* bu_g;
   unsigned long long* amax;   // [M] argmax keys, or null
 };
 
@@ -174,7 +181,9 @@ struct StepState {
   long long* counters;                          // steps, drafted, accepted, committed
   int* status;
 };
-cudaError_t launch_finalize_draft(const StepState& st, int j, cudaStream_t s);
+// `prep` (or null): the pass's drafter-head preparation without B u, run
+// before the next pass's embedding (the head computed B u itself).
+cudaError_t launch_finalize_draft(const StepState& st, int j, const HeadPrepArgs* prep, cudaStream_t s);
 cudaError_t launch_finalize_verify(const StepState& st, cudaStream_t s);
 cudaError_t launch_finalize_ar(const StepState& st, cudaStream_t s);
 cudaError_t launch_finalize_prefill(const StepState& st, int seq, int n_tokens, int32_t* first_out,

@@ -84,14 +84,12 @@ cudaError_t launch_embed(const EmbedArgs& a, cudaStream_t s) {
 // grid (rows, ceil(r/4) or 1); block 128.  Every CTA computes the row's
 // 1/rms; CTA y == 0 logs u and hands the row to the verify stream; each CTA
 // computes four entries of B u (one warp each).
+// One row of the drafter-head preparation (128 threads): x = h_k, its
+// per-tile sums of squares and 1/rms, u = x * rstd * gain into `us` (when
+// non-null), and, when `io` is set, u into the replay buffer and h_k handed
+// to the verify rows (x, x * g_copy and the sums of squares).
 template <typename T>
-__global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
-  __shared__ float red[kMaxTiles * 4];
-  __shared__ float rstd_s;
-  __shared__ __align__(16) float us[kMaxTiles * kTileRows];   // u = x * rstd * gain
-  griddep_launch();
-  griddep_wait();
-  const int row = blockIdx.x, grp = blockIdx.y;
+__device__ void prep_row(const HeadPrepArgs& a, int row, bool io, float* red, float* rstd_s, float* us) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float* x = a.x + static_cast<size_t>(row) * a.ldx;
   const int nt = a.d / kTileRows;
@@ -113,14 +111,16 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
   if (tid == 0) {
     float s = 0.f;
     for (int t = 0; t < nt; ++t) s += (red[t * 4] + red[t * 4 + 1]) + (red[t * 4 + 2] + red[t * 4 + 3]);
-    rstd_s = rsqrtf(s / static_cast<float>(a.d) + a.eps);
+    *rstd_s = rsqrtf(s / static_cast<float>(a.d) + a.eps);
   }
   __syncthreads();
-  const float rstd = rstd_s;
+  const float rstd = *rstd_s;
+  if (us) {
 #pragma unroll
-  for (int t = 0; t < kMaxTiles; ++t)
-    if (t < nt) us[t * kTileRows + tid] = xv[t] * rstd * gv[t];
-  if (grp == 0) {
+    for (int t = 0; t < kMaxTiles; ++t)
+      if (t < nt) us[t * kTileRows + tid] = xv[t] * rstd * gv[t];
+  }
+  if (io) {
     T* lu = nullptr;
     if (a.log_u && a.log_enabled) {
       const int ls = *a.log_step;
@@ -153,6 +153,18 @@ __global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
             (red[t * 4] + red[t * 4 + 1]) + (red[t * 4 + 2] + red[t * 4 + 3]);
     }
   }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(128) head_prep_kernel(const HeadPrepArgs a) {
+  __shared__ float red[kMaxTiles * 4];
+  __shared__ float rstd_s;
+  __shared__ __align__(16) float us[kMaxTiles * kTileRows];   // u = x * rstd * gain
+  griddep_launch();
+  griddep_wait();
+  const int row = blockIdx.x, grp = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  prep_row<T>(a, row, grp == 0, red, &rstd_s, us);
   if (a.r > 0 && a.bu) {
     __syncthreads();
     const int j = grp * 4 + warp;
@@ -203,12 +215,24 @@ __device__ void embed_rows(const StepState& st, const int* toks, float* red) {
                        st.ss_dr_ld, b, red);
 }
 
+// With `prep` set, the drafter-head preparation of the pass (the logged u
+// and the hand-off of h_k to the verify rows; the head computed B u itself)
+// runs here, for every row before its residual is overwritten by the next
+// pass's embedding.
 template <typename T>
-__global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st, int j) {
+__global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st, int j, const HeadPrepArgs hp,
+                                                             int prep) {
   __shared__ int tok_s[64];
   __shared__ float red[kMaxTiles * 4];
+  __shared__ float rstd_s;
   griddep_launch();
   griddep_wait();
+  if (prep) {
+    for (int b = 0; b < hp.rows; ++b) {
+      prep_row<T>(hp, b, true, red, &rstd_s, nullptr);
+      __syncthreads();
+    }
+  }
   for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
     const int t = take_argmax(st.amax + b, st.status);
     st.draft_ids[b * (st.K + 1) + j + 1] = t;
@@ -323,9 +347,12 @@ static cudaError_t launch1(K kern, cudaStream_t s, Args... args) {
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t launch_finalize_draft(const StepState& st, int j, cudaStream_t s) {
-  return st.dtype == DVI_BF16 ? launch1(finalize_draft_kernel<__nv_bfloat16>, s, st, j)
-                              : launch1(finalize_draft_kernel<float>, s, st, j);
+cudaError_t launch_finalize_draft(const StepState& st, int j, const HeadPrepArgs* prep, cudaStream_t s) {
+  HeadPrepArgs hp{};
+  if (prep) hp = *prep;
+  const int on = prep ? 1 : 0;
+  return st.dtype == DVI_BF16 ? launch1(finalize_draft_kernel<__nv_bfloat16>, s, st, j, hp, on)
+                              : launch1(finalize_draft_kernel<float>, s, st, j, hp, on);
 }
 cudaError_t launch_finalize_verify(const StepState& st, cudaStream_t s) {
   return st.dtype == DVI_BF16 ? launch1(finalize_verify_kernel<__nv_bfloat16>, s, st)

@@ -107,7 +107,8 @@ __device__ __forceinline__ uint32_t valid_cols(const ProjArgs& p, int c0) {
 // epilogue threads together (row = feature within tile).
 template <typename T>
 __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int row, int c0, float (&v)[kChunk],
-                               const float* rstd, const int* posn, EpiSmem& es, uint32_t own) {
+                               const float* rstd, const int* posn, EpiSmem& es, uint32_t own,
+                               const float* bu_s = nullptr) {
   const int warp = row >> 5, lane = row & 31;
   if (p.ss) {
 #pragma unroll
@@ -210,7 +211,7 @@ __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int 
       for (int j = 0; j < kChunk; ++j) {
         const int n = c0 + j;
         if ((own >> j) & 1u) {
-          const float* bu = p.lora_bu + static_cast<size_t>(n) * p.lora_r;
+          const float* bu = (p.lora_bmat ? bu_s : p.lora_bu) + static_cast<size_t>(n) * p.lora_r;
           float acc = 0.f;
           for (int q = 0; q < p.lora_r; ++q) acc = fmaf(arow[q], bu[q], acc);
           z[j] = fmaf(p.gamma, acc, z[j]);
@@ -351,6 +352,7 @@ __global__ void __launch_bounds__(192, 2)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(done + 1);
   float* rstd = reinterpret_cast<float*>(tmem_holder + 4);
   int* posn = reinterpret_cast<int*>(rstd + kMaxTokens);
+  float* bu_s = reinterpret_cast<float*>(posn + kMaxTokens);   // [kBuRows][kBuRank] in-kernel B u
 
   // after `done` every stage is free: epilogue scratch in the first A
   // stage, then this split's partial tile [n_pad][128] (n_pad * 512 bytes,
@@ -494,6 +496,31 @@ __global__ void __launch_bounds__(192, 2)
     }
     compute_rstd(p, rstd, posn, tid, kTileRows);
     named_bar(1, kTileRows);
+    if (p.lora_bmat) {
+      // B u of the LoRA term while the weights stream: warp w takes rows
+      // q = w, w + 4, ... of B; u = (x * rstd) * g, four features per lane
+      // per step, summed per lane in feature order then across the warp
+      for (int n = 0; n < p.M; ++n) {
+        const float r = rstd[n];
+        const float4* x4 = reinterpret_cast<const float4*>(p.bu_x + static_cast<size_t>(n) * p.bu_ldx);
+        const float4* g4 = reinterpret_cast<const float4*>(p.bu_g);
+        for (int q = warp; q < p.lora_r; q += 4) {
+          const float4* br = reinterpret_cast<const float4*>(p.lora_bmat + static_cast<size_t>(q) * p.K);
+          float acc = 0.f;
+#pragma unroll 4
+          for (int c = lane; c < p.K / 4; c += 32) {
+            const float4 b = br[c], xx = x4[c], gg = g4[c];
+            acc = fmaf(b.x, xx.x * r * gg.x, acc);
+            acc = fmaf(b.y, xx.y * r * gg.y, acc);
+            acc = fmaf(b.z, xx.z * r * gg.z, acc);
+            acc = fmaf(b.w, xx.w * r * gg.w, acc);
+          }
+          acc = warp_sum(acc);
+          if (lane == 0) bu_s[n * p.lora_r + q] = acc;
+        }
+      }
+      named_bar(1, kTileRows);
+    }
     ok = mbar_wait(done, 0, p.status);
     tc_fence_after();
     const uint32_t lane_base = tmem + ((static_cast<uint32_t>(warp) * 32u) << 16);
@@ -507,7 +534,8 @@ __global__ void __launch_bounds__(192, 2)
 #pragma unroll
         for (int j = 0; j < kChunk; ++j) v[j] += vl[j];
         if (ok)
-          epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, valid_cols(p, c * kChunk));
+          epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, valid_cols(p, c * kChunk),
+                                        bu_s);
       }
     } else {
       for (int c = 0; c < nchunks; ++c) {
@@ -564,7 +592,7 @@ __global__ void __launch_bounds__(192, 2)
         float v[kChunk];
 #pragma unroll
         for (int j = 0; j < kChunk; ++j) v[j] = ((own >> j) & 1u) ? part[(c * kChunk + j) * kTileRows + tid] : 0.f;
-        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, own);
+        epilogue_chunk<__nv_bfloat16>(p, tile, tid, c * kChunk, v, rstd, posn, es, own, bu_s);
       }
     }
     // every rank keeps its shared memory until all have read it
@@ -1137,7 +1165,8 @@ size_t proj_partial_floats(const ProjArgs& a, bool tc) {
 
 static int tc_stages(int n_pad, size_t* smem_bytes) {
   const int per = 16384 + 2 * n_pad * 128;   // weight tile + hi and lo activation rows
-  const int fixed = 1024 /*align*/ + 1024 /*barriers, tmem slot*/ + 8 * kMaxTokens /*rstd, positions*/;
+  const int fixed = 1024 /*align*/ + 1024 /*barriers, tmem slot*/ + 8 * kMaxTokens /*rstd, positions*/ +
+                    4 * kBuRows * kBuRank /*in-kernel B u*/;
   // two CTAs per SM while the ring keeps at least three stages
   int stages = std::max(2, std::min(4, (112 * 1024 - fixed) / per));
   *smem_bytes = static_cast<size_t>(fixed) + static_cast<size_t>(stages) * per;
