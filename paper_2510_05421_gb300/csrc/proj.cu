@@ -22,7 +22,8 @@
 // per-row scalar) multiplies the accumulators in the epilogue.
 // Launches use programmatic dependent launch: the weight tiles of the first
 // stages (which no earlier kernel writes) stream in before the kernel waits
-// for its predecessor.
+// for its predecessor.  The drafter head (bf16, few rows) also forms the
+// LoRA term's B u in its epilogue warps while the weights stream.
 //
 // f32 (FP32 FMA, no TF32): the same decomposition with a shared-memory tiled
 // FFMA main loop of 16 token columns per CTA.
