@@ -117,6 +117,8 @@ typedef struct {
 } dvi_layer_weights;
 
 /* Device pointers, caller-owned, read for the whole life of the context.
+ * final_norm and lora_b must be 16-byte aligned (dvi_create returns
+ * DVI_ERR_INVALID_ARG otherwise), and so must every bf16 weight matrix.
  * draft_head (W^(S)) may alias lm_head (W^(V)) only when head_mode == 0.
  * lora_a / lora_b are updated in place by dvi_update_drafter (head_mode 0);
  * draft_head is updated in place in head_mode 1: with dtype bf16 the

@@ -901,6 +901,11 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
                     "16-byte aligned\n");
     return DVI_ERR_INVALID_ARG;
   }
+  // B_s and the final-norm gain are read four floats at a time
+  if ((cfg->lora_rank > 0 && !aligned16(weights->lora_b)) || !aligned16(weights->final_norm)) {
+    fprintf(stderr, "dvi_create: lora_b and final_norm must be 16-byte aligned\n");
+    return DVI_ERR_INVALID_ARG;
+  }
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return DVI_ERR_INVALID_ARG;
   dvi_ctx* ctx = new dvi_ctx();
   init_dims(ctx, cfg, rt);

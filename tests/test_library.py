@@ -98,3 +98,20 @@ def test_null_context_calls_fail_cleanly(L):
     assert L.dvi_ar_step(None, None) == -1
     assert L.dvi_destroy(None) == -1
     assert L.dvi_last_error(None) == b"null context"
+
+
+@pytest.mark.parametrize("field", ["final_norm", "lora_b"])
+def test_misaligned_vectors_rejected(L, field):
+    """final_norm and lora_b are read four floats at a time: dvi_create
+    refuses pointers that are not 16-byte aligned, before any device work."""
+    cfg, rt = _cfgs(WORKLOADS["tiny"])
+    layers = (D.LayerWeightsC * cfg.n_layers)(*[D.LayerWeightsC(*[0x10000] * 9) for _ in range(cfg.n_layers)])
+    ptrs = dict(embed=0x20000, final_norm=0x30000, lm_head=0x40000, draft_head=0x40000, lora_a=0x50000,
+                lora_b=0x60000)
+    ptrs[field] += 4
+    w = D.WeightsC(ptrs["embed"], layers, ptrs["final_norm"], ptrs["lm_head"], ptrs["draft_head"], ptrs["lora_a"],
+                   ptrs["lora_b"])
+    ctx = ctypes.c_void_p()
+    rc = L.dvi_create(ctypes.byref(cfg), ctypes.byref(rt), ctypes.byref(w), ctypes.c_void_p(1 << 20), 1 << 30,
+                      None, ctypes.byref(ctx))
+    assert rc == -1 and not ctx.value
