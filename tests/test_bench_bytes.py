@@ -74,3 +74,20 @@ def test_committed_ncu_traffic_is_the_algorithmic_bytes():
     assert tp is not None and 1.0 <= tp / verify < 1.04
     # another shape has no capture
     assert bench.measured_traffic(workload("1b"), n) is None
+
+
+def test_prefill_flops_and_bound():
+    w = workload("7b")
+    # 2 FLOPs per weight per token over 32 layers of 202,375,168 weights,
+    # causal attention's two products (32 heads x 128, 1024 x 1025 / 2
+    # attended pairs per layer), the LM head on one row
+    expect = 32 * (2 * 202_375_168 * 1024 + 4 * 32 * 128 * (1024 * 1025 // 2)) + 2 * 32000 * 4096
+    assert bench.prefill_flops(w, 1024) == expect
+    assert expect == pytest.approx(13.54e12, rel=1e-3)
+    pk = {"hbm_gbs": 6785.5, "bf16_tflops": 1884.7}
+    # 128-row passes stream the weights 8 times: the bytes bound the time
+    r = bench.prefill_roofline(bench.prefill_bytes(w, 1024, 128), expect, 72.0, pk)
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s"
+    # one 1024-row pass: the tensor pipe bounds it
+    r = bench.prefill_roofline(bench.prefill_bytes(w, 1024, 1024), expect, 10.0, pk)
+    assert r["bound"] == "tensor" and r["achieved"] == pytest.approx(expect / 1e-2 / 1e12)
