@@ -231,7 +231,8 @@ class DVIEngine:
 
     def prefill(self, seq: int, tokens: torch.Tensor) -> torch.Tensor:
         """Run a device int32 prompt; returns the device tensor of first tokens [B]."""
-        assert tokens.dtype == torch.int32 and tokens.is_cuda and tokens.is_contiguous()
+        if not (tokens.dtype == torch.int32 and tokens.is_cuda and tokens.is_contiguous()):
+            raise ValueError("prefill: tokens must be a contiguous int32 CUDA tensor")
         self.stream.wait_stream(torch.cuda.current_stream(self.device))
         rc = lib().dvi_prefill(self.ctx, seq, _ptr(tokens), tokens.numel(),
                                ctypes.c_void_p(self.first.data_ptr() + 4 * seq))
@@ -240,7 +241,8 @@ class DVIEngine:
         return self.first
 
     def step(self):
-        """One draft -> verify -> commit step; device tensors (ids [B,K(+1)], n_committed [B], m [B])."""
+        """One draft -> verify -> commit step; device tensors (ids [B,K(+1)], n_committed [B], m [B])
+        written on the engine's stream (wait on `self.stream` before reading them elsewhere)."""
         rc = lib().dvi_draft_verify_commit(self.ctx, _ptr(self.out_ids), _ptr(self.n_committed),
                                            _ptr(self.n_accepted))
         self._check(rc, "dvi_draft_verify_commit")
