@@ -85,10 +85,11 @@ def prefill_flops(w, n):
 
 
 def prefill_bytes(w, n, chunk):
-    """Algorithmic HBM bytes of prefilling one n-token prompt in chunks of
-    `chunk` rows: every chunk streams all L layers' weights once, reads the
-    K/V rows of its prefix (its own included) once per layer and writes its
-    own; the LM head runs on the last row only."""
+    """HBM bytes of prefilling one n-token prompt in passes of `chunk` rows,
+    as this library runs it: every pass streams all L layers' weights once,
+    reads the K/V rows of its prefix (its own included) once per layer and
+    writes its own; the LM head runs on the last row only.  With chunk = n
+    (one pass over the whole prompt) this is the algorithm's own minimum."""
     s, esz = w.shape, (2 if w.dtype == "bf16" else 4)
     lb, kvb = layer_bytes(s, esz), kv_row_bytes(s, esz)
     total = s.vocab * s.d_model * esz
@@ -96,6 +97,12 @@ def prefill_bytes(w, n, chunk):
         rows = min(chunk, n - c0)
         total += s.n_layers * (lb + (c0 + rows) * kvb + rows * kvb)
     return total
+
+
+def prefill_alg_bytes(w, n):
+    """Algorithmic HBM bytes of an n-token prefill: every weight once, every
+    K/V row written once and read once."""
+    return prefill_bytes(w, n, n)
 
 
 def measured_traffic(w, n_attended, persistent=False):
@@ -129,18 +136,23 @@ def measured_traffic(w, n_attended, persistent=False):
     return deep * m["proj_bytes_per_deep_layer"] + attn + m["head_bytes"]
 
 
-def prefill_roofline(nbytes, flops, ms, pk):
-    """The prefill against whichever roofline bounds it: HBM bytes over the
-    copy bandwidth, or FLOPs over the burst bf16 tensor throughput."""
-    t_hbm = nbytes / (pk["hbm_gbs"] * 1e9)
+def prefill_roofline(flops, alg_bytes, ms, pk, traffic=None):
+    """The prefill against the roofline that bounds the algorithm: its FLOPs
+    over the burst bf16 tensor throughput, or its algorithmic bytes over the
+    copy bandwidth, whichever takes longer at peak.  `traffic` (the bytes the
+    implementation moves, weights re-read per pass included) is reported
+    beside it, not used for the fraction."""
+    t_hbm = alg_bytes / (pk["hbm_gbs"] * 1e9)
     t_tc = flops / (pk["bf16_tflops"] * 1e12)
-    if t_tc > t_hbm:
+    if t_tc >= t_hbm:
         ach = flops / (ms / 1e3) / 1e12
-        return {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": ach / pk["bf16_tflops"], "flops": flops, "bytes": nbytes}
-    ach = nbytes / (ms / 1e3) / 1e9
-    return {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": ach / pk["hbm_gbs"],
-            "flops": flops, "bytes": nbytes}
+        r = {"bound": "tensor", "achieved": ach, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+             "frac": ach / pk["bf16_tflops"]}
+    else:
+        ach = alg_bytes / (ms / 1e3) / 1e9
+        r = {"bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": ach / pk["hbm_gbs"]}
+    r.update({"flops": flops, "alg_bytes": alg_bytes, "traffic_model": traffic})
+    return r
 
 
 # ---------------------------------------------------------------- clocks
@@ -187,40 +199,72 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- CPU oracle
-def oracle_sample(w, W, budget_s, prompt_len=64, steps_cap=None, threads=None):
-    """Time the CPU oracle's DVI steps (float32) on a bounded sample.
+class OracleRun:
+    """The CPU oracle (numpy float32) on the workload's first prompt, at the
+    workload's own context: the whole prompt is prefilled once (untimed),
+    then DVI steps (with the drafter update every `update_every` steps) and
+    greedy AR steps are timed on the host cores in bounded samples."""
 
-    Prefill of a truncated prompt is untimed; then DVI steps with an update
-    every `update_every` steps run until `budget_s` of wall time has passed.
-    """
-    from oracle import OracleModel, DrafterUpdater
-    from oracle.decode import prefill, dvi_step
-    m = OracleModel(W, w.shape, w.lora_gamma, dtype=np.float32)
-    upd = DrafterUpdater(m, w.update)
-    P = make_prompts(w)[0][:prompt_len]
-    cache = m.new_cache(prompt_len + 4096)
-    tok, _ = prefill(m, cache, P)
-    n, committed, steps, buf = len(P), 0, 0, []
-    t0 = time.perf_counter()
-    while True:
-        fields, tuples, n, tok = dvi_step(m, cache, n, tok, w.split_k, w.k_spec)
-        committed += len(fields[3])
-        buf.extend(tuples)
-        steps += 1
-        if steps % w.update_every == 0:
-            upd.update(buf)
-            buf = []
-            if time.perf_counter() - t0 >= budget_s or (steps_cap and steps >= steps_cap):
-                break
-    dt = time.perf_counter() - t0
-    return dict(committed=committed, steps=steps, seconds=dt, prompt=len(P))
+    def __init__(self, w, W, room=1024):
+        from oracle import OracleModel, DrafterUpdater
+        from oracle.decode import prefill
+        self.w = w
+        self.m = OracleModel(W, w.shape, w.lora_gamma, dtype=np.float32)
+        self.upd = DrafterUpdater(self.m, w.update)
+        P = make_prompts(w)[0]
+        self.prompt = len(P)
+        self.cache = self.m.new_cache(len(P) + room)
+        t0 = time.perf_counter()
+        self.tok, _ = prefill(self.m, self.cache, P)
+        self.prefill_s = time.perf_counter() - t0
+        self.n, self.buf, self.steps = len(P), [], 0
+
+    def room(self, rows):
+        return self.n + rows + 1 <= self.cache.max_len
+
+    def dvi(self, budget_s, steps_cap=None):
+        """DVI steps until `budget_s` has passed at an update boundary (or the
+        cache is full): (tokens committed, steps, seconds)."""
+        from oracle.decode import dvi_step
+        w, committed, steps = self.w, 0, 0
+        t0 = time.perf_counter()
+        while self.room(w.k_spec):
+            fields, tuples, self.n, self.tok = dvi_step(self.m, self.cache, self.n, self.tok, w.split_k, w.k_spec)
+            committed += len(fields[3])
+            self.buf.extend(tuples)
+            steps += 1
+            self.steps += 1
+            if self.steps % w.update_every == 0:
+                self.upd.update(self.buf)
+                self.buf = []
+                if time.perf_counter() - t0 >= budget_s or (steps_cap and steps >= steps_cap):
+                    break
+        return committed, steps, time.perf_counter() - t0
+
+    def ar(self, budget_s):
+        """Greedy AR steps of the full model until `budget_s` has passed:
+        (tokens, seconds)."""
+        from oracle.decode import ar_step
+        n_tok = 0
+        t0 = time.perf_counter()
+        while self.room(1) and (n_tok == 0 or time.perf_counter() - t0 < budget_s):
+            self.tok, _ = ar_step(self.m, self.cache, self.n, self.tok)
+            self.n += 1
+            n_tok += 1
+        return n_tok, time.perf_counter() - t0
 
 
-def cpu_baseline_dict(res, w, cores):
-    return {"value": res["committed"] / res["seconds"], "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": (f"{w.shape.n_layers}-layer d{w.shape.d_model} decoder in numpy float32, prompt truncated "
-                       f"to {res['prompt']} tokens (prefill untimed), {res['steps']} DVI steps with an update "
-                       f"every {w.update_every}, {res['seconds']:.1f} s")}
+def cpu_baseline_dict(run, dvi, ar, cores):
+    c, st, sec = dvi
+    ntok, asec = ar
+    w = run.w
+    v, v_ar = c / sec, ntok / asec
+    return {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "ar_tokens_per_s": v_ar, "dvi_over_ar": v / v_ar,
+            "sample": (f"{w.shape.n_layers}-layer d{w.shape.d_model} decoder in numpy float32 on the "
+                       f"{run.prompt}-token prompt (prefill untimed, {run.prefill_s:.0f} s), {st} DVI steps "
+                       f"with an update every {w.update_every} in {sec:.1f} s, then {ntok} greedy AR steps "
+                       f"in {asec:.1f} s")}
 
 
 # ---------------------------------------------------------------- main
@@ -238,6 +282,153 @@ def combine_ranks(ms, committed, world):
     return float(tmax[0]), float(t[1])
 
 
+def reference_arm(args, w, rank):
+    """--impl reference: the oracle as it stands, timed on the host cores
+    (rank 0 only) on the workload's own prompt: one untimed prefill, W
+    warm-up samples, then K timed samples of about cpu_seconds / K each."""
+    if rank != 0:
+        return 0
+    cores = os.cpu_count() or 1
+    run = OracleRun(w, make_weights(w))
+    run.dvi(0.0, steps_cap=args.warmup * w.update_every)
+    per = max(1.0, args.cpu_seconds / max(1, args.steps))
+    tot_c, tot_s, tot_steps = 0, 0.0, 0
+    for _ in range(args.steps):
+        c, st, sec = run.dvi(per)
+        tot_c += c
+        tot_s += sec
+        tot_steps += st
+    val = tot_c / tot_s
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": {"workload": w.name},
+            "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{args.steps} samples of ~{per:.1f} s: numpy float32 oracle on the "
+                                       f"{run.prompt}-token prompt (prefill untimed, {run.prefill_s:.0f} s), "
+                                       f"{tot_steps} DVI steps with updates"},
+            "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def make_engine(w, dw, max_len, local, persistent=False):
+    from paper_2510_05421_gb300 import DVIEngine
+    return DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=w.k_spec, split_k=w.split_k,
+                     lora_rank=w.lora_rank, lora_gamma=w.lora_gamma, max_seq_len=max_len,
+                     log_steps=w.update_every, device=local, persistent=persistent)
+
+
+def time_dvi(eng, w, hyper, warmup, steps, dev, world=1, clocks=False):
+    """W warm-up and K timed bench steps (update_every decode steps + one
+    drafter update each), CUDA events on the engine's stream."""
+    import torch
+    import torch.distributed as dist
+    U = w.update_every
+
+    def one_step():
+        for _ in range(U):
+            eng.step()
+        eng.update(hyper)
+
+    eng.log(True)
+    for _ in range(warmup):
+        one_step()
+    eng.sync()
+    lens0 = eng.buffer("LENS", torch.int32).cpu().numpy()
+    st0 = eng.stats()
+    eng.get_timing()
+    eng.timing(True)
+    sampler = ClockSampler(dev.index) if clocks else None
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(eng.stream)
+    for _ in range(steps):
+        one_step()
+    e1.record(eng.stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    clk = sampler.stop() if sampler else None
+    ms = e0.elapsed_time(e1)
+    phases = eng.get_timing()
+    eng.timing(False)
+    st1 = eng.stats()
+    lens1 = eng.buffer("LENS", torch.int32).cpu().numpy()
+    dsteps = st1["steps"] - st0["steps"]
+    return dict(ms=ms, committed=st1["committed"] - st0["committed"], decode_steps=dsteps,
+                mat=(st1["accepted"] - st0["accepted"]) / max(1, dsteps * w.batch),
+                launches=st1["kernel_launches"] - st0["kernel_launches"], phases=phases,
+                lens0=lens0, lens1=lens1, clocks=clk, status=st1["device_flags"])
+
+
+def time_ar(eng, dP, lens0, n_tokens, dev):
+    """Greedy AR (dvi_ar_step, the speedup's denominator, Sec. 4.1) on the
+    same engine, weights and context: every prompt prefilled again, advanced
+    untimed to the context the timed DVI region started at, then enough AR
+    steps for the same number of committed tokens, timed with CUDA events."""
+    import torch
+    B = len(dP)
+    for b, p in enumerate(dP):
+        eng.prefill(b, p)
+    warm = max(3, int(round(float(np.mean([lens0[b] - len(dP[b]) for b in range(B)])))))
+    for _ in range(warm):
+        eng.ar_step()
+    n_steps = max(1, -(-int(n_tokens) // B))
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(eng.stream)
+    for _ in range(n_steps):
+        eng.ar_step()
+    e1.record(eng.stream)
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1)
+    return {"tokens_per_s": B * n_steps / (ms / 1e3), "ms_per_step": ms / n_steps, "steps": n_steps}
+
+
+def pass_rooflines(w, r, hbm):
+    """Draft- and verify-phase HBM fractions from the per-phase timing."""
+    n_mid = (r["lens0"] + r["lens1"]) / 2.0
+    draft_b, verify_b = step_bytes(w, n_mid)
+    ph = r["phases"]
+    v_ms = ph["verify"][0] / max(1, ph["verify"][1])
+    d_ms = ph["draft"][0] / max(1, ph["draft"][1])
+    u_ms = ph["update"][0] / max(1, ph["update"][1])
+    return n_mid, draft_b, verify_b, d_ms, v_ms, u_ms
+
+
+def extra_workload(name, args, local, dev, pk):
+    """A second workload in the same run, reported beside the headline: the
+    1B model's drafter and verifier often agree, so its stream exercises
+    acceptance (mean accepted length, speedup over greedy AR)."""
+    import torch
+    from paper_2510_05421_gb300 import DeviceWeights, update_config
+    w = workload(name)
+    W = make_weights(w)
+    dw = DeviceWeights.from_host(W, w.dtype, device=dev)
+    P = make_prompts(w)
+    U, K = w.update_every, w.k_spec
+    steps = max(6, args.steps // 2)
+    max_len = max(len(p) for p in P) + (args.warmup + steps) * U * K + 2 * K + 64
+    eng = make_engine(w, dw, max_len, local)
+    dP = [torch.from_numpy(p).to(dev) for p in P]
+    for b, p in enumerate(dP):
+        eng.prefill(b, p)
+    r = time_dvi(eng, w, update_config(w.update), args.warmup, steps, dev)
+    ar = time_ar(eng, dP, r["lens0"], r["committed"], dev)
+    eng.close()
+    _, draft_b, verify_b, d_ms, v_ms, u_ms = pass_rooflines(w, r, pk["hbm_gbs"])
+    value = r["committed"] / (r["ms"] / 1e3)
+    return {"workload": w.name, "value": value, "unit": "tokens/s", "steps": steps,
+            "decode_steps": r["decode_steps"], "mean_accepted_length": r["mat"],
+            "ar_tokens_per_s": ar["tokens_per_s"], "speedup_vs_ar": value / ar["tokens_per_s"],
+            "verify_frac": verify_b / (v_ms / 1e3) / 1e9 / pk["hbm_gbs"],
+            "draft_frac": draft_b / (d_ms / 1e3) / 1e9 / pk["hbm_gbs"], "update_ms": u_ms,
+            "device_flags": r["status"]}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -245,6 +436,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="dvi", choices=["dvi", "reference"])
     ap.add_argument("--workload", default="7b")
+    ap.add_argument("--extra", default="1b", help="second workload reported beside the headline ('' = none)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -266,38 +458,18 @@ def main():
     assert args.warmup >= 3, "at least 3 warm-up steps"
 
     if args.impl == "reference":
-        if rank != 0:
-            return 0
-        cores = os.cpu_count() or 1
-        W = make_weights(w)
-        res_w = oracle_sample(w, W, 1e9, steps_cap=args.warmup * w.update_every)
-        per = max(1.0, args.cpu_seconds / max(1, args.steps))
-        tot_c, tot_s, tot_steps = 0, 0.0, 0
-        for _ in range(args.steps):
-            r = oracle_sample(w, W, per)
-            tot_c += r["committed"]
-            tot_s += r["seconds"]
-            tot_steps += r["steps"]
-        val = tot_c / tot_s
-        line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": args.gpus,
-                "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
-                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-                "data": "synthetic", "config": {"workload": w.name},
-                "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                                 "sample": f"{args.steps} samples of ~{per:.1f} s: numpy float32 oracle, prompt "
-                                           f"truncated to 64 tokens, {tot_steps} DVI steps with updates"},
-                "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
-        print(json.dumps(line), flush=True)
-        return 0
+        return reference_arm(args, w, rank)
 
     import torch
     import torch.distributed as dist
-    from paper_2510_05421_gb300 import DVIEngine, DeviceWeights, update_config
+    from paper_2510_05421_gb300 import DeviceWeights, update_config
 
     if world > 1:
         dist.init_process_group("gloo", init_method="env://")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    pk, pk_src = peaks()
+    hbm = pk["hbm_gbs"]
 
     W = make_weights(w)
     dw = DeviceWeights.from_host(W, w.dtype, device=dev)
@@ -305,9 +477,7 @@ def main():
     U, K = w.update_every, w.k_spec
     gen_room = max(w.gen_tokens, (args.warmup + args.steps) * U * K)
     max_len = max(len(p) for p in P) + gen_room + 2 * K + 64
-    eng = DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=K, split_k=w.split_k, lora_rank=w.lora_rank,
-                    lora_gamma=w.lora_gamma, max_seq_len=max_len, log_steps=U, device=local,
-                    persistent=args.persistent)
+    eng = make_engine(w, dw, max_len, local, args.persistent)
     hyper = update_config(w.update)
     # prefill: sequence 0's prompt once to warm up, then every prompt timed
     # with CUDA events on the engine's stream (prompts already on the device)
@@ -322,66 +492,28 @@ def main():
     torch.cuda.synchronize(dev)
     pf_ms = pf0.elapsed_time(pf1)
     pf_tokens = sum(len(p) for p in P)
-    pf_bytes = sum(prefill_bytes(w, len(p), eng.rt.max_prefill_chunk or 128) for p in P)
+    chunk = eng.rt.max_prefill_chunk or (1024 if w.dtype == "bf16" else 128)
+    pf_traffic = sum(prefill_bytes(w, len(p), chunk) for p in P)
+    pf_alg = sum(prefill_alg_bytes(w, len(p)) for p in P)
     pf_flops = sum(prefill_flops(w, len(p)) for p in P)
-    eng.log(True)
 
-    def one_step():
-        for _ in range(U):
-            eng.step()
-        eng.update(hyper)
-
-    for _ in range(args.warmup):
-        one_step()
-    eng.sync()
-    lens0 = eng.buffer("LENS", torch.int32).clone()
-    st0 = eng.stats()
-    eng.get_timing()
-    eng.timing(True)
-    clocks = ClockSampler(local)
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize(dev)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(eng.stream)
-    for _ in range(args.steps):
-        one_step()
-    e1.record(eng.stream)
-    torch.cuda.synchronize(dev)
-    if world > 1:
-        dist.barrier()
-    clk = clocks.stop()
-    ms = e0.elapsed_time(e1)
-    phases = eng.get_timing()
-    eng.timing(False)
-    st1 = eng.stats()
-    lens1 = eng.buffer("LENS", torch.int32).cpu().numpy()
-    lens0 = lens0.cpu().numpy()
-    committed = st1["committed"] - st0["committed"]
-    dsteps = st1["steps"] - st0["steps"]
-    mat = (st1["accepted"] - st0["accepted"]) / max(1, dsteps * w.batch)
-    launches = st1["kernel_launches"] - st0["kernel_launches"]
-    ms_all, committed_all = combine_ranks(ms, committed, world)
+    r = time_dvi(eng, w, hyper, args.warmup, args.steps, dev, world, clocks=True)
+    ms_all, committed_all = combine_ranks(r["ms"], r["committed"], world)
     value = committed_all / (ms_all / 1e3)
-
-    # roofline of the verify pass (and the draft pass), from the phase timing
-    pk, pk_src = peaks()
-    n_mid = (lens0 + lens1) / 2.0
-    draft_b, verify_b = step_bytes(w, n_mid)
-    v_ms = phases["verify"][0] / max(1, phases["verify"][1])
-    d_ms = phases["draft"][0] / max(1, phases["draft"][1])
-    u_ms = phases["update"][0] / max(1, phases["update"][1])
-    hbm = pk["hbm_gbs"]
+    n_mid, draft_b, verify_b, d_ms, v_ms, u_ms = pass_rooflines(w, r, hbm)
     v_gbs = verify_b / (v_ms / 1e3) / 1e9
-    v_traffic = measured_traffic(w, n_mid, args.persistent)
     d_gbs = draft_b / (d_ms / 1e3) / 1e9
+    v_traffic = measured_traffic(w, n_mid, args.persistent)
+
+    # greedy AR on the same engine, context and token count (rank-local)
+    ar = time_ar(eng, dP, r["lens0"], r["committed"], dev)
+    ar_ms_all, ar_tok_all = combine_ranks(ar["ms_per_step"] * ar["steps"], w.batch * ar["steps"], world)
+    ar_value = ar_tok_all / (ar_ms_all / 1e3)
 
     e2e = None
     if not args.no_e2e:
         eng.close()
-        eng = DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=K, split_k=w.split_k, lora_rank=w.lora_rank,
-                        lora_gamma=w.lora_gamma, max_seq_len=max(len(p) for p in P) + w.gen_tokens * K + 64,
-                        log_steps=U, device=local, persistent=args.persistent)
+        eng = make_engine(w, dw, max(len(p) for p in P) + w.gen_tokens * K + 64, local, args.persistent)
         eng.generate(P, 8, update_every=U, hyper=w.update, max_steps=2 * U)
         torch.cuda.synchronize(dev)
         t0 = time.perf_counter()
@@ -396,6 +528,12 @@ def main():
                         f"({len(P[0])} ids) to host token lists, prefill included, drafter updated every {U} "
                         f"steps; {len(mats)} decode steps, MAT {float(np.mean(mats)):.3f}")}
     eng.close()
+    del eng, dw
+    torch.cuda.empty_cache()
+
+    extra = None
+    if args.extra and not args.layers and not args.prompt:
+        extra = extra_workload(args.extra, args, local, dev, pk)
 
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -408,10 +546,14 @@ def main():
                    "l2": "inputs larger than L2: ~13 GB of weights streamed per step",
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "projections": "persistent chain" if args.persistent else "one kernel each"},
-        "mean_accepted_length": mat,
-        "prefill": {"tokens": pf_tokens, "ms": pf_ms, "tokens_per_s": pf_tokens / (pf_ms / 1e3),
-                    "chunk": eng.rt.max_prefill_chunk or 128,
-                    "roofline": prefill_roofline(pf_bytes, pf_flops, pf_ms, pk)},
+        "mean_accepted_length": r["mat"],
+        "ar_tokens_per_s": ar_value,
+        "speedup_vs_ar": value / ar_value,
+        "ar": {"note": ("dvi_ar_step (greedy AR of the full model, CUDA-graph replay) on the same engine, "
+                        "weights and starting context, timed over the same number of committed tokens"),
+               "ms_per_step": ar["ms_per_step"], "steps": ar["steps"]},
+        "prefill": {"tokens": pf_tokens, "ms": pf_ms, "tokens_per_s": pf_tokens / (pf_ms / 1e3), "chunk": chunk,
+                    "roofline": prefill_roofline(pf_flops, pf_alg, pf_ms, pk, traffic=pf_traffic)},
         "roofline": {"bound": "hbm", "achieved": v_gbs, "peak": hbm, "unit": "GB/s", "frac": v_gbs / hbm,
                      "traffic": v_traffic, "kernel": "verify pass (layers k+1..L + LM head, CUDA-graph replay)",
                      "traffic_source": "profiles/verify_pass_dram_7b_width.md (ncu, 4-layer case scaled)"
@@ -420,15 +562,20 @@ def main():
         "roofline_draft": {"bound": "hbm", "achieved": d_gbs, "peak": hbm, "unit": "GB/s", "frac": d_gbs / hbm,
                            "bytes_per_launch": draft_b, "ms_per_launch": d_ms},
         "update_ms": u_ms,
-        "gpu_launches": launches,
-        "clocks": clk,
+        "gpu_launches": r["launches"],
+        "clocks": r["clocks"],
+        "device_flags": r["status"],
     }
     if e2e:
         line["e2e"] = e2e
+    if extra:
+        line["extra_workload"] = extra
     if rank == 0 and world == 1 and not args.no_cpu:
         cores = os.cpu_count() or 1
-        res = oracle_sample(w, W, args.cpu_seconds)
-        line["cpu_baseline"] = cpu_baseline_dict(res, w, cores)
+        run = OracleRun(w, W)
+        dvi = run.dvi(args.cpu_seconds)
+        arc = run.ar(args.cpu_seconds / 2)
+        line["cpu_baseline"] = cpu_baseline_dict(run, dvi, arc, cores)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

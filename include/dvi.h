@@ -89,7 +89,10 @@ typedef struct {
                            (the LoRA factors, if any, stay frozen; the workspace then holds
                            the Adam moments of W^(S), an f32 master copy of it when dtype is
                            bf16, and the gradient buffer: 12 (f32) or 16 (bf16) B per entry) */
-  int max_prefill_chunk;/* rows per prefill pass, 16..128 (multiple of 16); 0 = 128 */
+  int max_prefill_chunk;/* rows per prefill pass, a multiple of 16: bf16 16..4096 (0 = 1024),
+                           f32 16..128 (0 = 128).  A bf16 pass runs its projections on the
+                           prefill kernel (128 token rows x 256 features per tile), so the
+                           weights stream from HBM about once per pass. */
   int use_graphs;       /* capture the decode step in a CUDA graph on first use */
   int bonus;            /* 0: verify the K drafted rows and commit min(m+1, K) tokens (Sec. 3.3
                            emits y*_{n+m+1}, which the K verify rows hold only for m < K);
@@ -275,8 +278,12 @@ dvi_status dvi_linear(dvi_ctx* ctx, const void* d_w, int n_out, int k_in,
  * call; it is a deployment convenience.
  *  - dtype: DVI_BF16 (tcgen05 path; k_in % 8 == 0, 16-byte aligned d_w and
  *    d_x) or DVI_F32 (FP32 FMA path).  d_w [n_out][k_in] in that dtype,
- *    d_x [m_rows][k_in] f32 (rounded to the dtype), d_y [m_rows][n_out] f32,
- *    all device pointers owned by the caller; 1 <= m_rows <= 256.
+ *    d_x [m_rows][k_in] f32, d_y [m_rows][n_out] f32, all device pointers
+ *    owned by the caller, on the current device; 1 <= m_rows <= 256.  With
+ *    bf16 weights the kernel carries each f32 input as a bf16 pair hi + lo
+ *    (about 16 significant bits), so only the weights are rounded.
+ *  - Every device of the process has its own scratch and its own kernel
+ *    attributes, each set up on the first call with that device current.
  *  - Shapes whose split plan needs more scratch than the fixed array holds
  *    return DVI_ERR_CAPACITY (with a message on stderr); for example a
  *    4096 x 4096 weight fits for up to 32 rows.

@@ -51,6 +51,15 @@ def prefill(model: OracleModel, cache: KVCache, prompt: Sequence[int]):
     return _argmax(logits), logits
 
 
+def ar_step(model: OracleModel, cache: KVCache, n: int, tok: int):
+    """One greedy AR step: the pending token x_n (at position n) through all
+    L layers, then argmax of the verifier head; returns (next token, logits)."""
+    x = model.embed([tok])
+    x = model.layers_range(0, model.s.n_layers, x, n, cache)
+    logits = model.verifier_logits(x)[0]
+    return _argmax(logits), logits
+
+
 def greedy_ar(model: OracleModel, prompt: Sequence[int], n_gen: int,
               return_logits: bool = False):
     """Greedy autoregressive decoding of n_gen tokens after the prompt."""
@@ -60,10 +69,7 @@ def greedy_ar(model: OracleModel, prompt: Sequence[int], n_gen: int,
     out, rows, gaps = [tok], [logits], [_top2_gap(logits)]
     n = P
     while len(out) < n_gen:
-        x = model.embed([tok])
-        x = model.layers_range(0, model.s.n_layers, x, n, cache)
-        logits = model.verifier_logits(x)[0]
-        tok = _argmax(logits)
+        tok, logits = ar_step(model, cache, n, tok)
         out.append(tok)
         rows.append(logits)
         gaps.append(_top2_gap(logits))

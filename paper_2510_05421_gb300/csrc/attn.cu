@@ -844,12 +844,11 @@ static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
     // one cluster of n_splits_max (<= 8) CTAs per (sequence, query group, KV
     // head); decode and prefill chunks alike (16 / G query rows per group)
     const size_t smem = 1024 + static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * 2;
-    static bool mma_attr = false;
-    if (!mma_attr) {
+    static PerDevice mma_attr;
+    mma_attr.once([] {
       cudaFuncSetAttribute(attn_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
       cudaFuncSetAttribute(attn_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-      mma_attr = true;
-    }
+    });
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = dim3(128);
@@ -871,20 +870,16 @@ static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
     const size_t ring = static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * sizeof(T);
     const int qmax = std::min(kRegQ, a.rows_per_seq * (a.n_heads / a.n_kv_heads));
     const int wq = qmax <= kQPW ? 1 : (qmax <= 2 * kQPW ? 2 : 4);
-    static bool dec_attr = false;
-    if (!dec_attr) {
+    static PerDevice dec_attr;
+    dec_attr.once([] {
       cudaFuncSetAttribute(attn_dec_kernel<T, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
       cudaFuncSetAttribute(attn_dec_kernel<T, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-      dec_attr = true;
-    }
+    });
     if (a.head_dim == 128) return launch_pdl(attn_dec_kernel<T, 4>, grid, dim3(128), ring, s, a, wq);
     return launch_pdl(attn_dec_kernel<T, 2>, grid, dim3(128), ring, s, a, wq);
   }
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(attn_smem_kernel<T, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024);
-    attr = true;
-  }
+  static PerDevice attr;
+  attr.once([] { cudaFuncSetAttribute(attn_smem_kernel<T, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024); });
   return launch_pdl(attn_smem_kernel<T, T>, grid, dim3(128), attn_smem(a.head_dim), s, a);
 }
 

@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <utility>
 
 #include "../../include/dvi.h"
@@ -20,6 +21,7 @@ constexpr int kKBlock = 64;          // bf16 K elements per pipeline stage (128 
 constexpr int kKBlockF32 = 32;       // f32 K elements per stage of the FFMA kernel
 constexpr int kChunk = 16;           // token columns per epilogue chunk
 constexpr int kMaxTokens = 256;      // rows of one projection launch (tcgen05 N <= 256)
+constexpr int kMaxPrefillChunk = 4096;  // rows of one bf16 prompt pass (prefill kernel)
 constexpr int kAttnQ = 16;           // query vectors per attention CTA
 constexpr int kAttnBlk = 64;         // KV positions per attention sub-block
 
@@ -342,6 +344,31 @@ __host__ __device__ __forceinline__ uint32_t sw128_offset(int row, int k) {
   return static_cast<uint32_t>(row) * 128u + ((static_cast<uint32_t>(k >> 3) ^ (row & 7)) << 4) +
          static_cast<uint32_t>((k & 7) * 2);
 }
+
+// Function attributes (the dynamic shared-memory limit, the carveout) belong
+// to one device's context.  A launcher keeps one PerDevice and runs its
+// attribute calls through once(): the first time it launches with a device
+// current, and again for every further device of the process (ids 0..63;
+// others set the attributes on every call).  Two threads may both run the
+// set-up for one device; setting an attribute twice is harmless.
+class PerDevice {
+ public:
+  template <typename F>
+  void once(F set) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+      set();
+      return;
+    }
+    const uint64_t bit = 1ull << dev;
+    if (done_.load(std::memory_order_acquire) & bit) return;
+    set();
+    done_.fetch_or(bit, std::memory_order_acq_rel);
+  }
+
+ private:
+  std::atomic<uint64_t> done_{0};
+};
 
 // Launch with programmatic stream serialization (see griddep_wait).
 template <typename... KArgs, typename... Args>

@@ -24,6 +24,7 @@ namespace {
 
 struct LayerMaps {
   ProjMaps qkv, o, gu, down;
+  CUtensorMap gate128, up128;   // gate / up with 128-row boxes (prefill kernel)
 };
 
 // One pass of token rows through layers: the f32 residual stream x, its
@@ -40,6 +41,7 @@ struct Pass {
   int pos_off;
   void* xg;
   const CUtensorMap* xg_map;
+  bool pf = false;   // a bf16 prompt pass: projections on the prefill kernel
 };
 
 struct Plan {
@@ -60,6 +62,7 @@ struct dvi_ctx {
   bool tc = false;
   size_t esz = 4;
   int L, d, Hq, Hkv, hd, F, V, k, r, B, K, max_len, cap_steps, cap_rows, chunk, M_max, nq, nkv;
+  int pf_rows;   // rows of the prompt-pass buffers: chunk, rounded up to 128 for bf16
   int Kv;   // verify rows per sequence: K, or K + 1 with the bonus row
   // device state
   int *lens, *pending, *draft_ids, *status, *log_step, *log_meta;
@@ -100,12 +103,15 @@ struct dvi_ctx {
   ProjMaps head_v, head_s;
   // TMA descriptors of the activation buffers (bf16 model)
   CUtensorMap map_xg_dr, map_xg_ver, map_xg_pf, map_attn_o, map_ffn_h, map_log_u;
+  // the prompt-pass activation buffers with 128-row boxes (prefill kernel)
+  CUtensorMap map_pf_xg, map_pf_attn_o, map_pf_ffn_h;
   CUtensorMap map_kc, map_vc;   // K / V caches as [L*B*H_kv*max_len][hd]
   int log_enabled = 1;
   // graphs of one decode step: the K draft passes, then the verify pass
   cudaGraphExec_t draft_exec = nullptr, verify_exec = nullptr;
-  int step_calls = 0;
-  long long draft_launches = 0, verify_launches = 0;
+  cudaGraphExec_t ar_exec = nullptr;   // one greedy AR step of the full model
+  int step_calls = 0, ar_calls = 0;
+  long long draft_launches = 0, verify_launches = 0, ar_launches = 0;
   long long launches = 0;
   // optional per-phase timing (0 draft, 1 verify, 2 update): event pairs
   int timing = 0;
@@ -154,8 +160,9 @@ bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::
   if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
     return bad("log_steps * batch * k_spec must be in [1, 256]");
   if (rt->head_mode != 0 && rt->head_mode != 1) return bad("head_mode must be 0 (LoRA) or 1 (full W^S)");
-  if (rt->max_prefill_chunk && (rt->max_prefill_chunk < 16 || rt->max_prefill_chunk > 128 || rt->max_prefill_chunk % 16))
-    return bad("max_prefill_chunk must be 16..128, a multiple of 16");
+  if (rt->max_prefill_chunk && (rt->max_prefill_chunk < 16 || rt->max_prefill_chunk % 16 ||
+                                 rt->max_prefill_chunk > (c->dtype == DVI_BF16 ? kMaxPrefillChunk : 128)))
+    return bad("max_prefill_chunk must be a multiple of 16 in 16..4096 (bf16) or 16..128 (f32)");
   if (rt->batch * (rt->k_spec + rt->bonus) > kMaxTokens) return bad("batch * (k_spec + bonus) > 256");
   return true;
 }
@@ -185,13 +192,13 @@ size_t layout(dvi_ctx* c, char* base) {
   c->ss_dr = reinterpret_cast<float*>(take(sizeof(float) * st * B));
   c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * c->Kv * d));
   c->ss_ver = reinterpret_cast<float*>(take(sizeof(float) * st * B * c->Kv));
-  c->x_pf = reinterpret_cast<float*>(take(sizeof(float) * c->chunk * d));
-  c->ss_pf = reinterpret_cast<float*>(take(sizeof(float) * st * c->chunk));
+  c->x_pf = reinterpret_cast<float*>(take(sizeof(float) * c->pf_rows * d));
+  c->ss_pf = reinterpret_cast<float*>(take(sizeof(float) * st * c->pf_rows));
   // activation rows feeding matrix products: bf16 keeps a hi and a lo plane
   const size_t pl = c->tc ? 2 : 1;
   c->xg_dr = take(pl * e * B * d);
   c->xg_ver = take(pl * e * B * c->Kv * d);
-  c->xg_pf = take(pl * e * c->chunk * d);
+  c->xg_pf = take(pl * e * c->pf_rows * d);
   c->q = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * c->nq));
   c->bu = reinterpret_cast<float*>(take(sizeof(float) * c->M_max * (r > 0 ? r : 1)));
   c->attn_o = take(pl * e * c->M_max * c->nq);
@@ -298,8 +305,11 @@ void size_scratch(dvi_ctx* c) {
     ap = std::max(ap, attn_partial_floats(at));
     ac = std::max(ac, attn_counters(at));
   }
-  c->attn_part_floats = ap;
-  c->n_attn_ctr = ac;
+  // the bf16 tensor-core attention (GQA groups up to 8) combines its splits
+  // through distributed shared memory and needs no global scratch
+  const bool cluster_attn = c->tc && c->Hq / c->Hkv <= 8;
+  c->attn_part_floats = cluster_attn ? 0 : ap;
+  c->n_attn_ctr = cluster_attn ? 1 : ac;
   // persistent projection chain (runtime option; bf16 passes of up to
   // kChainMaxPad rows): as many CTAs as the SMs keep resident at every n_pad
   c->chain_ctas = 0;
@@ -333,9 +343,10 @@ bool init_dims(dvi_ctx* c, const dvi_model_config* cfg, const dvi_runtime_config
   c->max_len = rt->max_seq_len;
   c->cap_steps = rt->log_steps;
   c->cap_rows = rt->log_steps * rt->batch * rt->k_spec;
-  c->chunk = rt->max_prefill_chunk ? rt->max_prefill_chunk : 128;
+  c->chunk = rt->max_prefill_chunk ? rt->max_prefill_chunk : (cfg->dtype == DVI_BF16 ? 1024 : 128);
+  c->pf_rows = cfg->dtype == DVI_BF16 ? (c->chunk + 127) / 128 * 128 : c->chunk;
   c->Kv = c->K + (rt->bonus ? 1 : 0);
-  c->M_max = std::max(std::max(c->B * c->Kv, c->chunk), std::max(c->cap_rows, c->B));
+  c->M_max = std::max(std::max(c->B * c->Kv, c->pf_rows), std::max(c->cap_rows, c->B));
   c->nq = c->Hq * c->hd;
   c->nkv = c->Hkv * c->hd;
   c->tc = cfg->dtype == DVI_BF16;
@@ -395,7 +406,7 @@ ProjMaps with_act(const ProjMaps& w, const CUtensorMap* act) {
 int act_rows(const dvi_ctx* c, const void* buf) {
   if (buf == c->xg_dr) return c->B;
   if (buf == c->xg_ver) return c->B * c->Kv;
-  if (buf == c->xg_pf) return c->chunk;
+  if (buf == c->xg_pf) return c->pf_rows;
   if (buf == c->attn_o || buf == c->ffn_h) return c->M_max;
   if (buf == c->log_u) return c->cap_rows;
   return 0;
@@ -587,13 +598,45 @@ dvi_status chain_flush(dvi_ctx* ctx, ChainBuilder& cb) {
 
 // The persistent chain serves bf16 passes of up to kChainMaxPad rows.
 bool use_chain(const dvi_ctx* ctx, const Pass& ps) {
-  return ctx->tc && ctx->chain_ctas > 0 && (ps.M + 15) / 16 * 16 <= kChainMaxPad;
+  return ctx->tc && !ps.pf && ctx->chain_ctas > 0 && (ps.M + 15) / 16 * 16 <= kChainMaxPad;
 }
 
 // One decoder layer on the pass's rows, one kernel per projection.  `g_last`
 // is the gain of whatever consumes the pass's residual after this layer (the
 // next layer's attention norm, or the final norm before a head).
+// A projection of a bf16 prompt pass on the prefill kernel, with the
+// activation buffer's 128-row map and the weights' 128-row maps.
+dvi_status run_proj_pf(dvi_ctx* ctx, const ProjLaunch& pl, const CUtensorMap& act, const CUtensorMap& w0,
+                       const CUtensorMap* w1 = nullptr, const CUtensorMap* w2 = nullptr) {
+  ProjArgs a = pl.a;
+  if (a.xg_out) a.xg_plane = act_plane(ctx, a.xg_out, a.ld_xg);
+  if (a.h_out) a.h_plane = act_plane(ctx, a.h_out, a.ld_h);
+  PfMaps m;
+  m.act = act;
+  m.w0 = w0;
+  m.w1 = w1 ? *w1 : w0;
+  m.w2 = w2 ? *w2 : w0;
+  DVI_CUDA(launch_proj_pf(a, m, ctx->n_sms, ctx->stream));
+  ++ctx->launches;
+  return DVI_OK;
+}
+
+// One layer of a bf16 prompt pass: QKV, gate/up, O and down on the prefill
+// kernel, the attention on the decode attention kernel.
+dvi_status enqueue_layer_pf(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last) {
+  const LayerMaps& m = ctx->maps[l];
+  dvi_status st;
+  if ((st = run_proj_pf(ctx, qkv_launch(ctx, l, ps), ctx->map_pf_xg, m.qkv.m0, &m.qkv.m1, &m.qkv.m2)) != DVI_OK)
+    return st;
+  DVI_CUDA(launch_attn(attn_args(ctx, l, ps), ctx->stream));
+  ++ctx->launches;
+  if ((st = run_proj_pf(ctx, o_launch(ctx, l, ps), ctx->map_pf_attn_o, m.o.m0)) != DVI_OK) return st;
+  if ((st = run_proj_pf(ctx, gu_launch(ctx, l, ps), ctx->map_pf_xg, m.gate128, &m.up128)) != DVI_OK) return st;
+  return run_proj_pf(ctx, down_launch(ctx, l, ps, g_last), ctx->map_pf_ffn_h, m.down.m0);
+}
+
 dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last) {
+  if (ps.pf) return enqueue_layer_pf(ctx, l, ps, g_last);
   dvi_status st;
   if ((st = run_proj(ctx, qkv_launch(ctx, l, ps))) != DVI_OK) return st;
   DVI_CUDA(launch_attn(attn_args(ctx, l, ps), ctx->stream));
@@ -869,7 +912,8 @@ dvi_status run_graph(dvi_ctx* ctx, cudaGraphExec_t* exec, long long* nlaunch, bo
 void drop_graphs(dvi_ctx* c) {
   if (c->draft_exec) cudaGraphExecDestroy(c->draft_exec);
   if (c->verify_exec) cudaGraphExecDestroy(c->verify_exec);
-  c->draft_exec = c->verify_exec = nullptr;
+  if (c->ar_exec) cudaGraphExecDestroy(c->ar_exec);
+  c->draft_exec = c->verify_exec = c->ar_exec = nullptr;
 }
 
 }  // namespace
@@ -906,6 +950,12 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
     fprintf(stderr, "dvi_create: lora_b and final_norm must be 16-byte aligned\n");
     return DVI_ERR_INVALID_ARG;
   }
+  // the bf16 prompt passes read the layers' norm gains four floats at a time
+  for (int l = 0; l < cfg->n_layers && cfg->dtype == DVI_BF16; ++l)
+    if (!aligned16(weights->layers[l].attn_norm) || !aligned16(weights->layers[l].ffn_norm)) {
+      fprintf(stderr, "dvi_create: attn_norm and ffn_norm must be 16-byte aligned\n");
+      return DVI_ERR_INVALID_ARG;
+    }
   if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return DVI_ERR_INVALID_ARG;
   dvi_ctx* ctx = new dvi_ctx();
   init_dims(ctx, cfg, rt);
@@ -933,6 +983,7 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
            mk(&m.qkv.m2, lw.wv, ctx->nkv, ctx->d) && mk(&m.o.m0, lw.wo, ctx->d, ctx->nq) &&
            aligned16(lw.w_gate) && make_half_weight_map(&m.gu.m0, lw.w_gate, ctx->F, ctx->d) &&
            aligned16(lw.w_up) && make_half_weight_map(&m.gu.m1, lw.w_up, ctx->F, ctx->d) &&
+           mk(&m.gate128, lw.w_gate, ctx->F, ctx->d) && mk(&m.up128, lw.w_up, ctx->F, ctx->d) &&
            mk(&m.down.m0, lw.w_down, ctx->d, ctx->F);
     }
     ok = ok && mk(&ctx->head_v.m0, weights->lm_head, ctx->V, ctx->d) &&
@@ -940,7 +991,10 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
     // each map covers both planes of its buffer: [2][R][cols]
     ok = ok && make_act_map(&ctx->map_xg_dr, ctx->xg_dr, ctx->B, ctx->d) &&
          make_act_map(&ctx->map_xg_ver, ctx->xg_ver, ctx->B * ctx->Kv, ctx->d) &&
-         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, ctx->chunk, ctx->d) &&
+         make_act_map(&ctx->map_xg_pf, ctx->xg_pf, ctx->pf_rows, ctx->d) &&
+         make_act_map_box(&ctx->map_pf_xg, ctx->xg_pf, ctx->pf_rows, ctx->d, kTileRows) &&
+         make_act_map_box(&ctx->map_pf_attn_o, ctx->attn_o, ctx->M_max, ctx->nq, kTileRows) &&
+         make_act_map_box(&ctx->map_pf_ffn_h, ctx->ffn_h, ctx->M_max, ctx->F, kTileRows) &&
          make_act_map(&ctx->map_attn_o, ctx->attn_o, ctx->M_max, ctx->nq) &&
          make_act_map(&ctx->map_ffn_h, ctx->ffn_h, ctx->M_max, ctx->F) &&
          make_act_map(&ctx->map_log_u, ctx->log_u, ctx->cap_rows, ctx->d);
@@ -989,7 +1043,7 @@ dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tok
     e.x = ctx->x_pf;
     e.ldx = ctx->d;
     e.ss = ctx->ss_pf;
-    e.ss_ld = ctx->chunk;
+    e.ss_ld = ctx->pf_rows;
     e.g = norm_gain_before(ctx, 0);
     e.xg = ctx->xg_pf;
     e.xg_plane = act_plane(ctx, ctx->xg_pf, ctx->d);
@@ -998,14 +1052,14 @@ dvi_status dvi_prefill(dvi_ctx* ctx, int seq, const int32_t* d_tokens, int n_tok
     e.status = ctx->status;
     DVI_CUDA(launch_embed(e, s));
     ctx->launches += 1;
-    Pass ps{ctx->x_pf, ctx->ss_pf, ctx->chunk, rows, rows, seq, 1, c0, ctx->xg_pf, &ctx->map_xg_pf};
+    Pass ps{ctx->x_pf, ctx->ss_pf, ctx->pf_rows, rows, rows, seq, 1, c0, ctx->xg_pf, &ctx->map_xg_pf, ctx->tc};
     dvi_status rc = enqueue_layers(ctx, 0, ctx->L, ps);
     if (rc != DVI_OK) return rc;
     last_rows = rows;
   }
   // verifier head on the last prompt row
   dvi_status rc = enqueue_head(ctx, false, 1, 0, ctx->xg_pf, &ctx->map_xg_pf, last_rows - 1,
-                               ctx->ss_pf + (last_rows - 1), ctx->chunk);
+                               ctx->ss_pf + (last_rows - 1), ctx->pf_rows);
   if (rc != DVI_OK) return rc;
   DVI_CUDA(launch_finalize_prefill(st, seq, n_tokens, d_first_token, s));
   ctx->launches += 2;
@@ -1131,15 +1185,23 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
 dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
   if (!ctx) return DVI_ERR_INVALID_ARG;
   cudaStream_t s = ctx->stream;
-  StepState st = step_state(ctx);
-  st.out_ids = ctx->ar_out;
-  Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr};
-  dvi_status rc = enqueue_layers(ctx, 0, ctx->L, ps);
+  ctx->ar_calls += 1;
+  // like the decode step: the first call runs eagerly, later calls replay
+  // its captured graph (every input of the step is device-side state)
+  const bool g = ctx->rt.use_graphs && ctx->ar_calls > 1;
+  dvi_status rc = run_graph(ctx, &ctx->ar_exec, &ctx->ar_launches, g, [&]() -> dvi_status {
+    StepState st = step_state(ctx);
+    st.out_ids = ctx->ar_out;
+    Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr};
+    dvi_status r = enqueue_layers(ctx, 0, ctx->L, ps);
+    if (r != DVI_OK) return r;
+    if ((r = enqueue_head(ctx, false, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
+      return r;
+    DVI_CUDA(launch_finalize_ar(st, s));
+    ctx->launches += 1;
+    return DVI_OK;
+  });
   if (rc != DVI_OK) return rc;
-  if ((rc = enqueue_head(ctx, false, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
-    return rc;
-  DVI_CUDA(launch_finalize_ar(st, s));
-  ctx->launches += 1;
   if (d_out_ids) DVI_CUDA(cudaMemcpyAsync(d_out_ids, ctx->ar_out, sizeof(int) * ctx->B, cudaMemcpyDeviceToDevice, s));
   return DVI_OK;
 }

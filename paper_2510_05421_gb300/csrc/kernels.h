@@ -88,6 +88,19 @@ cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s)
 bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols);   // 64-row boxes (gate/up)
 bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);   // [2 planes][rows][cols]
+// The same activation buffer with boxes of `box_rows` (<= 256) rows.
+bool make_act_map_box(CUtensorMap* map, const void* act, int rows, int cols, int box_rows);
+
+// Prompt passes (bf16): the prefill kernel (prefill.cu) puts 128 token rows
+// on the MMA's M side and 256 output features on N, persistent CTAs, two
+// TMEM accumulators.  `a` is the decode launch's ProjArgs (flavours QKV,
+// RESID, GATEUP; rows of one sequence); `act` maps the activation buffer
+// with 128-row boxes; w0..w2 map the weights with 128-row boxes (QKV: wq,
+// wk, wv; gate/up: gate, up).
+struct PfMaps {
+  CUtensorMap act, w0, w1, w2;
+};
+cudaError_t launch_proj_pf(const ProjArgs& a, const PfMaps& m, int n_sms, cudaStream_t s);
 
 // Persistent projection chain (bf16): up to kChainMax projections of one
 // pass in a single launch, each phase's output feeding the next phase's B

@@ -77,6 +77,9 @@ extern "C" dvi_status dvi_linear_noalloc(int dtype, const void* d_w, int n_out, 
   const bool tc = dtype == DVI_BF16;
   if (tc && (k_in % 8 || (reinterpret_cast<uintptr_t>(d_w) & 15u) || (reinterpret_cast<uintptr_t>(d_x) & 15u)))
     return DVI_ERR_INVALID_ARG;
+  // An error left pending by the caller's earlier CUDA work must not be
+  // reported as this call's launch failure.
+  cudaGetLastError();
   DeviceScratch s;
   const dvi_status rc = current_scratch(&s);
   if (rc != DVI_OK) return rc;

@@ -1177,12 +1177,11 @@ static int tc_stages(int n_pad, size_t* smem_bytes) {
 cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s) {
   cudaError_t e;
   if (a0.dtype == DVI_BF16) {
-    static bool attr = false;
-    if (!attr) {
+    static PerDevice attr;
+    attr.once([] {
       cudaFuncSetAttribute(proj_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
       cudaFuncSetAttribute(proj_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-      attr = true;
-    }
+    });
     ProjArgs a = a0;
     size_t smem = 0;
     const int stages = tc_stages(a.n_pad, &smem);
@@ -1223,13 +1222,12 @@ static int chain_stages(int n_pad, size_t* smem_bytes) {
 }
 
 static void chain_attr() {
-  static bool done = false;
-  if (!done) {
+  static PerDevice done;
+  done.once([] {
     cudaFuncSetAttribute(proj_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     cudaFuncSetAttribute(proj_chain_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                          cudaSharedmemCarveoutMaxShared);
-    done = true;
-  }
+  });
 }
 
 int chain_ctas_per_sm(int n_pad) {
@@ -1310,18 +1308,21 @@ bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
   return make_map(map, w, rows, cols, kGuRows);
 }
-bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols) {
-  // two planes (hi, lo) of [rows][cols] bf16, boxes of 16 rows x 64 columns
+bool make_act_map_box(CUtensorMap* map, const void* act, int rows, int cols, int box_rows) {
+  // two planes (hi, lo) of [rows][cols] bf16, boxes of box_rows rows x 64 columns
   auto encode = encoder();
-  if (!encode) return false;
+  if (!encode || box_rows < 1 || box_rows > 256) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows), 2};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2, static_cast<cuuint64_t>(rows) * cols * 2};
-  cuuint32_t box[3] = {kKBlock, 16, 1};
+  cuuint32_t box[3] = {kKBlock, static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(act), dims, strides, box,
                             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols) {
+  return make_act_map_box(map, act, rows, cols, 16);
 }
 bool make_kv_map(CUtensorMap* map, const void* cache, long long rows, int hd) {
   auto encode = encoder();

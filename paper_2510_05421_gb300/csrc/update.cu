@@ -582,11 +582,10 @@ cudaError_t launch_update_coef(const UpdateArgs& a, cudaStream_t s) {
 cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s) {
   if (a.r == 0) return cudaSuccess;
   const size_t smem = sizeof(float) * (static_cast<size_t>(a.cap) * 128 + 128 * a.r);
-  static size_t attr = 0;
-  if (smem > 48 * 1024 && smem > attr) {
+  // set on every call above 48 KiB (once per update; the attribute is per
+  // device, and this keeps it right on whichever device is current)
+  if (smem > 48 * 1024)
     cudaFuncSetAttribute(update_grad_a_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-    attr = smem;
-  }
   const cudaError_t e = launch_pdl(update_grad_a_kernel, dim3(a.n_vtiles), dim3(128), smem, s, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

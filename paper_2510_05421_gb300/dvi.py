@@ -163,17 +163,45 @@ class DeviceWeights:
                              draft_head=lm.clone(), lora_a=f32(w.lora_a), lora_b=f32(w.lora_b))
 
 
+def check_linear_noalloc_args(w, x, y) -> None:
+    """Raise ValueError unless (w, x, y) is a call dvi_linear_noalloc can run:
+    w [N, K] bf16 or f32, x [M, K] f32, y [M, N] f32, all contiguous and on
+    one CUDA device, 1 <= M <= 256.  Nothing is launched before this passes,
+    so a wrong tensor never reaches the kernel as a raw pointer."""
+    if w.dtype not in (torch.bfloat16, torch.float32):
+        raise ValueError("linear_noalloc: w must be bf16 or float32")
+    if x.dtype != torch.float32 or y.dtype != torch.float32:
+        raise ValueError("linear_noalloc: x and y must be float32")
+    if len(w.shape) != 2 or len(x.shape) != 2 or len(y.shape) != 2:
+        raise ValueError("linear_noalloc: w, x and y must be 2-D")
+    n, k = w.shape
+    m = x.shape[0]
+    if x.shape[1] != k or tuple(y.shape) != (m, n):
+        raise ValueError(f"linear_noalloc: shapes w {tuple(w.shape)}, x {tuple(x.shape)}, y {tuple(y.shape)} "
+                         "do not match y[M, N] = x[M, K] w[N, K]^T")
+    if not 1 <= m <= 256 or n < 1 or k < 1:
+        raise ValueError("linear_noalloc: needs 1 <= M <= 256 rows and a non-empty weight")
+    if not (w.is_contiguous() and x.is_contiguous() and y.is_contiguous()):
+        raise ValueError("linear_noalloc: w, x and y must be contiguous")
+    if not (w.is_cuda and x.is_cuda and y.is_cuda) or not (w.device == x.device == y.device):
+        raise ValueError("linear_noalloc: w, x and y must be on one CUDA device")
+
+
 def linear_noalloc(w: torch.Tensor, x: torch.Tensor, y: torch.Tensor, stream=None) -> int:
     """Y = X W^T through dvi_linear_noalloc (no context, no device allocation).
 
     For callers that cannot allocate device memory: the caller provides w
     ([N, K] bf16 or f32), x ([M, K] f32) and y ([M, N] f32); the library's
-    fixed scratch is used.  Returns the status code (0 on success).
+    fixed scratch on w's device is used (the call runs with that device
+    current).  Raises ValueError on tensors the kernel cannot take; returns
+    the library's status code (0 on success).
     """
+    check_linear_noalloc_args(w, x, y)
     dtype = DVI_BF16 if w.dtype == torch.bfloat16 else DVI_F32
-    s = stream if stream is not None else torch.cuda.current_stream(w.device)
-    return lib().dvi_linear_noalloc(dtype, _ptr(w), w.shape[0], w.shape[1], _ptr(x), x.shape[0], _ptr(y),
-                                    ctypes.c_void_p(s.cuda_stream))
+    with torch.cuda.device(w.device):
+        s = stream if stream is not None else torch.cuda.current_stream(w.device)
+        return lib().dvi_linear_noalloc(dtype, _ptr(w), w.shape[0], w.shape[1], _ptr(x), x.shape[0], _ptr(y),
+                                        ctypes.c_void_p(s.cuda_stream))
 
 
 class DVIEngine:
@@ -181,7 +209,7 @@ class DVIEngine:
 
     def __init__(self, shape, dtype: str, weights: DeviceWeights, *, batch: int, k_spec: int, split_k: int,
                  lora_rank: int, lora_gamma: float = 1.0, max_seq_len: int, log_steps: int,
-                 prefill_chunk: int = 128, use_graphs: bool = True, device: int = 0, head_mode: int = 0,
+                 prefill_chunk: int = 0, use_graphs: bool = True, device: int = 0, head_mode: int = 0,
                  bonus: bool = False, persistent: bool = False):
         L = lib()
         self.shape, self.dtype, self.w = shape, dtype, weights

@@ -41,3 +41,82 @@ def teacher_forced_logits(model, seq_tokens):
     cache = model.new_cache(len(seq_tokens) + 1)
     x = model.layers_range(0, L, model.embed(seq_tokens), 0, cache)
     return model.verifier_logits(x)
+
+
+def teacher_forced_tail(model, seq_tokens, start):
+    """Verifier logits at input positions start.. of one full sequence (one
+    causal pass through every layer; the head only on the rows asked for)."""
+    L = model.s.n_layers
+    cache = model.new_cache(len(seq_tokens) + 1)
+    x = model.layers_range(0, L, model.embed(seq_tokens), 0, cache)
+    return model.verifier_logits(x[start:])
+
+
+def run_logged_steps(eng, prompts, n_steps, update_every=0, hyper=None):
+    """Prefill every prompt, then run `n_steps` decode steps one at a time and
+    read the replay buffer after each: the verify rows every step logged.
+
+    Returns (committed tokens per sequence including the prefill's first
+    token, rows) with rows = [(b, input position, logits float64 [V], y*)];
+    row i of a step for a sequence at committed length n has its input token
+    at position n + i, so the oracle's teacher-forced logits at that position
+    are its reference.  The drafter is updated every `update_every` steps."""
+    B, K, V = eng.B, eng.K, eng.shape.vocab
+    for b, p in enumerate(prompts):
+        eng.prefill(b, torch.from_numpy(np.ascontiguousarray(p, dtype=np.int32)).to(eng.device))
+    eng.log(True)
+    eng.sync()
+    first = eng.first.cpu().numpy()
+    toks = [[int(first[b])] for b in range(B)]
+    n = [len(p) for p in prompts]
+    rows = []
+    j = 0
+    meta_all = eng.buffer("LOG_META", torch.int32).view(-1, 6)
+    lg_all = eng.buffer("LOG_LOGITS", torch.float32).view(-1, V)
+    for _ in range(n_steps):
+        ids, cnt, _ = eng.step()
+        eng.sync()
+        ids, cnt = ids.cpu().numpy(), cnt.cpu().numpy()
+        base = j * B * K
+        meta = meta_all[base:base + B * K].cpu().numpy()
+        lg = lg_all[base:base + B * K].double().cpu().numpy()
+        for b in range(B):
+            c = int(cnt[b])
+            assert 1 <= c <= K
+            for i in range(K):
+                slot = b * K + i
+                assert meta[slot, 0] == (1 if i < c else 0), (b, i, meta[slot])
+                if i < c:
+                    rows.append((b, n[b] + i, lg[slot], int(meta[slot, 5])))
+            toks[b].extend(int(t) for t in ids[b, :c])
+            n[b] += c
+        j += 1
+        if update_every and hyper is not None and j == update_every:
+            eng.update(hyper)
+            j = 0
+    return toks, rows
+
+
+def check_rows_against_oracle(model, prompts, toks, rows, tol):
+    """Every logged verify row within `tol` (max abs) of the oracle's
+    teacher-forced logits on the committed sequence, y* the argmax of the
+    GPU row, and y* equal to the oracle's argmax wherever the oracle's top-2
+    gap exceeds 2 tol.  Returns the largest error seen."""
+    worst = 0.0
+    by_seq = {}
+    for b, pos, lg, ys in rows:
+        by_seq.setdefault(b, []).append((pos, lg, ys))
+    for b, rs in by_seq.items():
+        seq = np.concatenate([prompts[b], np.asarray(toks[b], dtype=np.int32)])
+        start = len(prompts[b])
+        ref = teacher_forced_tail(model, seq, start)
+        for pos, lg, ys in rs:
+            r = ref[pos - start]
+            err = float(np.abs(lg - r).max())
+            worst = max(worst, err)
+            assert err < tol, (b, pos, err)
+            assert int(np.argmax(lg)) == ys, (b, pos)
+            top2 = np.partition(r, -2)[-2:]
+            if top2[1] - top2[0] > 2 * tol:
+                assert int(np.argmax(r)) == ys, (b, pos)
+    return worst

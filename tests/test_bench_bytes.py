@@ -85,9 +85,14 @@ def test_prefill_flops_and_bound():
     assert bench.prefill_flops(w, 1024) == expect
     assert expect == pytest.approx(13.54e12, rel=1e-3)
     pk = {"hbm_gbs": 6785.5, "bf16_tflops": 1884.7}
-    # 128-row passes stream the weights 8 times: the bytes bound the time
-    r = bench.prefill_roofline(bench.prefill_bytes(w, 1024, 128), expect, 72.0, pk)
-    assert r["bound"] == "hbm" and r["unit"] == "GB/s"
-    # one 1024-row pass: the tensor pipe bounds it
-    r = bench.prefill_roofline(bench.prefill_bytes(w, 1024, 1024), expect, 10.0, pk)
-    assert r["bound"] == "tensor" and r["achieved"] == pytest.approx(expect / 1e-2 / 1e12)
+    # the algorithm reads every weight once: 13.5 TFLOP against ~14.3 GB is
+    # far above the ridge, so the tensor pipe bounds it whatever the passes
+    alg = bench.prefill_alg_bytes(w, 1024)
+    assert alg == 32 * 404_750_336 + 32000 * 4096 * 2 + 32 * 16_384 * 2 * 1024
+    r = bench.prefill_roofline(expect, alg, 72.0, pk, traffic=bench.prefill_bytes(w, 1024, 128))
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+    assert r["frac"] == pytest.approx(expect / 0.072 / 1e12 / 1884.7)
+    assert r["traffic_model"] == 106_831_020_032
+    # a short prompt is bound by its bytes
+    r = bench.prefill_roofline(bench.prefill_flops(w, 16), bench.prefill_alg_bytes(w, 16), 5.0, pk)
+    assert r["bound"] == "hbm"

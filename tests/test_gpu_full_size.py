@@ -8,9 +8,11 @@ size:
 
 * losslessness (Sec. 3.3): the committed DVI stream equals the GPU's own
   greedy autoregressive stream bit for bit, with the drafter training online;
-* teacher-forced verifier logits of the first step's verify rows against the
-  oracle (float32 arithmetic on the bf16-rounded weights, bf16 KV cache),
-  within 3e-2 (1B and 7B);
+* teacher-forced verifier logits of every logged verify row of an 8-step
+  run with the drafter training, against the oracle (float32 arithmetic on
+  the bf16-rounded weights, bf16 KV cache; float32 keeps the 7B oracle
+  within minutes, and its rounding is far below the bound), within 3e-2,
+  with y* the row's argmax (1B and 7B);
 * the 8-sequence ragged batch over two prompt waves whose drafter state
   carries over, and the 16K-token prompt with K = 8;
 * one LoRA update at the 7B shape: dA, dB against the oracle's closed-form
@@ -24,7 +26,7 @@ import torch
 
 from oracle import OracleModel
 from workloads import workload, make_weights, make_prompts
-from gpu_helpers import rounded_weights, teacher_forced_logits
+from gpu_helpers import rounded_weights, run_logged_steps, check_rows_against_oracle
 
 pytestmark = pytest.mark.gpu
 GEN = 24
@@ -65,24 +67,16 @@ def _lossless(w, dw, P, n_gen=GEN):
     return toks, mats
 
 
-def _first_step_logits(w, dw, W, P):
-    """Verify-row logits of the first decode step: GPU log against the oracle."""
+def _every_step_logits(w, dw, W, P, n_steps=8):
+    """Verify-row logits of every step of an 8-step run: GPU log against the oracle."""
     eng = _engine(w, dw, _capacity(w, P))
-    toks, _, _, _ = eng.generate(P, 10 ** 6, max_steps=1, log=True)
-    eng.sync()
-    meta = eng.buffer("LOG_META", torch.int32).view(-1, 6).cpu().numpy()
-    lg = eng.buffer("LOG_LOGITS", torch.float32).view(-1, w.shape.vocab).cpu().numpy()
+    toks, rows = run_logged_steps(eng, P, n_steps, update_every=w.update_every, hyper=w.update)
+    st = eng.stats()
     eng.close()
-    rows = [i for i in range(w.k_spec) if meta[i, 0]]
-    assert rows and rows == list(range(len(rows)))
+    assert st["device_status"] == 0, st["device_flags"]
+    assert len(rows) >= n_steps
     model = OracleModel(rounded_weights(W), w.shape, w.lora_gamma, dtype=np.float32, kv_dtype="bf16")
-    seq = np.concatenate([P[0], np.array(toks[0][:len(rows)], dtype=np.int32)])
-    ref = teacher_forced_logits(model, seq)
-    n0 = len(P[0])
-    for i in rows:
-        err = np.abs(lg[i] - ref[n0 + i]).max()
-        assert err < 3e-2, (i, err)
-        assert int(np.argmax(lg[i])) == int(meta[i, 5])
+    check_rows_against_oracle(model, P, toks, rows, 3e-2)
 
 
 def test_1b_gqa_lossless_and_teacher_forced():
@@ -90,7 +84,7 @@ def test_1b_gqa_lossless_and_teacher_forced():
     W, dw = _weights("1b")
     P = make_prompts(w)
     _lossless(w, dw, P)
-    _first_step_logits(w, dw, W, P)
+    _every_step_logits(w, dw, W, P)
 
 
 def test_7b_lossless_and_teacher_forced():
@@ -98,7 +92,7 @@ def test_7b_lossless_and_teacher_forced():
     W, dw = _weights("7b")
     P = make_prompts(w)
     _lossless(w, dw, P)
-    _first_step_logits(w, dw, W, P)
+    _every_step_logits(w, dw, W, P)
 
 
 def test_7b_batch8_ragged_two_waves():

@@ -115,3 +115,51 @@ def test_misaligned_vectors_rejected(L, field):
     rc = L.dvi_create(ctypes.byref(cfg), ctypes.byref(rt), ctypes.byref(w), ctypes.c_void_p(1 << 20), 1 << 30,
                       None, ctypes.byref(ctx))
     assert rc == -1 and not ctx.value
+
+
+class _FakeTensor:
+    """Stands in for a CUDA tensor in the host-side argument checks (no GPU here)."""
+
+    def __init__(self, shape, dtype, device="cuda:0", contiguous=True, cuda=True):
+        import torch
+        self.shape, self.dtype = tuple(shape), dtype
+        self.device = torch.device(device) if cuda else torch.device("cpu")
+        self.is_cuda, self._c = cuda, contiguous
+
+    def is_contiguous(self):
+        return self._c
+
+
+def _noalloc_args(**over):
+    import torch
+    a = dict(w=_FakeTensor((64, 32), torch.bfloat16), x=_FakeTensor((5, 32), torch.float32),
+             y=_FakeTensor((5, 64), torch.float32))
+    a.update(over)
+    return a
+
+
+def test_noalloc_args_accepted():
+    D.check_linear_noalloc_args(**_noalloc_args())
+
+
+@pytest.mark.parametrize("case", ["x_bf16", "w_f16", "x_short", "y_shape", "rows", "noncontig", "cpu", "devices"])
+def test_noalloc_args_rejected_before_any_launch(monkeypatch, case):
+    """Every malformed call raises ValueError in the binding, before the
+    library is loaded or a pointer reaches the kernel."""
+    import torch
+    over = {
+        "x_bf16": dict(x=_FakeTensor((5, 32), torch.bfloat16)),
+        "w_f16": dict(w=_FakeTensor((64, 32), torch.float16)),
+        "x_short": dict(x=_FakeTensor((5, 16), torch.float32)),
+        "y_shape": dict(y=_FakeTensor((5, 32), torch.float32)),
+        "rows": dict(x=_FakeTensor((300, 32), torch.float32), y=_FakeTensor((300, 64), torch.float32)),
+        "noncontig": dict(y=_FakeTensor((5, 64), torch.float32, contiguous=False)),
+        "cpu": dict(x=_FakeTensor((5, 32), torch.float32, cuda=False)),
+        "devices": dict(y=_FakeTensor((5, 64), torch.float32, device="cuda:1")),
+    }[case]
+
+    def no_lib():
+        raise AssertionError("the library was reached")
+    monkeypatch.setattr(D, "lib", no_lib)
+    with pytest.raises(ValueError):
+        D.linear_noalloc(**_noalloc_args(**over))

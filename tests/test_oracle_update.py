@@ -173,6 +173,29 @@ def test_adam_first_steps_move_by_lr_sign():
     np.testing.assert_allclose(p, -0.02 * np.sign(g), rtol=1e-8)
 
 
+def test_adam_two_steps_hand_computed():
+    """Two bias-corrected Adam steps with a changing gradient and an epsilon
+    large enough to matter (lr 0.01, betas 0.9 / 0.999, eps 1e-3, p0 = 1):
+
+    step 1, g = 2e-3:  m = 0.1 g = 2e-4, v = 0.001 g^2 = 4e-9,
+      m^ = m / 0.1 = 2e-3, v^ = v / 0.001 = 4e-6, sqrt(v^) = 2e-3,
+      p = 1 - 0.01 * 2e-3 / (2e-3 + 1e-3) = 1 - 0.02/3
+    step 2, g = -1e-3: m = 0.9 * 2e-4 - 1e-4 = 8e-5,
+      v = 0.999 * 4e-9 + 0.001 * 1e-6 = 4.996e-9,
+      m^ = 8e-5 / 0.19 = 4.2105263157894737e-4,
+      v^ = 4.996e-9 / 0.001999 = 2.4992496248124062e-6, sqrt(v^) = 1.5809015228066567e-3,
+      p = p1 - 0.01 * m^ / (sqrt(v^) + 1e-3) = p1 - 1.6314168822724575e-3
+    (worked by hand in decimal arithmetic).  Epsilon under the square root
+    would give p1 = 0.99936880..., no bias correction p1 = 0.99811897..."""
+    p = np.array([1.0])
+    st = AdamState(np.zeros(1), np.zeros(1))
+    adam_step(p, np.array([2e-3]), st, 0.01, 0.9, 0.999, 1e-3)
+    assert p[0] == pytest.approx(0.99333333333333333, rel=1e-14)
+    adam_step(p, np.array([-1e-3]), st, 0.01, 0.9, 0.999, 1e-3)
+    assert p[0] == pytest.approx(0.99170191645106088, rel=1e-14)
+    assert st.m[0] == pytest.approx(8e-5, rel=1e-12) and st.v[0] == pytest.approx(4.996e-9, rel=1e-12)
+
+
 def _tuples(seed, n=6, d=32, V=64):
     g = np.random.default_rng(seed)
     return [LoggedTuple(seq=0, u=g.standard_normal(d), a=int(g.integers(V)),
