@@ -825,6 +825,246 @@ static size_t attn_smem(int hd) {
   return sizeof(float) * (kAttnQ * hd + kAttnBlk * (hd + 1) + kAttnBlk * hd + kAttnQ * kAttnBlk + 3 * kAttnQ) + 16;
 }
 
+// ------------------------------------------------------------------ prefill, bf16
+// Prompt passes have many query rows per (sequence, KV head).  A CTA takes
+// 64 query vectors -- four warps of 16 (pass rows x the GQA heads of one KV
+// head) -- and walks every 64-position chunk of the cache its rows can see,
+// double-buffered by TMA; the four warps share each chunk, so the cache is
+// streamed once per 64 query vectors.  Per warp and 32-position half chunk:
+// S = Q K^T with the query as a bf16 pair hi + lo (two MMA chains), the
+// causal mask (a position is seen by rows at or after it), an online softmax
+// in base 2, then O += P V with P as a bf16 pair.  There is no position
+// split and no merge: a row's result is its own online softmax over chunks
+// 0 .. p/64 in order (a chunk wholly past the row leaves its state exactly
+// as it was), whichever rows share the CTA or the pass.
+constexpr int kPfWarpQ = 16;   // query vectors per warp (the mma M)
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_pf_kernel(const __grid_constant__ CUtensorMap mk,
+                                                      const __grid_constant__ CUtensorMap mv, const AttnArgs a) {
+  constexpr int kBoxes = HD / 64;                    // 64-dim TMA boxes per row
+  constexpr int kBoxBytes = 64 * 128;                // 64 positions x 128 B
+  constexpr int kStage = 2 * kBoxes * kBoxBytes;     // K boxes, then V boxes
+  constexpr int kNT = HD / 8;                        // O n-tiles
+  extern __shared__ __align__(1024) uint8_t dsm_raw[];
+  __shared__ __align__(8) uint64_t full[kDecStages];
+  __shared__ int abort_flag;
+  const uint32_t raw = smem_u32(dsm_raw);
+  uint8_t* ring = dsm_raw + (((raw + 1023u) & ~1023u) - raw);
+  griddep_launch();
+  griddep_wait();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int gq = lane >> 2, tq = lane & 3;           // mma fragment coordinates
+  const int G = a.n_heads / a.n_kv_heads;
+  const int RW = kPfWarpQ / G;                       // pass rows per warp
+  const int RC = 4 * RW;                             // pass rows per CTA
+  const int g = blockIdx.x;
+  const int n_grp = (a.rows_per_seq + RC - 1) / RC;
+  const int grp = n_grp - 1 - static_cast<int>(blockIdx.y);   // longest prefixes first
+  const int sl = blockIdx.z, seq = a.seq0 + sl;
+  const int base = a.lens[seq] + a.pos_off;          // position of pass row 0
+  const int i0 = grp * RC;
+  const int nrows = min(RC, a.rows_per_seq - i0);
+  const int p_max = min(base + i0 + nrows - 1, a.max_len - 1);
+  const int nch = p_max / kChunkPos + 1;
+  // chunks this warp's rows can see (0 if it has no row)
+  const int wr = min(RW, nrows - warp * RW);
+  const int w_nch = wr > 0 ? min(base + i0 + warp * RW + wr - 1, a.max_len - 1) / kChunkPos + 1 : 0;
+  const int row0 = static_cast<int>(a.kv_row0 + (static_cast<long long>(seq) * a.n_kv_heads + g) * a.max_len);
+
+  auto issue = [&](int ch) {
+    const int st = ch % kDecStages;
+    const int y = row0 + ch * kChunkPos;
+    mbar_arrive_expect_tx(&full[st], kStage);
+    for (int b = 0; b < kBoxes; ++b) {
+      tma_load_2d(ring + st * kStage + b * kBoxBytes, &mk, b * 64, y, &full[st], 0ull);
+      tma_load_2d(ring + st * kStage + (kBoxes + b) * kBoxBytes, &mv, b * 64, y, &full[st], 0ull);
+    }
+  };
+  if (tid == 0) {
+    for (int st = 0; st < kDecStages; ++st) mbar_init(&full[st], 1);
+    mbar_fence_init();
+    tma_prefetch_desc(&mk);
+    tma_prefetch_desc(&mv);
+    abort_flag = 0;
+  }
+  __syncthreads();
+  if (tid == 0)
+    for (int ch = 0; ch < min(kDecStages, nch); ++ch) issue(ch);
+
+  // Q fragments of rows gq and gq+8 of this warp, scaled by 1/sqrt(hd) *
+  // log2(e), as a bf16 pair hi + lo
+  uint32_t qa[HD / 16][4], qb[HD / 16][4];
+  int lim0 = -1, lim1 = -1;
+  {
+    const float sc = a.scale * kLog2e;
+    const float* qrow[2] = {nullptr, nullptr};
+    for (int h = 0; h < 2; ++h) {
+      const int v = warp * kPfWarpQ + gq + 8 * h;
+      const int ii = v / G, hh = v % G;
+      if (ii < nrows) {
+        const int n = sl * a.rows_per_seq + i0 + ii;
+        qrow[h] = a.q + static_cast<size_t>(n) * a.ld_q + (g * G + hh) * HD;
+        if (h == 0) lim0 = base + i0 + ii;
+        else lim1 = base + i0 + ii;
+      }
+    }
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const float* qr = qrow[r & 1];
+        const int col = kk * 16 + (r >> 1) * 8 + 2 * tq;
+        qa[kk][r] = 0u;
+        qb[kk][r] = 0u;
+        if (qr) {
+          const float2 v = *reinterpret_cast<const float2*>(qr + col);
+          split_bf16x2(v.x * sc, v.y * sc, qa[kk][r], qb[kk][r]);
+        }
+      }
+    }
+  }
+  float o[kNT][4];
+#pragma unroll
+  for (int nt = 0; nt < kNT; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o[nt][e] = 0.f;
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+
+  int ch = 0;
+  for (; ch < nch; ++ch) {
+    const int st = ch % kDecStages;
+    if (!mbar_wait(&full[st], (ch / kDecStages) & 1, a.status)) abort_flag = 1;
+    const uint8_t* ks = ring + st * kStage;
+    const uint8_t* vs = ks + kBoxes * kBoxBytes;
+    if (ch < w_nch) {
+#pragma unroll 1
+      for (int hb = 0; hb < 2; ++hb) {
+        const int pc = ch * kChunkPos + hb * 32;
+        // S = Q K^T for 32 positions (four n-tiles of 8)
+        float sacc[4][4], slo[4][4];
+#pragma unroll
+        for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) sacc[nt][e] = slo[nt][e] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const int box = (kk * 16) / 64, c = ((kk * 16) % 64) / 8;
+#pragma unroll
+          for (int nt = 0; nt < 4; ++nt) {
+            const int pr = hb * 32 + nt * 8 + gq;                 // row of the chunk
+            const uint8_t* rowp = ks + box * kBoxBytes + pr * 128;
+            const uint32_t b0 = *reinterpret_cast<const uint32_t*>(rowp + ((c ^ (pr & 7)) << 4) + 4 * tq);
+            const uint32_t b1 = *reinterpret_cast<const uint32_t*>(rowp + (((c + 1) ^ (pr & 7)) << 4) + 4 * tq);
+            mma_bf16_16816(sacc[nt], qa[kk], b0, b1);
+            mma_bf16_16816(slo[nt], qb[kk], b0, b1);
+          }
+        }
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int pos = pc + nt * 8 + 2 * tq + e;
+            sacc[nt][e] = pos <= lim0 ? sacc[nt][e] + slo[nt][e] : -INFINITY;
+            sacc[nt][2 + e] = pos <= lim1 ? sacc[nt][2 + e] + slo[nt][2 + e] : -INFINITY;
+            mx0 = fmaxf(mx0, sacc[nt][e]);
+            mx1 = fmaxf(mx1, sacc[nt][2 + e]);
+          }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        // a row with nothing visible so far keeps its state untouched
+        const float c0 = (mn0 == -INFINITY) ? 1.f : (m0 == -INFINITY ? 0.f : exp2f(m0 - mn0));
+        const float c1 = (mn1 == -INFINITY) ? 1.f : (m1 == -INFINITY ? 0.f : exp2f(m1 - mn1));
+        uint32_t pa[2][4], pb[2][4];   // P as a bf16 pair hi + lo, per 16-position k-step
+        float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+        for (int k2 = 0; k2 < 2; ++k2) {
+          float pv[2][4];
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const float* sv = sacc[2 * k2 + h2];
+              pv[h2][e] = (sv[e] == -INFINITY) ? 0.f : exp2f(sv[e] - mn0);
+              pv[h2][2 + e] = (sv[2 + e] == -INFINITY) ? 0.f : exp2f(sv[2 + e] - mn1);
+            }
+          s0 += (pv[0][0] + pv[0][1]) + (pv[1][0] + pv[1][1]);
+          s1 += (pv[0][2] + pv[0][3]) + (pv[1][2] + pv[1][3]);
+          split_bf16x2(pv[0][0], pv[0][1], pa[k2][0], pb[k2][0]);
+          split_bf16x2(pv[0][2], pv[0][3], pa[k2][1], pb[k2][1]);
+          split_bf16x2(pv[1][0], pv[1][1], pa[k2][2], pb[k2][2]);
+          split_bf16x2(pv[1][2], pv[1][3], pa[k2][3], pb[k2][3]);
+        }
+        l0 = l0 * c0 + s0;
+        l1 = l1 * c1 + s1;
+        m0 = mn0;
+        m1 = mn1;
+#pragma unroll
+        for (int nt = 0; nt < kNT; ++nt) {
+          o[nt][0] *= c0;
+          o[nt][1] *= c0;
+          o[nt][2] *= c1;
+          o[nt][3] *= c1;
+        }
+        // O += P V over the 32 positions, V read transposed
+#pragma unroll
+        for (int k2 = 0; k2 < 2; ++k2) {
+#pragma unroll
+          for (int nt = 0; nt < kNT; nt += 2) {
+            const int mi = lane >> 3, rr = lane & 7;
+            const int pr = hb * 32 + k2 * 16 + (mi & 1) * 8 + rr;
+            const int db = nt + (mi >> 1);                          // 8-dim block
+            const int box = db / 8, c = db % 8;
+            const uint32_t addr = smem_u32(vs + box * kBoxBytes + pr * 128 + ((c ^ (pr & 7)) << 4));
+            uint32_t r[4];
+            ldmatrix_x4_trans(r, addr);
+            mma_bf16_16816(o[nt], pa[k2], r[0], r[1]);
+            mma_bf16_16816(o[nt], pb[k2], r[0], r[1]);
+            mma_bf16_16816(o[nt + 1], pa[k2], r[2], r[3]);
+            mma_bf16_16816(o[nt + 1], pb[k2], r[2], r[3]);
+          }
+        }
+      }
+    }
+    __syncthreads();                      // stage `st` consumed by every warp
+    if (abort_flag) break;
+    if (tid == 0 && ch + kDecStages < nch) issue(ch + kDecStages);
+  }
+  if (abort_flag) {
+    // a wait gave up at chunk ch: the copies issued from there on (chunks
+    // ch .. ch + kDecStages - 1) must land, or time out, before the CTA exits
+    if (tid == 0)
+      for (int c = ch; c < min(nch, ch + kDecStages); ++c)
+        mbar_wait(&full[c % kDecStages], (c / kDecStages) & 1, a.status);
+    return;
+  }
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  __nv_bfloat16* out = static_cast<__nv_bfloat16*>(a.o);
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int v = warp * kPfWarpQ + gq + 8 * h;
+    const int ii = v / G, hh = v % G;
+    if (ii >= nrows) continue;
+    const float inv = 1.f / (h == 0 ? l0 : l1);
+    const size_t row = static_cast<size_t>(sl * a.rows_per_seq + i0 + ii) * a.ld_o + (g * G + hh) * HD;
+#pragma unroll
+    for (int nt = 0; nt < kNT; ++nt) {
+      const int d = nt * 8 + 2 * tq;
+      uint32_t hi, lo;
+      split_bf16x2(o[nt][2 * h] * inv, o[nt][2 * h + 1] * inv, hi, lo);
+      *reinterpret_cast<uint32_t*>(out + row + d) = hi;
+      *reinterpret_cast<uint32_t*>(out + row + d + a.o_plane) = lo;
+    }
+  }
+}
+
 static int n_qgroups(const AttnArgs& a, bool bf16) {
   const int RQ = rows_per_group(a.rows_per_seq, a.n_heads / a.n_kv_heads, bf16);
   return (a.rows_per_seq + RQ - 1) / RQ;
@@ -840,6 +1080,19 @@ template <typename T>
 static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
   const bool bf16 = sizeof(T) == 2;
   dim3 grid(a.n_splits_max, a.n_kv_heads, a.n_seqs * n_qgroups(a, bf16));
+  if (bf16 && a.prefill && a.n_heads / a.n_kv_heads <= kRegQ) {
+    const int G = a.n_heads / a.n_kv_heads;
+    const int rc = 4 * (kPfWarpQ / G);
+    const dim3 pgrid(a.n_kv_heads, (a.rows_per_seq + rc - 1) / rc, a.n_seqs);
+    const size_t smem = 1024 + static_cast<size_t>(kDecStages) * 2 * kChunkPos * a.head_dim * 2;
+    static PerDevice pf_attr;
+    pf_attr.once([] {
+      cudaFuncSetAttribute(attn_pf_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+      cudaFuncSetAttribute(attn_pf_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+    });
+    if (a.head_dim == 128) return launch_pdl(attn_pf_kernel<128>, pgrid, dim3(128), smem, s, *a.kmap, *a.vmap, a);
+    return launch_pdl(attn_pf_kernel<64>, pgrid, dim3(128), smem, s, *a.kmap, *a.vmap, a);
+  }
   if (bf16 && a.n_heads / a.n_kv_heads <= kRegQ) {
     // one cluster of n_splits_max (<= 8) CTAs per (sequence, query group, KV
     // head); decode and prefill chunks alike (16 / G query rows per group)

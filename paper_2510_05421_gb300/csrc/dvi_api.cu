@@ -480,7 +480,10 @@ AttnArgs attn_args(dvi_ctx* ctx, int l, const Pass& ps) {
   t.pos_off = ps.pos_off;
   const bool dec_cluster = ctx->tc && ctx->Hq / ctx->Hkv <= 8;   // the tensor-core kernel
   t.split_len = dec_cluster ? 0 : ctx->attn_split_len;
-  t.n_splits_max = dec_cluster ? ctx->dec_nsplits : ctx->attn_nsplits;
+  // a prompt pass has query rows enough to fill the GPU without splitting
+  // the positions: one CTA walks its rows' whole prefix
+  t.n_splits_max = dec_cluster ? (ps.pf ? 1 : ctx->dec_nsplits) : ctx->attn_nsplits;
+  t.prefill = ps.pf && dec_cluster ? 1 : 0;
   t.part = ctx->attn_part;
   t.counters = ctx->attn_ctr;
   t.status = ctx->status;

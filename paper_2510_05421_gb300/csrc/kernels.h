@@ -145,6 +145,7 @@ struct AttnArgs {
   long long kv_row0;                 // bf16 decode: row of (layer, seq 0, head 0, pos 0) in the cache maps
   const CUtensorMap* kmap;           // bf16 decode: the K / V caches as [rows][hd] (box 64 x 64)
   const CUtensorMap* vmap;
+  int prefill;                       // a prompt pass (bf16, GQA group <= 8): the prefill attention kernel
 };
 bool make_kv_map(CUtensorMap* map, const void* cache, long long rows, int hd);
 size_t attn_partial_floats(const AttnArgs& a);
