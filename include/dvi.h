@@ -246,7 +246,9 @@ enum {
   DVI_BUF_V_CACHE = 11,
   DVI_BUF_STATUS = 12,     /* int32 device status word */
   DVI_BUF_GRAD_W = 13,     /* f32 [V][d] last dL/dW^(S) (head_mode 1, written when keep_grad_w) */
-  DVI_BUF_Z = 14,          /* f32 [cap][V] drafter logits of the last update */
+  DVI_BUF_Z = 14,          /* f32 [cap][V] drafter logits z of the buffer rows: logged by the drafter
+                              head while drafting (head_mode 0; A, B and W^(S) change only at an
+                              update, which empties the buffer), else recomputed by the update */
   DVI_BUF_COUNT
 };
 dvi_status dvi_debug_buffer(dvi_ctx* ctx, int which, void** dptr, size_t* bytes);

@@ -68,6 +68,7 @@ struct dvi_ctx {
   int *lens, *pending, *draft_ids, *status, *log_step, *log_meta;
   long long* counters;
   float* dev_state;
+  int* upd_ctr;   // [4 + cap_rows] the update kernels' counters and grid barrier
   float *x_dr, *ss_dr, *x_ver, *ss_ver, *x_pf, *ss_pf, *q, *bu;
   void *xg_dr, *xg_ver, *xg_pf, *attn_o, *ffn_h;
   unsigned long long* amax;
@@ -89,7 +90,7 @@ struct dvi_ctx {
   int* chain_ctr = nullptr;
   void* log_u;
   float* log_logits;
-  float *Z, *rowstat, *coef, *ub, *ga, *ga_part;
+  float *Z, *rowstat, *stat_part, *coef, *ub, *ga, *ga_part;
   float *m_a, *v_a, *m_b, *v_b, *grad_a, *grad_b;
   // full-head mode (head_mode 1): f32 master of W^S (bf16 only), Adam
   // moments, per-row logit gradients G, the optional gradient copy
@@ -188,6 +189,7 @@ size_t layout(dvi_ctx* c, char* base) {
   c->log_meta = reinterpret_cast<int*>(take(sizeof(int) * 6 * c->cap_rows));
   c->counters = reinterpret_cast<long long*>(take(sizeof(long long) * 8));
   c->dev_state = reinterpret_cast<float*>(take(sizeof(float) * 16));
+  c->upd_ctr = reinterpret_cast<int*>(take(sizeof(int) * (4 + c->cap_rows)));
   c->x_dr = reinterpret_cast<float*>(take(sizeof(float) * B * d));
   c->ss_dr = reinterpret_cast<float*>(take(sizeof(float) * st * B));
   c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * c->Kv * d));
@@ -218,11 +220,14 @@ size_t layout(dvi_ctx* c, char* base) {
   c->log_logits = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
   c->Z = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(c->cap_rows) * V));
   c->rowstat = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * 8));
+  c->stat_part = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * ((V + 2047) / 2048) * 9));
   c->coef = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * 8));
   const int rr = r > 0 ? r : 1;
   c->ub = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * rr));
   c->ga = reinterpret_cast<float*>(take(sizeof(float) * c->cap_rows * rr));
-  const int nvt = (V + 127) / 128;
+  // partials of G A: one per 128-entry vocabulary tile (separate kernels) or
+  // one per CTA of the fused update (at most 256)
+  const int nvt = std::max((V + 127) / 128, 256);
   c->ga_part = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(nvt) * c->cap_rows * rr));
   c->m_a = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(V) * rr));
   c->v_a = reinterpret_cast<float*>(take(sizeof(float) * static_cast<size_t>(V) * rr));
@@ -723,7 +728,8 @@ StepState step_state(dvi_ctx* c) {
 // With `bu_inline` (bf16 drafter head) the kernel computes B u itself from
 // the draft residual rows instead of reading it from `bu`.
 dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, const void* act,
-                        const CUtensorMap* act_map, int row0, const float* ss, int ss_ld, bool bu_inline = false) {
+                        const CUtensorMap* act_map, int row0, const float* ss, int ss_ld, bool bu_inline = false,
+                        int draft_pass = 0) {
   Pass ps{nullptr, nullptr, 0, rows, 1, 0, 1, 0, nullptr, nullptr};
   ProjArgs a = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
   a.act = act;
@@ -749,13 +755,23 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
   }
   if (logits_mode == 2) {
     a.logits_mode = 2;
-    a.logits_out = ctx->log_logits;
     a.ld_logits = ctx->V;
     a.log_step = ctx->log_step;
     a.log_cap_steps = ctx->cap_steps;
     a.log_rows_per_step = ctx->B * ctx->K;
-    a.log_src_rows = ctx->Kv;   // verify rows per sequence; the log keeps the first K
-    a.log_dst_rows = ctx->K;
+    if (draft) {
+      // the drafter's logits of pass j are z of tuple j + 1: the update
+      // reads them instead of recomputing them (A, B and W^S only change at
+      // an update, which empties the buffer)
+      a.logits_out = ctx->Z;
+      a.log_src_rows = 1;         // one row per sequence; slot b * K + j
+      a.log_dst_rows = ctx->K;
+      a.log_dst_off = draft_pass;
+    } else {
+      a.logits_out = ctx->log_logits;
+      a.log_src_rows = ctx->Kv;   // verify rows per sequence; the log keeps the first K
+      a.log_dst_rows = ctx->K;
+    }
   }
   ProjMaps pm{};
   if (ctx->tc) pm = with_act(draft ? ctx->head_s : ctx->head_v, act_map);
@@ -819,7 +835,8 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
       ctx->launches += 1;
     }
     if (!drafts) continue;
-    if ((rc = enqueue_head(ctx, true, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B, fused)) !=
+    const int zlog = ctx->log_enabled && ctx->rt.head_mode == 0 ? 2 : 0;   // the drafter's logits of the tuple
+    if ((rc = enqueue_head(ctx, true, ctx->B, zlog, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B, fused, j)) !=
         DVI_OK)
       return rc;
     DVI_CUDA(launch_finalize_draft(st, j, fused ? &h : nullptr, s));
@@ -1125,6 +1142,7 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   a.log_step = ctx->log_step;
   a.Z = ctx->Z;
   a.rowstat = ctx->rowstat;
+  a.stat_part = ctx->stat_part;
   a.coef = ctx->coef;
   a.ub = ctx->ub;
   a.ga = ctx->ga;
@@ -1147,10 +1165,18 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   a.grad_w = ctx->grad_w;
   a.keep_grad_w = u->keep_grad_w ? 1 : 0;
   a.dev_state = ctx->dev_state;
+  a.ctr = ctx->upd_ctr;
   a.counters = ctx->counters;
   a.status = ctx->status;
   a.cfg = *u;
   cudaEvent_t t0 = mark_begin(ctx);
+  if (!full && update_fused_ok(a, ctx->n_sms)) {
+    // one cooperative launch: the drafter logits were logged while drafting
+    DVI_CUDA(launch_update_fused(a, ctx->n_sms, s));
+    ctx->launches += 1;
+    mark_end(ctx, 2, t0);
+    return DVI_OK;
+  }
   DVI_CUDA(launch_update_prep(a, s));
   // drafter logits of every buffer row: Z = U W^S^T + gamma (U B^T) A^T
   Pass ps{nullptr, nullptr, 0, ctx->cap_rows, 1, 0, 1, 0, nullptr, nullptr};
@@ -1170,17 +1196,19 @@ dvi_status dvi_update_drafter(dvi_ctx* ctx, const dvi_update_config* u) {
   ProjMaps pm{};
   if (ctx->tc) pm = with_act(ctx->head_s, &ctx->map_log_u);
   DVI_CUDA(launch_proj_ctx(ctx, p, ctx->tc ? &pm : nullptr, s));
+  // row statistics; the last row's CTA forms the loss and the coefficients
   DVI_CUDA(launch_update_rowstats(a, s));
-  DVI_CUDA(launch_update_coef(a, s));
   if (full) {
     DVI_CUDA(launch_update_full(a, s));
-    ctx->launches += (ctx->r > 0 ? 1 : 0) + 6;
+    DVI_CUDA(launch_update_finish(a, s));
+    ctx->launches += (ctx->r > 0 ? 1 : 0) + 5;
   } else {
+    // dA with Adam on A, the G A reduction, then dB with Adam on B; the last
+    // grad_b CTA ends the update
     DVI_CUDA(launch_update_grad_a(a, s));
     DVI_CUDA(launch_update_grad_b(a, s));
-    ctx->launches += 8;
+    ctx->launches += 6;
   }
-  DVI_CUDA(launch_update_finish(a, s));
   mark_end(ctx, 2, t0);
   return DVI_OK;
 }

@@ -66,7 +66,10 @@ struct ProjArgs {
   float* logits_out; int ld_logits;
   int logits_mode;            // 0 none, 1 row n -> logits_out[n], 2 replay-buffer slot
   const int* log_step; int log_cap_steps; int log_rows_per_step;
-  int log_src_rows, log_dst_rows;   // mode 2: launch rows per sequence, of which the log keeps the first
+  // mode 2: of each sequence's log_src_rows launch rows the log keeps the
+  // first min(log_src_rows, log_dst_rows), at slots b * log_dst_rows +
+  // log_dst_off + i of the step's rows
+  int log_src_rows, log_dst_rows, log_dst_off;
   const float* lora_a; const float* lora_bu; int lora_r; float gamma;
   // bf16 drafter head, M <= kBuRows and lora_r <= kBuRank: B u computed by
   // the kernel itself (lora_bu unused), u = (x * rstd) * g from the f32
@@ -210,6 +213,7 @@ struct UpdateArgs {
   const void* log_u; size_t log_plane; const float* log_logits; int* log_meta; int* log_step;
   float* Z;                                     // [cap][V] drafter logits
   float* rowstat;                               // [cap][8]
+  float* stat_part;                             // [cap][ceil(V / 2048)][9] merged parts of the row statistics
   float* coef;                                  // [cap][4] + globals
   float* ub;                                    // [cap][r]  U B^T
   float* ga;                                    // [cap][r]  G A
@@ -221,16 +225,21 @@ struct UpdateArgs {
   // Adam moments, G [cap][V], the optional gradient copy
   void* w_head; float* w_master; float* m_w; float* v_w; float* G; float* grad_w; int keep_grad_w;
   float* dev_state;                             // [0]=t, [1]=b, [2..] loss parts
+  int* ctr;                                     // [4 + cap] last-CTA counters (rows done, update end, per
+                                                // row; 0 between updates), grid barrier (count, generation)
   long long* counters;
   int* status;
   dvi_update_config cfg;
 };
 cudaError_t launch_update_prep(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_rowstats(const UpdateArgs& a, cudaStream_t s);
-cudaError_t launch_update_coef(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_full(const UpdateArgs& a, cudaStream_t s);
+// LoRA mode: everything after the logits GEMM in one cooperative launch of
+// n_sms CTAs (grid barriers between its phases), when update_fused_ok.
+bool update_fused_ok(const UpdateArgs& a, int n_sms);
+cudaError_t launch_update_fused(const UpdateArgs& a, int n_sms, cudaStream_t s);
 cudaError_t launch_master_init(const void* w_bf16, float* master, size_t n, cudaStream_t s);
 cudaError_t launch_update_finish(const UpdateArgs& a, cudaStream_t s);
 

@@ -215,31 +215,67 @@ __device__ void embed_rows(const StepState& st, const int* toks, float* red) {
                        st.ss_dr_ld, b, red);
 }
 
+// 16-byte asynchronous copy global -> shared (completes at cp_async_wait).
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_all;" ::: "memory");
+}
+
 // With `prep` set, the drafter-head preparation of the pass (the logged u
 // and the hand-off of h_k to the verify rows; the head computed B u itself)
 // runs here, for every row before its residual is overwritten by the next
-// pass's embedding.
+// pass's embedding.  The drafted tokens are read first; with `stage` set the
+// next pass's embedding rows are copied into shared memory asynchronously
+// while the preparation runs, so their load is off the critical path.
 template <typename T>
 __global__ void __launch_bounds__(128) finalize_draft_kernel(const StepState st, int j, const HeadPrepArgs hp,
-                                                             int prep) {
+                                                             int prep, int stage) {
   __shared__ int tok_s[64];
   __shared__ float red[kMaxTiles * 4];
   __shared__ float rstd_s;
+  extern __shared__ __align__(16) uint8_t emb_raw[];
   griddep_launch();
   griddep_wait();
-  if (prep) {
-    for (int b = 0; b < hp.rows; ++b) {
-      prep_row<T>(hp, b, true, red, &rstd_s, nullptr);
-      __syncthreads();
-    }
-  }
   for (int b = threadIdx.x; b < st.B; b += blockDim.x) {
     const int t = take_argmax(st.amax + b, st.status);
     st.draft_ids[b * (st.K + 1) + j + 1] = t;
     tok_s[b] = t;
   }
   __syncthreads();
-  if (j + 1 < st.Kv) embed_rows<T>(st, tok_s, red);   // the next pass's token (t~_K feeds the bonus row)
+  const bool next = j + 1 < st.Kv;   // the next pass's token (t~_K feeds the bonus row)
+  T* emb_s = reinterpret_cast<T*>(emb_raw);
+  if (next && stage) {
+    const int per_row = st.d * static_cast<int>(sizeof(T)) / 16;
+    for (int i = threadIdx.x; i < st.B * per_row; i += blockDim.x) {
+      const int b = i / per_row, c = i % per_row;
+      int tok = tok_s[b];
+      if (tok < 0 || tok >= st.vocab) tok = 0;   // flagged by the embedding below
+      cp_async16(emb_raw + static_cast<size_t>(i) * 16,
+                 reinterpret_cast<const uint8_t*>(static_cast<const T*>(st.embed) + static_cast<size_t>(tok) * st.d) +
+                     static_cast<size_t>(c) * 16);
+    }
+  }
+  if (prep) {
+    for (int b = 0; b < hp.rows; ++b) {
+      prep_row<T>(hp, b, true, red, &rstd_s, nullptr);
+      __syncthreads();
+    }
+  }
+  if (!next) return;
+  if (!stage) {
+    embed_rows<T>(st, tok_s, red);
+    return;
+  }
+  cp_async_wait();
+  __syncthreads();
+  for (int b = 0; b < st.B; ++b) {
+    if (threadIdx.x == 0 && (tok_s[b] < 0 || tok_s[b] >= st.vocab)) flag_status(st.status, DVI_DEV_BAD_TOKEN);
+    embed_row_block<T>(emb_s + static_cast<size_t>(b) * st.d, 0, st.d, st.x_dr + static_cast<size_t>(b) * st.d,
+                       st.g0, static_cast<T*>(st.xg_dr) + static_cast<size_t>(b) * st.d, st.xg_dr_plane, st.ss_dr,
+                       st.ss_dr_ld, b, red);
+  }
 }
 
 template <typename T>
@@ -347,12 +383,28 @@ static cudaError_t launch1(K kern, cudaStream_t s, Args... args) {
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+constexpr size_t kStageMax = 64 * 1024;   // shared memory for staged embedding rows
+
 cudaError_t launch_finalize_draft(const StepState& st, int j, const HeadPrepArgs* prep, cudaStream_t s) {
   HeadPrepArgs hp{};
   if (prep) hp = *prep;
   const int on = prep ? 1 : 0;
-  return st.dtype == DVI_BF16 ? launch1(finalize_draft_kernel<__nv_bfloat16>, s, st, j, hp, on)
-                              : launch1(finalize_draft_kernel<float>, s, st, j, hp, on);
+  const size_t esz = st.dtype == DVI_BF16 ? 2 : 4;
+  const size_t bytes = static_cast<size_t>(st.B) * st.d * esz;
+  const int stage = bytes <= kStageMax ? 1 : 0;
+  const size_t smem = stage ? bytes : 0;
+  static PerDevice attr;
+  attr.once([] {
+    cudaFuncSetAttribute(finalize_draft_kernel<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         static_cast<int>(kStageMax));
+    cudaFuncSetAttribute(finalize_draft_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         static_cast<int>(kStageMax));
+  });
+  const cudaError_t e =
+      st.dtype == DVI_BF16
+          ? launch_pdl(finalize_draft_kernel<__nv_bfloat16>, dim3(1), dim3(128), smem, s, st, j, hp, on, stage)
+          : launch_pdl(finalize_draft_kernel<float>, dim3(1), dim3(128), smem, s, st, j, hp, on, stage);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 cudaError_t launch_finalize_verify(const StepState& st, cudaStream_t s) {
   return st.dtype == DVI_BF16 ? launch1(finalize_verify_kernel<__nv_bfloat16>, s, st)

@@ -209,13 +209,31 @@ __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int 
     for (int j = 0; j < kChunk; ++j) z[j] = v[j];
     if (p.lora_r > 0 && ok) {
       const float* arow = p.lora_a + static_cast<size_t>(f) * p.lora_r;
-      for (int j = 0; j < kChunk; ++j) {
-        const int n = c0 + j;
-        if ((own >> j) & 1u) {
-          const float* bu = (p.lora_bmat ? bu_s : p.lora_bu) + static_cast<size_t>(n) * p.lora_r;
-          float acc = 0.f;
-          for (int q = 0; q < p.lora_r; ++q) acc = fmaf(arow[q], bu[q], acc);
-          z[j] = fmaf(p.gamma, acc, z[j]);
+      if (p.lora_r <= kBuRank) {
+        // the row of A once into registers for every column of the chunk
+        float av[kBuRank];
+#pragma unroll
+        for (int q = 0; q < kBuRank; ++q) av[q] = q < p.lora_r ? arow[q] : 0.f;
+        for (int j = 0; j < kChunk; ++j) {
+          const int n = c0 + j;
+          if ((own >> j) & 1u) {
+            const float* bu = (p.lora_bmat ? bu_s : p.lora_bu) + static_cast<size_t>(n) * p.lora_r;
+            float acc = 0.f;
+#pragma unroll
+            for (int q = 0; q < kBuRank; ++q)
+              if (q < p.lora_r) acc = fmaf(av[q], bu[q], acc);
+            z[j] = fmaf(p.gamma, acc, z[j]);
+          }
+        }
+      } else {
+        for (int j = 0; j < kChunk; ++j) {
+          const int n = c0 + j;
+          if ((own >> j) & 1u) {
+            const float* bu = (p.lora_bmat ? bu_s : p.lora_bu) + static_cast<size_t>(n) * p.lora_r;
+            float acc = 0.f;
+            for (int q = 0; q < p.lora_r; ++q) acc = fmaf(arow[q], bu[q], acc);
+            z[j] = fmaf(p.gamma, acc, z[j]);
+          }
         }
       }
     }
@@ -234,7 +252,7 @@ __device__ __forceinline__ void epilogue_chunk(const ProjArgs& p, int tile, int 
           int row = c0 + j;
           if (p.logits_mode == 2) {   // replay-buffer slot of (sequence, block row)
             const int i = row % p.log_src_rows;
-            row = i < p.log_dst_rows ? row / p.log_src_rows * p.log_dst_rows + i : -1;
+            row = i < p.log_dst_rows ? row / p.log_src_rows * p.log_dst_rows + p.log_dst_off + i : -1;
           }
           if (((own >> j) & 1u) && row >= 0) dst[static_cast<size_t>(row) * p.ld_logits + f] = z[j];
         }
