@@ -69,6 +69,7 @@ struct dvi_ctx {
   long long* counters;
   float* dev_state;
   int* upd_ctr;   // [4 + cap_rows] the update kernels' counters and grid barrier
+  int* fin_ctr;   // arrivals of a head projection's CTAs (finalize in its last CTA)
   float *x_dr, *ss_dr, *x_ver, *ss_ver, *x_pf, *ss_pf, *q, *bu;
   void *xg_dr, *xg_ver, *xg_pf, *attn_o, *ffn_h;
   unsigned long long* amax;
@@ -190,6 +191,7 @@ size_t layout(dvi_ctx* c, char* base) {
   c->counters = reinterpret_cast<long long*>(take(sizeof(long long) * 8));
   c->dev_state = reinterpret_cast<float*>(take(sizeof(float) * 16));
   c->upd_ctr = reinterpret_cast<int*>(take(sizeof(int) * (4 + c->cap_rows)));
+  c->fin_ctr = reinterpret_cast<int*>(take(sizeof(int) * 4));
   c->x_dr = reinterpret_cast<float*>(take(sizeof(float) * B * d));
   c->ss_dr = reinterpret_cast<float*>(take(sizeof(float) * st * B));
   c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * c->Kv * d));
@@ -421,10 +423,11 @@ size_t act_plane(const dvi_ctx* c, const void* buf, int ld) {
 }
 
 // launch_proj with the plane strides of the context's activation buffers.
-cudaError_t launch_proj_ctx(const dvi_ctx* c, ProjArgs a, const ProjMaps* m, cudaStream_t s) {
+cudaError_t launch_proj_ctx(const dvi_ctx* c, ProjArgs a, const ProjMaps* m, cudaStream_t s,
+                            const FinArgs* fin = nullptr) {
   if (a.xg_out) a.xg_plane = act_plane(c, a.xg_out, a.ld_xg);
   if (a.h_out) a.h_plane = act_plane(c, a.h_out, a.ld_h);
-  return launch_proj(a, m, s);
+  return launch_proj(a, m, s, fin);
 }
 
 struct ProjLaunch {
@@ -727,9 +730,11 @@ StepState step_state(dvi_ctx* c) {
 // at row `row0` of `act`; 1/rms from `ss`.  W^S (+ LoRA) when `draft`.
 // With `bu_inline` (bf16 drafter head) the kernel computes B u itself from
 // the draft residual rows instead of reading it from `bu`.
+// With `fin` (kind set), the head's last CTA runs that finalize step when the
+// head launch can (bf16, unsplit); *fin_done tells the caller whether it did.
 dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, const void* act,
                         const CUtensorMap* act_map, int row0, const float* ss, int ss_ld, bool bu_inline = false,
-                        int draft_pass = 0) {
+                        int draft_pass = 0, FinArgs* fin = nullptr, bool* fin_done = nullptr) {
   Pass ps{nullptr, nullptr, 0, rows, 1, 0, 1, 0, nullptr, nullptr};
   ProjArgs a = base_args(ctx, EPI_HEAD, ctx->p_head, ps);
   a.act = act;
@@ -775,7 +780,16 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
   }
   ProjMaps pm{};
   if (ctx->tc) pm = with_act(draft ? ctx->head_s : ctx->head_v, act_map);
-  DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &pm : nullptr, ctx->stream));
+  bool fused = false;
+  if (fin && fin_done) {
+    bool stage = false;
+    const size_t stage_bytes = fin->kind == FIN_DRAFT ? static_cast<size_t>(ctx->B) * ctx->d * ctx->esz : 0;
+    fused = head_fin_ok(a, stage_bytes, &stage);
+    fin->stage = stage && fin->kind == FIN_DRAFT ? 1 : 0;
+    fin->ctr = ctx->fin_ctr;
+    *fin_done = fused;
+  }
+  DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &pm : nullptr, ctx->stream, fused ? fin : nullptr));
   ctx->launches += 1;
   return DVI_OK;
 }
@@ -836,11 +850,20 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
     }
     if (!drafts) continue;
     const int zlog = ctx->log_enabled && ctx->rt.head_mode == 0 ? 2 : 0;   // the drafter's logits of the tuple
-    if ((rc = enqueue_head(ctx, true, ctx->B, zlog, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B, fused, j)) !=
-        DVI_OK)
+    FinArgs fa{};
+    fa.kind = FIN_DRAFT;
+    fa.j = j;
+    fa.prep = fused ? 1 : 0;
+    fa.st = st;
+    fa.hp = h;
+    bool fin_done = false;
+    if ((rc = enqueue_head(ctx, true, ctx->B, zlog, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B, fused, j,
+                           &fa, &fin_done)) != DVI_OK)
       return rc;
-    DVI_CUDA(launch_finalize_draft(st, j, fused ? &h : nullptr, s));
-    ctx->launches += 1;
+    if (!fin_done) {
+      DVI_CUDA(launch_finalize_draft(st, j, fused ? &h : nullptr, s));
+      ctx->launches += 1;
+    }
   }
   return DVI_OK;
 }
@@ -852,11 +875,17 @@ dvi_status enqueue_verify(dvi_ctx* ctx) {
   const int M = ctx->B * ctx->Kv;
   Pass pv{ctx->x_ver, ctx->ss_ver, M, M, ctx->Kv, 0, ctx->B, 0, ctx->xg_ver, &ctx->map_xg_ver};
   if ((rc = enqueue_layers(ctx, ctx->k, ctx->L, pv)) != DVI_OK) return rc;
-  if ((rc = enqueue_head(ctx, false, M, ctx->log_enabled ? 2 : 0, ctx->xg_ver, &ctx->map_xg_ver, 0, ctx->ss_ver,
-                         M)) != DVI_OK)
+  FinArgs fa{};
+  fa.kind = FIN_VERIFY;
+  fa.st = st;
+  bool fin_done = false;
+  if ((rc = enqueue_head(ctx, false, M, ctx->log_enabled ? 2 : 0, ctx->xg_ver, &ctx->map_xg_ver, 0, ctx->ss_ver, M,
+                         false, 0, &fa, &fin_done)) != DVI_OK)
     return rc;
-  DVI_CUDA(launch_finalize_verify(st, s));
-  ctx->launches += 1;
+  if (!fin_done) {
+    DVI_CUDA(launch_finalize_verify(st, s));
+    ctx->launches += 1;
+  }
   return DVI_OK;
 }
 
@@ -1226,10 +1255,17 @@ dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
     Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr};
     dvi_status r = enqueue_layers(ctx, 0, ctx->L, ps);
     if (r != DVI_OK) return r;
-    if ((r = enqueue_head(ctx, false, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B)) != DVI_OK)
+    FinArgs fa{};
+    fa.kind = FIN_AR;
+    fa.st = st;
+    bool fin_done = false;
+    if ((r = enqueue_head(ctx, false, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr, 0, ctx->ss_dr, ctx->B, false, 0, &fa,
+                          &fin_done)) != DVI_OK)
       return r;
-    DVI_CUDA(launch_finalize_ar(st, s));
-    ctx->launches += 1;
+    if (!fin_done) {
+      DVI_CUDA(launch_finalize_ar(st, s));
+      ctx->launches += 1;
+    }
     return DVI_OK;
   });
   if (rc != DVI_OK) return rc;

@@ -87,7 +87,6 @@ struct ProjMaps {
 // so a row's result does not depend on how many rows share the launch.
 void plan_splits(ProjArgs& a, int n_sms, bool tc);
 size_t proj_partial_floats(const ProjArgs& a, bool tc);
-cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s);
 bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols);   // 64-row boxes (gate/up)
 bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);   // [2 planes][rows][cols]
@@ -206,6 +205,26 @@ cudaError_t launch_finalize_ar(const StepState& st, cudaStream_t s);
 cudaError_t launch_finalize_prefill(const StepState& st, int seq, int n_tokens, int32_t* first_out,
                                     cudaStream_t s);
 cudaError_t launch_reset_seq(const StepState& st, int seq, cudaStream_t s);
+
+// A finalize step run by the last CTA of a head projection (bf16, unsplit
+// head): FIN_DRAFT after the drafter head of pass j (with the head
+// preparation when `prep`), FIN_VERIFY after the verifier head, FIN_AR after
+// the head of a greedy AR step.  `stage`: the head CTA has shared memory
+// for the next pass's embedding rows.
+enum FinKind : int { FIN_NONE = 0, FIN_DRAFT = 1, FIN_VERIFY = 2, FIN_AR = 3 };
+struct FinArgs {
+  int kind, j, prep, stage;
+  int* ctr;          // arrivals of the head's CTAs; 0 before a launch, reset by the last CTA
+  StepState st;
+  HeadPrepArgs hp;
+};
+// Shared memory a finalize step needs in the head CTA (without staging).
+size_t fin_smem_bytes();
+
+cudaError_t launch_proj(const ProjArgs& a, const ProjMaps* maps, cudaStream_t s, const FinArgs* fin = nullptr);
+// Whether a head launch of these arguments can run a finalize step, and
+// whether its free shared memory holds `stage_bytes` of staged rows.
+bool head_fin_ok(const ProjArgs& a, size_t stage_bytes, bool* stage);
 
 // ---- drafter update (update.cu)
 struct UpdateArgs {

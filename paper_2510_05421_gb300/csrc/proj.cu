@@ -50,8 +50,7 @@
 #include <algorithm>
 #include <cudaTypedefs.h>
 
-#include "common.cuh"
-#include "kernels.h"
+#include "finalize.cuh"
 
 namespace dvi {
 
@@ -352,12 +351,14 @@ __device__ __forceinline__ void produce_b_f32(const ProjArgs& p, uint8_t* bs, in
 
 // ------------------------------------------------------------------ tcgen05
 // kSplit: the launch splits K over a cluster (n_splits > 1); the unsplit
-// instantiation carries no cluster code.
-template <bool kSplit>
+// instantiation carries no cluster code.  kFinNT > 0: a head whose last CTA
+// may run a finalize step (row arrays of kFinNT tiles: d <= 128 kFinNT); the
+// other instantiations carry none of its code or registers.
+template <bool kSplit, int kFinNT = 0>
 __global__ void __launch_bounds__(192, 2)
     proj_tc_kernel(const __grid_constant__ CUtensorMap m0, const __grid_constant__ CUtensorMap m1,
                    const __grid_constant__ CUtensorMap m2, const __grid_constant__ CUtensorMap mb,
-                   const ProjArgs p, int stages) {
+                   const ProjArgs p, int stages, const __grid_constant__ FinArgs fin) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);
@@ -571,6 +572,10 @@ __global__ void __launch_bounds__(192, 2)
     if (warp == 0) {
       tc_fence_after();
       tmem_dealloc(tmem, ncols);
+    }
+    // a head whose last CTA runs the pass's finalize step (the ring is free)
+    if constexpr (!kSplit && kFinNT > 0) {
+      if (fin.kind != FIN_NONE) head_finalize<kFinNT>(fin, sA + abytes, tid);
     }
   }
   if (kSplit) {
@@ -1192,13 +1197,28 @@ static int tc_stages(int n_pad, size_t* smem_bytes) {
   return stages;
 }
 
-cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s) {
+size_t fin_smem_bytes() { return (sizeof(FinSmem) + 15) / 16 * 16; }
+
+bool head_fin_ok(const ProjArgs& a, size_t stage_bytes, bool* stage) {
+  if (a.dtype != DVI_BF16 || a.flavor != EPI_HEAD || a.n_splits != 1) return false;
+  size_t smem = 0;
+  const int stages = tc_stages(a.n_pad, &smem);
+  const size_t ring = static_cast<size_t>(stages) * (16384 + 2 * static_cast<size_t>(a.n_pad) * 128);
+  *stage = ring >= 16384 + fin_smem_bytes() + stage_bytes;
+  return ring >= 16384 + fin_smem_bytes();
+}
+
+cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s, const FinArgs* fin) {
   cudaError_t e;
+  FinArgs f{};
+  if (fin) f = *fin;
   if (a0.dtype == DVI_BF16) {
     static PerDevice attr;
     attr.once([] {
       cudaFuncSetAttribute(proj_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
       cudaFuncSetAttribute(proj_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      cudaFuncSetAttribute(proj_tc_kernel<false, 32>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+      cudaFuncSetAttribute(proj_tc_kernel<false, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     });
     ProjArgs a = a0;
     size_t smem = 0;
@@ -1217,9 +1237,14 @@ cudaError_t launch_proj(const ProjArgs& a0, const ProjMaps* maps, cudaStream_t s
     at[1].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = a.n_splits > 1 ? 2 : 1;
-    e = a.n_splits > 1
-            ? cudaLaunchKernelEx(&cfg, proj_tc_kernel<true>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages)
-            : cudaLaunchKernelEx(&cfg, proj_tc_kernel<false>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages);
+    if (a.n_splits > 1)
+      e = cudaLaunchKernelEx(&cfg, proj_tc_kernel<true>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages, f);
+    else if (f.kind == FIN_NONE)
+      e = cudaLaunchKernelEx(&cfg, proj_tc_kernel<false>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages, f);
+    else if (a.K <= 32 * kTileRows)
+      e = cudaLaunchKernelEx(&cfg, proj_tc_kernel<false, 32>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages, f);
+    else
+      e = cudaLaunchKernelEx(&cfg, proj_tc_kernel<false, 64>, maps->m0, maps->m1, maps->m2, maps->mb, a, stages, f);
   } else {
     ProjArgs b = a0;
     b.n_ttiles = (a0.M + kChunk - 1) / kChunk;
