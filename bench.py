@@ -72,6 +72,18 @@ def step_bytes(w, n_ctx):
     return draft, verify
 
 
+def update_bytes(w, rows):
+    """Algorithmic HBM bytes of one LoRA drafter update on `rows` buffer rows:
+    the logged drafter logits z and verifier logits (rows x V f32 each) and
+    head inputs u (bf16 hi/lo or f32), and A, B with their Adam moments read
+    and written plus their gradients written.  W^S is not read: z was logged
+    by the drafter head while drafting."""
+    s = w.shape
+    usz = 4  # bf16 hi + lo planes, or one f32 plane
+    lora = (s.vocab + s.d_model) * w.lora_rank * 4
+    return 2 * rows * s.vocab * 4 + rows * s.d_model * usz + 7 * lora
+
+
 def prefill_flops(w, n):
     """Algorithmic FLOPs of prefilling one n-token prompt: 2 per weight per
     token for every layer's projections, the causal attention's two
@@ -166,7 +178,7 @@ class ClockSampler:
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
         try:
             self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits",
-                                       "-i", str(gpu_index), "-lms", "100"], stdout=self.f,
+                                       "-i", str(gpu_index), "-lms", "25"], stdout=self.f,
                                       stderr=subprocess.DEVNULL)
         except OSError:
             self.p = None
@@ -388,6 +400,15 @@ def time_ar(eng, dP, lens0, n_tokens, dev):
     return {"tokens_per_s": B * n_steps / (ms / 1e3), "ms_per_step": ms / n_steps, "steps": n_steps}
 
 
+def update_roofline(w, u_ms, hbm):
+    """The drafter update against its bytes (one update on a full buffer)."""
+    rows = w.update_every * w.batch * w.k_spec
+    nb = update_bytes(w, rows)
+    ach = nb / (u_ms / 1e3) / 1e9
+    return {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm, "bytes": nb,
+            "rows": rows, "note": "latency-bound: one cooperative launch, two grid barriers; W^S is not re-read"}
+
+
 def pass_rooflines(w, r, hbm):
     """Draft- and verify-phase HBM fractions from the per-phase timing."""
     n_mid = (r["lens0"] + r["lens1"]) / 2.0
@@ -562,6 +583,7 @@ def main():
         "roofline_draft": {"bound": "hbm", "achieved": d_gbs, "peak": hbm, "unit": "GB/s", "frac": d_gbs / hbm,
                            "bytes_per_launch": draft_b, "ms_per_launch": d_ms},
         "update_ms": u_ms,
+        "roofline_update": update_roofline(w, u_ms, hbm),
         "gpu_launches": r["launches"],
         "clocks": r["clocks"],
         "device_flags": r["status"],

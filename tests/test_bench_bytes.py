@@ -96,3 +96,13 @@ def test_prefill_flops_and_bound():
     # a short prompt is bound by its bytes
     r = bench.prefill_roofline(bench.prefill_flops(w, 16), bench.prefill_alg_bytes(w, 16), 5.0, pk)
     assert r["bound"] == "hbm"
+
+
+def test_update_bytes_of_the_7b_workload():
+    w = workload("7b")
+    # 20 rows: logged z and verifier logits (2 x 20 x 32000 x 4 B), u as two
+    # bf16 planes (20 x 4096 x 4 B), and A [32000 x 16], B [16 x 4096] f32
+    # with their Adam moments read and written and the gradient written
+    expect = 2 * 20 * 32000 * 4 + 20 * 4096 * 4 + 7 * (32000 + 4096) * 16 * 4
+    assert bench.update_bytes(w, 20) == expect
+    assert expect == pytest.approx(21.6e6, rel=1e-2)
