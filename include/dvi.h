@@ -105,6 +105,14 @@ typedef struct {
                            its own); the context then needs every CTA of that launch resident
                            at once (two per SM) and ignores the flag when they do not fit.
                            Results differ from mode 0 in summation order only. */
+  int chain_counters;   /* 0: each launch of a decode pass waits for its predecessor's whole
+                           grid (programmatic dependent launch).  1: bf16 decode passes
+                           (draft, verify, AR step; not with persistent = 1) chain their
+                           projection, attention and head launches through per-launch
+                           completion counters: each CTA adds 1 with release semantics
+                           after its last write and the next launch polls the count with
+                           acquire semantics (bounded: DVI_DEV_TIMEOUT).  Same arithmetic,
+                           bit-identical results. */
 } dvi_runtime_config;
 
 typedef struct {

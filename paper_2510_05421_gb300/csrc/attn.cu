@@ -373,7 +373,12 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
   float* wO = reinterpret_cast<float*>(ring);                       // [4][16][HD], after the loop
   float* cO = reinterpret_cast<float*>(ring) + 4 * kMmaQ * HD;      // [16][HD] this split's O
   griddep_launch();
-  griddep_wait();
+  if (a.dep_wait) {
+    if (threadIdx.x == 0) dep_wait(a.dep_wait, a.dep_count, a.status);
+    __syncthreads();
+  } else {
+    griddep_wait();
+  }
   cg::cluster_group cluster = cg::this_cluster();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gq = lane >> 2, tq = lane & 3;           // mma fragment coordinates
@@ -649,6 +654,10 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const __grid_constant__ C
                            a.o_plane, O * rinv[qi]);
   }
   cluster.sync();   // every rank keeps its shared memory until all have read it
+  if (a.dep_signal) {
+    __syncthreads();
+    if (threadIdx.x == 0) dep_signal(a.dep_signal);
+  }
 }
 
 // ------------------------------------------------------------------ prefill
@@ -1134,6 +1143,19 @@ static cudaError_t launch_attn_t(const AttnArgs& a, cudaStream_t s) {
   static PerDevice attr;
   attr.once([] { cudaFuncSetAttribute(attn_smem_kernel<T, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024); });
   return launch_pdl(attn_smem_kernel<T, T>, grid, dim3(128), attn_smem(a.head_dim), s, a);
+}
+
+bool attn_chainable(const AttnArgs& a) {
+  return a.dtype == DVI_BF16 && !a.prefill && a.n_heads / a.n_kv_heads <= kRegQ;
+}
+
+int attn_grid_ctas(const AttnArgs& a) {
+  const int G = a.n_heads / a.n_kv_heads;
+  if (a.dtype == DVI_BF16 && a.prefill && G <= kRegQ) {
+    const int rc = 4 * (kPfWarpQ / G);
+    return a.n_kv_heads * ((a.rows_per_seq + rc - 1) / rc) * a.n_seqs;
+  }
+  return a.n_splits_max * a.n_kv_heads * a.n_seqs * n_qgroups(a, a.dtype == DVI_BF16);
 }
 
 cudaError_t launch_attn(const AttnArgs& a, cudaStream_t s) {

@@ -129,6 +129,27 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// ---------------------------------------------------------------- chained launches
+// Inside a captured decode pass, consecutive kernels can be chained by a
+// completion counter instead of grid dependency: each CTA of a kernel adds 1
+// to its counter (release) after its last global write, and the next kernel
+// polls that counter (acquire) until it reaches the kernel's grid size.  The
+// next kernel is launched with programmatic stream serialization, which
+// starts it only once every CTA of its predecessor has started, so the
+// count it waits for always comes.  The poll is bounded like every other
+// wait (then DVI_DEV_TIMEOUT and false).  With no counter, the kernel waits
+// for its predecessor's grid (griddep_wait).  `fence.proxy.async` orders the
+// acquired writes before the caller's later TMA reads.
+__device__ __forceinline__ int ld_acquire_gpu_i32(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ bool dep_wait(const int* ctr, int count, int* status);
+__device__ __forceinline__ void dep_signal(int* ctr) {
+  if (ctr) asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(ctr) : "memory");
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
@@ -188,6 +209,24 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
   }
   flag_status(status, DVI_DEV_TIMEOUT);
   return false;
+}
+
+__device__ __forceinline__ bool dep_wait(const int* ctr, int count, int* status) {
+  if (!ctr) {
+    griddep_wait();
+    return true;
+  }
+  if (ld_acquire_gpu_i32(ctr) < count) {
+    const uint64_t t0 = global_ns();
+    while (ld_acquire_gpu_i32(ctr) < count) {
+      if (global_ns() - t0 > kWaitLimitNs) {
+        flag_status(status, DVI_DEV_TIMEOUT);
+        return false;
+      }
+    }
+  }
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  return true;
 }
 
 // ---------------------------------------------------------------- cluster

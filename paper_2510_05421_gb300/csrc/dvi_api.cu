@@ -70,6 +70,14 @@ struct dvi_ctx {
   float* dev_state;
   int* upd_ctr;   // [4 + cap_rows] the update kernels' counters and grid barrier
   int* fin_ctr;   // arrivals of a head projection's CTAs (finalize in its last CTA)
+  // chained launches of a bf16 decode pass: one completion counter per
+  // launch, cleared by a memset at the pass's start
+  int* dep_ctr = nullptr;
+  int n_dep_ctr = 0;
+  bool dep_on = false;
+  int dep_slot = 0;
+  int* dep_prev = nullptr;   // counter of the previous launch, if it signals
+  int dep_prev_count = 0;    // that launch's CTAs
   float *x_dr, *ss_dr, *x_ver, *ss_ver, *x_pf, *ss_pf, *q, *bu;
   void *xg_dr, *xg_ver, *xg_pf, *attn_o, *ffn_h;
   unsigned long long* amax;
@@ -157,6 +165,7 @@ bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::
   if (rt->k_spec < 1 || rt->k_spec > 16) return bad("k_spec must be in [1, 16]");
   if (rt->bonus != 0 && rt->bonus != 1) return bad("bonus must be 0 or 1");
   if (rt->persistent != 0 && rt->persistent != 1) return bad("persistent must be 0 or 1");
+  if (rt->chain_counters != 0 && rt->chain_counters != 1) return bad("chain_counters must be 0 or 1");
   if (rt->k_spec + rt->bonus > 16) return bad("k_spec + bonus must be <= 16");
   if (rt->max_seq_len < rt->k_spec + 2) return bad("max_seq_len too small");
   if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
@@ -192,6 +201,7 @@ size_t layout(dvi_ctx* c, char* base) {
   c->dev_state = reinterpret_cast<float*>(take(sizeof(float) * 16));
   c->upd_ctr = reinterpret_cast<int*>(take(sizeof(int) * (4 + c->cap_rows)));
   c->fin_ctr = reinterpret_cast<int*>(take(sizeof(int) * 4));
+  c->dep_ctr = reinterpret_cast<int*>(take(sizeof(int) * c->n_dep_ctr));
   c->x_dr = reinterpret_cast<float*>(take(sizeof(float) * B * d));
   c->ss_dr = reinterpret_cast<float*>(take(sizeof(float) * st * B));
   c->x_ver = reinterpret_cast<float*>(take(sizeof(float) * B * c->Kv * d));
@@ -354,6 +364,9 @@ bool init_dims(dvi_ctx* c, const dvi_model_config* cfg, const dvi_runtime_config
   c->pf_rows = cfg->dtype == DVI_BF16 ? (c->chunk + 127) / 128 * 128 : c->chunk;
   c->Kv = c->K + (rt->bonus ? 1 : 0);
   c->M_max = std::max(std::max(c->B * c->Kv, c->pf_rows), std::max(c->cap_rows, c->B));
+  // launches of the longest decode pass: the draft phase (Kv passes of k
+  // layers and a head), the verify pass, or an AR step
+  c->n_dep_ctr = std::max(c->Kv * (5 * c->k + 3), 5 * c->L + 3) + 8;
   c->nq = c->Hq * c->hd;
   c->nkv = c->Hkv * c->hd;
   c->tc = cfg->dtype == DVI_BF16;
@@ -433,6 +446,50 @@ cudaError_t launch_proj_ctx(const dvi_ctx* c, ProjArgs a, const ProjMaps* m, cud
 struct ProjLaunch {
   ProjArgs a;
   ProjMaps m;
+};
+
+// Completion-counter chaining of a bf16 decode pass (runtime option
+// chain_counters; common.cuh): clears the pass's counters and turns chaining
+// on; bf16 only, and not with the persistent projection chain.
+cudaError_t dep_begin(dvi_ctx* c) {
+  c->dep_on = false;
+  c->dep_prev = nullptr;
+  if (!c->tc || c->chain_ctas > 0 || !c->rt.chain_counters) return cudaSuccess;
+  const cudaError_t e = cudaMemsetAsync(c->dep_ctr, 0, sizeof(int) * c->n_dep_ctr, c->stream);
+  if (e != cudaSuccess) return e;
+  c->dep_on = true;
+  c->dep_slot = 0;
+  return cudaSuccess;
+}
+void dep_end(dvi_ctx* c) {
+  c->dep_on = false;
+  c->dep_prev = nullptr;
+}
+// A launch of `grid` CTAs joins the chain: it waits for the previous
+// launch's counter (if that one signals) and signals its own.
+template <typename A>
+void dep_link(dvi_ctx* c, A& a, int grid) {
+  a.dep_wait = nullptr;
+  a.dep_signal = nullptr;
+  if (!c->dep_on) return;
+  a.dep_wait = c->dep_prev;
+  a.dep_count = c->dep_prev_count;
+  if (c->dep_slot < c->n_dep_ctr) {
+    a.dep_signal = c->dep_ctr + c->dep_slot++;
+    c->dep_prev = a.dep_signal;
+    c->dep_prev_count = grid;
+  } else {
+    c->dep_prev = nullptr;
+  }
+}
+// A launch outside the chain (it waits for its predecessor's grid): the
+// next launch waits for it the same way.
+void dep_break(dvi_ctx* c) { c->dep_prev = nullptr; }
+// Chaining for the launches enqueued while it lives.
+struct DepScope {
+  dvi_ctx* c;
+  explicit DepScope(dvi_ctx* ctx) : c(ctx) {}
+  ~DepScope() { dep_end(c); }
 };
 
 // q, k, v of RMSNorm(x) (gain folded into xg, 1/rms in the epilogue), RoPE,
@@ -568,7 +625,10 @@ ProjLaunch down_launch(dvi_ctx* ctx, int l, const Pass& ps, const float* g_last)
 }
 
 dvi_status run_proj(dvi_ctx* ctx, const ProjLaunch& pl) {
-  DVI_CUDA(launch_proj_ctx(ctx, pl.a, ctx->tc ? &pl.m : nullptr, ctx->stream));
+  ProjArgs a = pl.a;
+  if (ctx->tc) dep_link(ctx, a, a.n_tiles * a.n_splits);
+  else dep_break(ctx);
+  DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &pl.m : nullptr, ctx->stream));
   ++ctx->launches;
   return DVI_OK;
 }
@@ -650,7 +710,10 @@ dvi_status enqueue_layer(dvi_ctx* ctx, int l, const Pass& ps, const float* g_las
   if (ps.pf) return enqueue_layer_pf(ctx, l, ps, g_last);
   dvi_status st;
   if ((st = run_proj(ctx, qkv_launch(ctx, l, ps))) != DVI_OK) return st;
-  DVI_CUDA(launch_attn(attn_args(ctx, l, ps), ctx->stream));
+  AttnArgs at = attn_args(ctx, l, ps);
+  if (ctx->tc && attn_chainable(at)) dep_link(ctx, at, attn_grid_ctas(at));
+  else dep_break(ctx);
+  DVI_CUDA(launch_attn(at, ctx->stream));
   ++ctx->launches;
   if ((st = run_proj(ctx, o_launch(ctx, l, ps))) != DVI_OK) return st;
   if ((st = run_proj(ctx, gu_launch(ctx, l, ps))) != DVI_OK) return st;
@@ -789,6 +852,8 @@ dvi_status enqueue_head(dvi_ctx* ctx, bool draft, int rows, int logits_mode, con
     fin->ctr = ctx->fin_ctr;
     *fin_done = fused;
   }
+  if (ctx->tc) dep_link(ctx, a, a.n_tiles * a.n_splits);
+  else dep_break(ctx);
   DVI_CUDA(launch_proj_ctx(ctx, a, ctx->tc ? &pm : nullptr, ctx->stream, fused ? fin : nullptr));
   ctx->launches += 1;
   return DVI_OK;
@@ -804,6 +869,8 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   dvi_status rc;
+  DepScope dep(ctx);
+  DVI_CUDA(dep_begin(ctx));
   // passes j = 0..K-1 draft t~_{j+1}; with the bonus row, pass K only hands
   // h_{k,n+K} (of t~_K) to the verify rows
   for (int j = 0; j < ctx->Kv; ++j) {
@@ -845,6 +912,7 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
       h.r = ctx->r;
     }
     if (!fused) {
+      dep_break(ctx);
       DVI_CUDA(launch_head_prep(h, s));
       ctx->launches += 1;
     }
@@ -861,6 +929,7 @@ dvi_status enqueue_draft(dvi_ctx* ctx) {
                            &fa, &fin_done)) != DVI_OK)
       return rc;
     if (!fin_done) {
+      dep_break(ctx);
       DVI_CUDA(launch_finalize_draft(st, j, fused ? &h : nullptr, s));
       ctx->launches += 1;
     }
@@ -873,6 +942,8 @@ dvi_status enqueue_verify(dvi_ctx* ctx) {
   const StepState st = step_state(ctx);
   dvi_status rc;
   const int M = ctx->B * ctx->Kv;
+  DepScope dep(ctx);
+  DVI_CUDA(dep_begin(ctx));
   Pass pv{ctx->x_ver, ctx->ss_ver, M, M, ctx->Kv, 0, ctx->B, 0, ctx->xg_ver, &ctx->map_xg_ver};
   if ((rc = enqueue_layers(ctx, ctx->k, ctx->L, pv)) != DVI_OK) return rc;
   FinArgs fa{};
@@ -883,6 +954,7 @@ dvi_status enqueue_verify(dvi_ctx* ctx) {
                          false, 0, &fa, &fin_done)) != DVI_OK)
     return rc;
   if (!fin_done) {
+    dep_break(ctx);
     DVI_CUDA(launch_finalize_verify(st, s));
     ctx->launches += 1;
   }
@@ -1252,6 +1324,8 @@ dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
   dvi_status rc = run_graph(ctx, &ctx->ar_exec, &ctx->ar_launches, g, [&]() -> dvi_status {
     StepState st = step_state(ctx);
     st.out_ids = ctx->ar_out;
+    DepScope dep(ctx);
+    DVI_CUDA(dep_begin(ctx));
     Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr};
     dvi_status r = enqueue_layers(ctx, 0, ctx->L, ps);
     if (r != DVI_OK) return r;
@@ -1263,6 +1337,7 @@ dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
                           &fin_done)) != DVI_OK)
       return r;
     if (!fin_done) {
+      dep_break(ctx);
       DVI_CUDA(launch_finalize_ar(st, s));
       ctx->launches += 1;
     }

@@ -76,6 +76,10 @@ struct ProjArgs {
   // residual rows bu_x and the final-norm gain bu_g
   const float* lora_bmat; const float* bu_x; int bu_ldx; const float* bu_g;
   unsigned long long* amax;   // [M] argmax keys, or null
+  // chained launch (decode passes): wait until *dep_wait >= dep_count (the
+  // predecessor's CTAs), else for the predecessor's grid; add 1 to
+  // *dep_signal after this CTA's last write (null: no signal)
+  const int* dep_wait; int dep_count; int* dep_signal;
 };
 
 struct ProjMaps {
@@ -148,7 +152,13 @@ struct AttnArgs {
   const CUtensorMap* kmap;           // bf16 decode: the K / V caches as [rows][hd] (box 64 x 64)
   const CUtensorMap* vmap;
   int prefill;                       // a prompt pass (bf16, GQA group <= 8): the prefill attention kernel
+  const int* dep_wait; int dep_count; int* dep_signal;   // chained launch (as ProjArgs; bf16 decode kernel)
 };
+// CTAs of the attention launch for these arguments.
+int attn_grid_ctas(const AttnArgs& a);
+// The decode attention kernel that takes part in completion-counter chaining
+// (bf16 decode rows, at most kRegQ query heads per KV head).
+bool attn_chainable(const AttnArgs& a);
 bool make_kv_map(CUtensorMap* map, const void* cache, long long rows, int hd);
 size_t attn_partial_floats(const AttnArgs& a);
 int attn_counters(const AttnArgs& a);

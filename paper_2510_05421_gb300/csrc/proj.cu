@@ -454,7 +454,7 @@ __global__ void __launch_bounds__(192, 2)
         mbar_arrive_expect_tx(&full[i], tx);
         load_a(i);
       }
-      griddep_wait();
+      dep_wait(p.dep_wait, p.dep_count, p.status);
       for (int i = 0; i < pre; ++i) load_b(i);
       int issued = pre;
       for (int i = pre; i < nkb; ++i) {
@@ -502,7 +502,12 @@ __global__ void __launch_bounds__(192, 2)
   } else {
     // ---------------- warps 0-3: (B producer for f32 rows), norm scales, TMEM
     const int tid = threadIdx.x;
-    griddep_wait();
+    if (p.dep_wait) {
+      if (tid == 0) dep_wait(p.dep_wait, p.dep_count, p.status);
+      named_bar(1, kTileRows);
+    } else {
+      griddep_wait();
+    }
     if (soft_b) {
       for (int i = 0; i < nkb; ++i) {
         const int s = i % stages;
@@ -622,6 +627,12 @@ __global__ void __launch_bounds__(192, 2)
     // every rank keeps its shared memory until all have read it
     cluster_arrive_release();
     cluster_wait_acquire();
+  }
+  if (p.dep_signal) {
+    // this CTA's outputs (and a head's finalize step) are written; the
+    // barrier orders them before thread 0's release
+    __syncthreads();
+    if (threadIdx.x == 0) dep_signal(p.dep_signal);
   }
 }
 
