@@ -324,11 +324,11 @@ def reference_arm(args, w, rank):
     return 0
 
 
-def make_engine(w, dw, max_len, local, persistent=False):
+def make_engine(w, dw, max_len, local, persistent=False, megakernel=False):
     from paper_2510_05421_gb300 import DVIEngine
     return DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=w.k_spec, split_k=w.split_k,
                      lora_rank=w.lora_rank, lora_gamma=w.lora_gamma, max_seq_len=max_len,
-                     log_steps=w.update_every, device=local, persistent=persistent)
+                     log_steps=w.update_every, device=local, persistent=persistent, megakernel=megakernel)
 
 
 def time_dvi(eng, w, hyper, warmup, steps, dev, world=1, clocks=False):
@@ -433,7 +433,7 @@ def extra_workload(name, args, local, dev, pk):
     U, K = w.update_every, w.k_spec
     steps = max(6, args.steps // 2)
     max_len = max(len(p) for p in P) + (args.warmup + steps) * U * K + 2 * K + 64
-    eng = make_engine(w, dw, max_len, local)
+    eng = make_engine(w, dw, max_len, local, megakernel=args.megakernel)
     dP = [torch.from_numpy(p).to(dev) for p in P]
     for b, p in enumerate(dP):
         eng.prefill(b, p)
@@ -463,6 +463,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling cases)")
     ap.add_argument("--prompt", type=int, default=0, help="override the prompt length (small profiling cases)")
+    ap.add_argument("--megakernel", action="store_true",
+                    help="run the draft phase as one persistent launch (runtime option megakernel = 1)")
     ap.add_argument("--persistent", action="store_true",
                     help="run each layer's projections as one persistent launch (runtime option persistent = 1)")
     args = ap.parse_args()
@@ -498,7 +500,8 @@ def main():
     U, K = w.update_every, w.k_spec
     gen_room = max(w.gen_tokens, (args.warmup + args.steps) * U * K)
     max_len = max(len(p) for p in P) + gen_room + 2 * K + 64
-    eng = make_engine(w, dw, max_len, local, args.persistent)
+    eng = make_engine(w, dw, max_len, local, args.persistent, args.megakernel)
+    mk_ctas = eng.stats()["megakernel_ctas"]
     hyper = update_config(w.update)
     # prefill: sequence 0's prompt once to warm up, then every prompt timed
     # with CUDA events on the engine's stream (prompts already on the device)
@@ -534,7 +537,8 @@ def main():
     e2e = None
     if not args.no_e2e:
         eng.close()
-        eng = make_engine(w, dw, max(len(p) for p in P) + w.gen_tokens * K + 64, local, args.persistent)
+        eng = make_engine(w, dw, max(len(p) for p in P) + w.gen_tokens * K + 64, local, args.persistent,
+                          args.megakernel)
         eng.generate(P, 8, update_every=U, hyper=w.update, max_steps=2 * U)
         torch.cuda.synchronize(dev)
         t0 = time.perf_counter()
@@ -566,7 +570,9 @@ def main():
                    "step": f"{U} draft_verify_commit calls + 1 update_drafter",
                    "l2": "inputs larger than L2: ~13 GB of weights streamed per step",
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "projections": "persistent chain" if args.persistent else "one kernel each"},
+                   "projections": "persistent chain" if args.persistent else "one kernel each",
+                   "draft_phase": (f"one persistent launch of {mk_ctas} CTAs (megakernel)" if mk_ctas
+                                   else "one kernel per projection, attention and head")},
         "mean_accepted_length": r["mat"],
         "ar_tokens_per_s": ar_value,
         "speedup_vs_ar": value / ar_value,

@@ -113,6 +113,17 @@ typedef struct {
                            after its last write and the next launch polls the count with
                            acquire semantics (bounded: DVI_DEV_TIMEOUT).  Same arithmetic,
                            bit-identical results. */
+  int megakernel;       /* 0: the draft passes run one kernel per projection, attention and
+                           head.  1: bf16 contexts of at most 2 sequences with k <= 16 draft
+                           layers (GQA groups <= 8, head_dim 64 or 128, d a multiple of 128)
+                           run the whole draft phase -- every draft pass's k layers, the
+                           drafter head with its argmax, the hand-off of h_k to the verify
+                           rows -- as one persistent launch of one CTA per SM (Sec. 3.3
+                           draft rollout), and the greedy AR step runs its first k layers
+                           the same way, so the DVI stream stays bit-identical to AR.  Its
+                           projections are row-split GEMVs on f32 activations; its phases
+                           meet at completion counters with bounded waits.  Ignored when the
+                           shape or the device does not allow it (stats: megakernel_ctas). */
 } dvi_runtime_config;
 
 typedef struct {
@@ -178,6 +189,8 @@ typedef struct {
   int device_status;      /* DVI_DEV_* bits */
   int persistent_ctas;    /* grid of the persistent projection launch (runtime option
                              persistent = 1 in effect), else 0 */
+  int megakernel_ctas;    /* grid of the draft-phase megakernel (runtime option megakernel = 1
+                             in effect), else 0 */
 } dvi_stats;
 
 /* Bytes of device workspace a context needs (KV caches, residual streams,

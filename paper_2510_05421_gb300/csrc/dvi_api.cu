@@ -94,6 +94,16 @@ struct dvi_ctx {
   int attn_split_len, attn_nsplits;
   int dec_nsplits;                  // bf16 decode attention: splits (one cluster) per KV head
   int chain_ctas = 0;               // persistent projection chain: grid size (0: not used)
+  // draft-phase megakernel (runtime option megakernel): the static part of
+  // its arguments, its scratch, and whether it runs (bf16, eligible shapes,
+  // one CTA per SM resident)
+  bool mk_sized = false;
+  bool mk_on = false;
+  MkArgs mk{};
+  size_t mk_sync_bytes = 0;
+  void* mk_sync = nullptr;   // argmax keys, then the completion counters and abort flag
+  CUtensorMap* mk_maps_dev = nullptr;   // the kernel's weight descriptors (workspace)
+  std::vector<CUtensorMap> mk_maps;     // their host copy (source of the upload)
   float* chain_part = nullptr;
   size_t chain_part_floats = 0;
   int* chain_ctr = nullptr;
@@ -166,6 +176,7 @@ bool valid_config(const dvi_model_config* c, const dvi_runtime_config* rt, std::
   if (rt->bonus != 0 && rt->bonus != 1) return bad("bonus must be 0 or 1");
   if (rt->persistent != 0 && rt->persistent != 1) return bad("persistent must be 0 or 1");
   if (rt->chain_counters != 0 && rt->chain_counters != 1) return bad("chain_counters must be 0 or 1");
+  if (rt->megakernel != 0 && rt->megakernel != 1) return bad("megakernel must be 0 or 1");
   if (rt->k_spec + rt->bonus > 16) return bad("k_spec + bonus must be <= 16");
   if (rt->max_seq_len < rt->k_spec + 2) return bad("max_seq_len too small");
   if (rt->log_steps < 1 || rt->log_steps * rt->batch * rt->k_spec > kMaxTokens)
@@ -259,6 +270,23 @@ size_t layout(dvi_ctx* c, char* base) {
   c->n_committed = reinterpret_cast<int*>(take(sizeof(int) * B));
   c->n_accepted = reinterpret_cast<int*>(take(sizeof(int) * B));
   c->ar_out = reinterpret_cast<int*>(take(sizeof(int) * B));
+  if (c->mk_sized) {
+    MkArgs& a = c->mk;
+    const size_t nqkv = static_cast<size_t>(c->Hq + 2 * c->Hkv) * c->hd;
+    a.xr = reinterpret_cast<float*>(take(sizeof(float) * 2 * B * d));
+    a.qkv = reinterpret_cast<float*>(take(sizeof(float) * B * nqkv));
+    a.att = reinterpret_cast<float*>(take(sizeof(float) * B * c->Hq * a.P * (c->hd + 2)));
+    a.ao = reinterpret_cast<float*>(take(sizeof(float) * B * d));
+    a.hbuf = reinterpret_cast<float*>(take(sizeof(float) * B * c->F));
+    a.y = reinterpret_cast<float*>(take(sizeof(float) * B * d));
+    a.bu_part = reinterpret_cast<float*>(take(sizeof(float) * c->n_sms * B * (r > 0 ? r : 1)));
+    c->mk_sync = take(c->mk_sync_bytes);
+    c->mk_maps_dev = reinterpret_cast<CUtensorMap*>(take(sizeof(CUtensorMap) * (7 * c->k + 1)));
+    a.keys = reinterpret_cast<unsigned long long*>(c->mk_sync);
+    a.ctr = c->mk_sync ? reinterpret_cast<int*>(static_cast<char*>(c->mk_sync) +
+                                                sizeof(unsigned long long) * c->Kv * B)
+                       : nullptr;
+  }
   return align_up(off, 256);
 }
 
@@ -273,6 +301,8 @@ Plan plan_for(dvi_ctx* c, int flavor, int n_out, int K, int rq, int rk, int rv) 
   plan_splits(a, c->n_sms, c->tc);
   return Plan{a.n_tiles, a.n_splits, a.kb_total, a.kb_per_split};
 }
+
+void size_mk(dvi_ctx* c);
 
 void size_scratch(dvi_ctx* c) {
   const int Ms[2] = {c->M_max, 1};
@@ -341,6 +371,47 @@ void size_scratch(dvi_ctx* c) {
       c->chain_part_floats = chain_partial_floats(max_tiles, c->chain_ctas, kChainMaxPad);
     }
   }
+  size_mk(c);
+}
+
+// The draft-phase megakernel's static arguments and scratch (runtime option
+// megakernel): bf16, at most kMkMaxRows sequences, k <= kMkMaxLayers shallow
+// layers, GQA groups up to kMkMaxGroup, d a multiple of 128, and a ring of at
+// least four 16 KB stages beside the kernel's other shared memory.
+void size_mk(dvi_ctx* c) {
+  c->mk_sized = false;
+  if (!c->tc || !c->rt.megakernel || c->B > kMkMaxRows || c->k > kMkMaxLayers || c->Hq / c->Hkv > kMkMaxGroup ||
+      c->d % 128 || c->F % 64 || (c->hd != 64 && c->hd != 128) || c->B * c->Hkv > c->n_sms)
+    return;
+  MkArgs& a = c->mk;
+  a = MkArgs{};
+  a.B = c->B;
+  a.k = c->k;
+  a.d = c->d;
+  a.Hq = c->Hq;
+  a.Hkv = c->Hkv;
+  a.hd = c->hd;
+  a.F = c->F;
+  a.V = c->V;
+  a.max_len = c->max_len;
+  a.K = c->K;
+  a.Kv = c->Kv;
+  a.r = c->r;
+  a.eps = c->cfg.rms_eps;
+  a.gamma = c->cfg.lora_gamma;
+  a.P = std::max(1, std::min(16, c->n_sms / (c->B * c->Hkv)));
+  a.mode = MK_DRAFT;
+  a.rows_max = mk_rows_max(a, c->n_sms);
+  a.n_bound = mk_bounds(a);
+  MkArgs ar = a;
+  ar.mode = MK_AR;
+  a.n_bound = std::max(a.n_bound, mk_bounds(ar));
+  a.n_stages = 0;
+  for (int ns = 12; ns >= 4 && !a.n_stages; --ns)
+    if (mk_smem_bytes(a, ns) <= 227 * 1024) a.n_stages = ns;
+  if (!a.n_stages) return;
+  c->mk_sync_bytes = sizeof(unsigned long long) * c->Kv * c->B + sizeof(int) * (a.n_bound + 1);
+  c->mk_sized = true;
 }
 
 bool init_dims(dvi_ctx* c, const dvi_model_config* cfg, const dvi_runtime_config* rt) {
@@ -865,7 +936,41 @@ bool bu_inline_ok(const dvi_ctx* ctx) {
   return ctx->tc && ctx->r > 0 && ctx->r <= kBuRank && ctx->B <= kBuRows && ctx->d % 128 == 0;
 }
 
+// The draft-phase megakernel: every draft pass with its head (MK_DRAFT,
+// h_k of pass j to verify row j) or the shallow layers of an AR step (MK_AR,
+// h_k to the AR rows that the deep layers read).  Its argmax keys and
+// completion counters are cleared first.
+dvi_status enqueue_mk(dvi_ctx* ctx, int mode) {
+  MkArgs a = ctx->mk;
+  a.mode = mode;
+  if (mode == MK_DRAFT) {
+    a.x_copy = ctx->x_ver;
+    a.copy_row_stride = ctx->Kv;
+    a.ss_copy = ctx->ss_ver;
+    a.ss_copy_ld = ctx->B * ctx->Kv;
+    a.xg_copy = ctx->xg_ver;
+    a.xg_copy_plane = act_plane(ctx, ctx->xg_ver, ctx->d);
+    a.log_enabled = ctx->log_enabled;
+    a.log_u = ctx->log_u;
+    a.log_plane = act_plane(ctx, ctx->log_u, ctx->d);
+    a.zlog = ctx->log_enabled && ctx->rt.head_mode == 0 ? ctx->Z : nullptr;
+  } else {
+    a.x_copy = ctx->x_dr;
+    a.copy_row_stride = 1;
+    a.ss_copy = ctx->ss_dr;
+    a.ss_copy_ld = ctx->B;
+    a.xg_copy = ctx->xg_dr;
+    a.xg_copy_plane = act_plane(ctx, ctx->xg_dr, ctx->d);
+    a.log_enabled = 0;
+  }
+  DVI_CUDA(cudaMemsetAsync(ctx->mk_sync, 0, ctx->mk_sync_bytes, ctx->stream));
+  DVI_CUDA(launch_mk(a, ctx->n_sms, ctx->stream));
+  ctx->launches += 1;
+  return DVI_OK;
+}
+
 dvi_status enqueue_draft(dvi_ctx* ctx) {
+  if (ctx->mk_on) return enqueue_mk(ctx, MK_DRAFT);
   cudaStream_t s = ctx->stream;
   const StepState st = step_state(ctx);
   dvi_status rc;
@@ -1091,6 +1196,46 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
   ctx->layers.assign(weights->layers, weights->layers + cfg->n_layers);
   ctx->w.layers = ctx->layers.data();
   ctx->stream = reinterpret_cast<cudaStream_t>(stream);
+  if (ctx->mk_sized) {
+    MkArgs& a = ctx->mk;
+    for (int l = 0; l < ctx->k; ++l) {
+      const dvi_layer_weights& lw = ctx->layers[l];
+      a.layer[l] = MkLayerW{lw.wq, lw.wk, lw.wv, lw.wo, lw.w_gate, lw.w_up, lw.w_down,
+                            static_cast<const float*>(lw.attn_norm), static_cast<const float*>(lw.ffn_norm)};
+    }
+    a.embed = weights->embed;
+    a.final_norm = static_cast<const float*>(weights->final_norm);
+    a.g_hand = norm_gain_before(ctx, ctx->k);
+    a.w_head = weights->draft_head;
+    a.lora_a = weights->lora_a;
+    a.lora_b = weights->lora_b;
+    a.kc = ctx->kcache;
+    a.vc = ctx->vcache;
+    a.rope = ctx->rope;
+    a.lens = ctx->lens;
+    a.pending = ctx->pending;
+    a.draft_ids = ctx->draft_ids;
+    a.log_step = ctx->log_step;
+    a.log_cap_steps = ctx->cap_steps;
+    a.status = ctx->status;
+    // weight descriptors (16 tiles of 8 rows x 64 per box): [k][wq, wk, wv, wo, wg, wu, wd], then W^S
+    ctx->mk_maps.assign(7 * ctx->k + 1, CUtensorMap{});
+    bool ok = true;
+    for (int l = 0; l < ctx->k && ok; ++l) {
+      const dvi_layer_weights& lw = ctx->layers[l];
+      CUtensorMap* m = ctx->mk_maps.data() + 7 * l;
+      ok = make_weight_map_kblocks(m + 0, lw.wq, ctx->nq, ctx->d, 8, 16) &&
+           make_weight_map_kblocks(m + 1, lw.wk, ctx->nkv, ctx->d, 8, 16) &&
+           make_weight_map_kblocks(m + 2, lw.wv, ctx->nkv, ctx->d, 8, 16) &&
+           make_weight_map_kblocks(m + 3, lw.wo, ctx->d, ctx->nq, 8, 16) &&
+           make_weight_map_kblocks(m + 4, lw.w_gate, ctx->F, ctx->d, 8, 16) &&
+           make_weight_map_kblocks(m + 5, lw.w_up, ctx->F, ctx->d, 8, 16) &&
+           make_weight_map_kblocks(m + 6, lw.w_down, ctx->d, ctx->F, 8, 16);
+    }
+    ok = ok && make_weight_map_kblocks(ctx->mk_maps.data() + 7 * ctx->k, weights->draft_head, ctx->V, ctx->d, 8, 16);
+    a.wmaps = ctx->mk_maps_dev;   // uploaded after the workspace is cleared (below)
+    ctx->mk_on = ok && mk_ctas_per_sm(a) >= 1;
+  }
   if (ctx->tc) {
     auto mk = [&](CUtensorMap* m, const void* p, int rows, int cols) {
       return aligned16(p) && make_weight_map(m, p, rows, cols);
@@ -1133,6 +1278,8 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
   if (cudaMemsetAsync(workspace, 0, ctx->ws_bytes, ctx->stream) != cudaSuccess ||
       cudaMemcpyAsync(ctx->rope, rope.data(), rope.size() * sizeof(float2), cudaMemcpyHostToDevice, ctx->stream) !=
           cudaSuccess ||
+      (ctx->mk_on && cudaMemcpyAsync(ctx->mk_maps_dev, ctx->mk_maps.data(), sizeof(CUtensorMap) * ctx->mk_maps.size(),
+                                     cudaMemcpyHostToDevice, ctx->stream) != cudaSuccess) ||
       (ctx->w_master && launch_master_init(weights->draft_head, ctx->w_master,
                                            static_cast<size_t>(ctx->V) * ctx->d, ctx->stream) != cudaSuccess) ||
       cudaStreamSynchronize(ctx->stream) != cudaSuccess) {
@@ -1325,10 +1472,17 @@ dvi_status dvi_ar_step(dvi_ctx* ctx, int32_t* d_out_ids) {
     StepState st = step_state(ctx);
     st.out_ids = ctx->ar_out;
     DepScope dep(ctx);
-    DVI_CUDA(dep_begin(ctx));
     Pass ps{ctx->x_dr, ctx->ss_dr, ctx->B, ctx->B, 1, 0, ctx->B, 0, ctx->xg_dr, &ctx->map_xg_dr};
-    dvi_status r = enqueue_layers(ctx, 0, ctx->L, ps);
-    if (r != DVI_OK) return r;
+    dvi_status r;
+    if (ctx->mk_on) {
+      // the shallow layers as in a draft pass (same arithmetic: the DVI
+      // stream stays bit-identical to AR), the deep ones as in verify
+      if ((r = enqueue_mk(ctx, MK_AR)) != DVI_OK) return r;
+      if ((r = enqueue_layers(ctx, ctx->k, ctx->L, ps)) != DVI_OK) return r;
+    } else {
+      DVI_CUDA(dep_begin(ctx));
+      if ((r = enqueue_layers(ctx, 0, ctx->L, ps)) != DVI_OK) return r;
+    }
     FinArgs fa{};
     fa.kind = FIN_AR;
     fa.st = st;
@@ -1376,6 +1530,7 @@ dvi_status dvi_get_stats(dvi_ctx* ctx, dvi_stats* out) {
   out->last_accept_rate = ds[9];
   out->device_status = status;
   out->persistent_ctas = ctx->chain_ctas;
+  out->megakernel_ctas = ctx->mk_on ? ctx->n_sms : 0;
   return DVI_OK;
 }
 

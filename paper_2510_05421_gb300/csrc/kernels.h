@@ -93,6 +93,10 @@ void plan_splits(ProjArgs& a, int n_sms, bool tc);
 size_t proj_partial_floats(const ProjArgs& a, bool tc);
 bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols);
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols);   // 64-row boxes (gate/up)
+// W [rows][cols] (cols a multiple of 64) as [cols / 64][rows][64]: a box is
+// `box_kblocks` consecutive tiles of `box_rows` rows x 64 columns, each tile
+// 128-byte swizzled as a 2D box of that shape would be.
+bool make_weight_map_kblocks(CUtensorMap* map, const void* w, int rows, int cols, int box_rows, int box_kblocks);
 bool make_act_map(CUtensorMap* map, const void* act, int rows, int cols);   // [2 planes][rows][cols]
 // The same activation buffer with boxes of `box_rows` (<= 256) rows.
 bool make_act_map_box(CUtensorMap* map, const void* act, int rows, int cols, int box_rows);
@@ -266,6 +270,65 @@ cudaError_t launch_update_grad_a(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_grad_b(const UpdateArgs& a, cudaStream_t s);
 cudaError_t launch_update_full(const UpdateArgs& a, cudaStream_t s);
 // LoRA mode: everything after the logits GEMM in one cooperative launch of
+// ------------------------------------------------------------ draft-phase megakernel
+// One persistent launch (one CTA per SM, every CTA resident) runs the
+// shallow passes of a decode step (Sec. 3.3): the k draft layers of every
+// draft pass with the drafter head, its argmax and the hand-off of h_k to the
+// verify rows (MK_DRAFT), or the k shallow layers of one greedy AR step with
+// the hand-off to the AR rows (MK_AR).  Phases (QKV, attention, O, gate/up,
+// down, head) meet at release/acquire completion counters, one per phase
+// boundary, with bounded polls.  bf16 weights only; at most kMkMaxRows
+// sequences.
+constexpr int kMkMaxLayers = 16;
+constexpr int kMkMaxRows = 2;
+constexpr int kMkMaxGroup = 8;     // query heads per KV head
+enum MkMode : int { MK_DRAFT = 0, MK_AR = 1 };
+struct MkLayerW {
+  const void *wq, *wk, *wv, *wo, *wg, *wu, *wd;   // bf16 [out][in]
+  const float *g_attn, *g_ffn;
+};
+struct MkArgs {
+  MkLayerW layer[kMkMaxLayers];
+  int mode;
+  int B, k, d, Hq, Hkv, hd, F, V, max_len, K, Kv, r;
+  const CUtensorMap* wmaps;   // [k][7] (wq, wk, wv, wo, wg, wu, wd), then W^S: 16 tiles of 8 rows x 64
+  int P;                 // attention position splits per (sequence, KV head)
+  int n_stages;          // weight ring stages of 16 KB
+  int rows_max;          // output rows of one CTA in any phase
+  int n_bound;           // completion counters (the abort flag follows them)
+  float eps, gamma;
+  const void* embed; const float* final_norm; const float* g_hand;
+  const void* w_head; const float* lora_a; const float* lora_b;
+  void* kc; void* vc;    // caches [L][B][H_kv][max_len][hd]; the first k layers are written
+  const float2* rope;
+  const int* lens; const int* pending; int* draft_ids;
+  // hand-off of h_k: residual row, x * g_hand (hi/lo planes), per-tile sums of squares
+  float* x_copy; int copy_row_stride; float* ss_copy; int ss_copy_ld; void* xg_copy; size_t xg_copy_plane;
+  // replay buffer: u (hi/lo planes) and the drafter logits z of the logged tuples
+  void* log_u; size_t log_plane; const int* log_step; int log_cap_steps; int log_enabled;
+  float* zlog;
+  // scratch
+  float* xr;             // [2][B][d] residual stream (double buffered)
+  float* qkv;            // [B][(H_q + 2 H_kv) hd] projections before RoPE
+  float* att;            // [B][H_q][P][hd + 2] attention partials (max, sum, o)
+  float* ao;             // [B][d] output projection
+  float* hbuf;           // [B][F] SwiGLU
+  float* y;              // [B][d] down projection
+  float* bu_part;        // [n_ctas][r] partial B u
+  unsigned long long* keys;   // [Kv][B] argmax keys, zero before the launch
+  int* ctr;              // [n_bound + 1] zero before the launch
+  int* status;
+};
+// Shared memory of the kernel with `n_stages` ring stages (0: too large).
+size_t mk_smem_bytes(const MkArgs& a, int n_stages);
+// Completion counters of one launch.
+int mk_bounds(const MkArgs& a);
+// Output rows of one CTA in the widest phase.
+int mk_rows_max(const MkArgs& a, int n_ctas);
+// CTAs of the kernel one SM holds with a.n_stages ring stages (0: none).
+int mk_ctas_per_sm(const MkArgs& a);
+cudaError_t launch_mk(const MkArgs& a, int n_ctas, cudaStream_t s);
+
 // n_sms CTAs (grid barriers between its phases), when update_fused_ok.
 bool update_fused_ok(const UpdateArgs& a, int n_sms);
 cudaError_t launch_update_fused(const UpdateArgs& a, int n_sms, cudaStream_t s);

@@ -1362,6 +1362,22 @@ bool make_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
 bool make_half_weight_map(CUtensorMap* map, const void* w, int rows, int cols) {
   return make_map(map, w, rows, cols, kGuRows);
 }
+bool make_weight_map_kblocks(CUtensorMap* map, const void* w, int rows, int cols, int box_rows, int box_kblocks) {
+  // W [rows][cols] bf16 seen as [cols / 64][rows][64]: one box is box_kblocks
+  // tiles of box_rows x 64 (each tile 128-byte swizzled, tiles consecutive)
+  auto encode = encoder();
+  if (!encode || cols % kKBlock || box_rows < 1 || box_rows > 256 || box_kblocks < 1 || box_kblocks > 256)
+    return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(kKBlock), static_cast<cuuint64_t>(rows),
+                        static_cast<cuuint64_t>(cols / kKBlock)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(cols) * 2, static_cast<cuuint64_t>(kKBlock) * 2};
+  cuuint32_t box[3] = {kKBlock, static_cast<cuuint32_t>(box_rows), static_cast<cuuint32_t>(box_kblocks)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(w), dims, strides, box,
+                            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
 bool make_act_map_box(CUtensorMap* map, const void* act, int rows, int cols, int box_rows) {
   // two planes (hi, lo) of [rows][cols] bf16, boxes of box_rows rows x 64 columns
   auto encode = encoder();

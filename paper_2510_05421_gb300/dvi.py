@@ -40,7 +40,7 @@ class RuntimeConfig(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int), ("k_spec", ctypes.c_int), ("max_seq_len", ctypes.c_int),
                 ("log_steps", ctypes.c_int), ("head_mode", ctypes.c_int), ("max_prefill_chunk", ctypes.c_int),
                 ("use_graphs", ctypes.c_int), ("bonus", ctypes.c_int), ("persistent", ctypes.c_int),
-                ("chain_counters", ctypes.c_int)]
+                ("chain_counters", ctypes.c_int), ("megakernel", ctypes.c_int)]
 
 
 class LayerWeightsC(ctypes.Structure):
@@ -70,7 +70,8 @@ class StatsC(ctypes.Structure):
                 ("last_loss", ctypes.c_float), ("last_kl", ctypes.c_float), ("last_pg", ctypes.c_float),
                 ("last_ce", ctypes.c_float), ("last_ent", ctypes.c_float), ("last_rl", ctypes.c_float),
                 ("last_kl1", ctypes.c_float), ("last_accept_rate", ctypes.c_float), ("baseline_b", ctypes.c_float),
-                ("update_t", ctypes.c_int), ("device_status", ctypes.c_int), ("persistent_ctas", ctypes.c_int)]
+                ("update_t", ctypes.c_int), ("device_status", ctypes.c_int), ("persistent_ctas", ctypes.c_int),
+                ("megakernel_ctas", ctypes.c_int)]
 
 
 _lib = None
@@ -211,7 +212,8 @@ class DVIEngine:
     def __init__(self, shape, dtype: str, weights: DeviceWeights, *, batch: int, k_spec: int, split_k: int,
                  lora_rank: int, lora_gamma: float = 1.0, max_seq_len: int, log_steps: int,
                  prefill_chunk: int = 0, use_graphs: bool = True, device: int = 0, head_mode: int = 0,
-                 bonus: bool = False, persistent: bool = False, chain_counters: bool = False):
+                 bonus: bool = False, persistent: bool = False, chain_counters: bool = False,
+                 megakernel: bool = False):
         L = lib()
         self.shape, self.dtype, self.w = shape, dtype, weights
         self.B, self.K = batch, k_spec
@@ -222,7 +224,7 @@ class DVIEngine:
                                shape.rope_theta, DVI_BF16 if dtype == "bf16" else DVI_F32)
         self.rt = RuntimeConfig(batch, k_spec, max_seq_len, log_steps, head_mode, prefill_chunk,
                                 1 if use_graphs else 0, 1 if bonus else 0, 1 if persistent else 0,
-                                1 if chain_counters else 0)
+                                1 if chain_counters else 0, 1 if megakernel else 0)
         nbytes = L.dvi_workspace_bytes(ctypes.byref(self.cfg), ctypes.byref(self.rt))
         if nbytes == 0:
             raise DVIError("invalid configuration")

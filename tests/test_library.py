@@ -40,7 +40,7 @@ def _cfgs(w, **rt):
                         w.lora_rank, 1.0, s.rms_eps, s.rope_theta, D.DVI_BF16 if w.dtype == "bf16" else D.DVI_F32)
     base = dict(batch=w.batch, k_spec=w.k_spec, max_seq_len=w.prompt_len[1] + w.gen_tokens + 64,
                 log_steps=w.update_every, head_mode=0, max_prefill_chunk=128, use_graphs=1, bonus=0,
-                persistent=0, chain_counters=0)
+                persistent=0, chain_counters=0, megakernel=0)
     base.update(rt)
     return cfg, D.RuntimeConfig(**base)
 
@@ -59,7 +59,7 @@ def test_workspace_sizes(L, name):
 @pytest.mark.parametrize("bad", [dict(k_spec=0), dict(k_spec=17), dict(batch=0), dict(max_seq_len=3),
                                  dict(log_steps=100), dict(max_prefill_chunk=24), dict(head_mode=2),
                                  dict(bonus=2), dict(k_spec=16, bonus=1), dict(persistent=2),
-                                 dict(chain_counters=2)])
+                                 dict(chain_counters=2), dict(megakernel=2)])
 def test_invalid_runtime_rejected(L, bad):
     cfg, rt = _cfgs(WORKLOADS["tiny"], **bad)
     assert L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt)) == 0
