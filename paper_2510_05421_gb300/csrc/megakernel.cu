@@ -73,6 +73,14 @@ __host__ __device__ __forceinline__ void part_range(int N, int c, int n, int& lo
 }
 __host__ __device__ __forceinline__ int mk_groups(int N) { return (N + kMkGroup - 1) / kMkGroup; }
 __host__ __device__ __forceinline__ int mk_chunks(int K) { return (K + kMkChunk - 1) / kMkChunk; }
+// bf16 elements per plane of the A operand: every phase's K rounded up to
+// whole 1024-column chunks, plus 8 (the planes start 16 bytes apart modulo
+// 128, so one ldmatrix's rows fall in different banks)
+__host__ __device__ __forceinline__ int mk_plane(const MkArgs& a) {
+  int maxK = a.d > a.F ? a.d : a.F;
+  if (a.Hq * a.hd > maxK) maxK = a.Hq * a.hd;
+  return mk_chunks(maxK) * kMkChunk + 8;
+}
 
 // ------------------------------------------------------------------ layout
 struct MkLayout {
@@ -90,13 +98,10 @@ __host__ __device__ inline MkLayout mk_layout(const MkArgs& a, int ns) {
   const int dh = a.d > a.Hq * a.hd ? a.d : a.Hq * a.hd;
   L.act = off;
   off = al16(off + static_cast<size_t>(a.B) * dh * 4);
-  // the MMA's A operand: [K_pad / 2][2 B] words, each the bf16 pair (k, k+1)
-  // of the hi or lo half of one decode row; K_pad covers every phase's K
-  int maxK = a.d > a.F ? a.d : a.F;
-  if (a.Hq * a.hd > maxK) maxK = a.Hq * a.hd;
-  const size_t kpad = static_cast<size_t>(mk_chunks(maxK)) * kMkChunk;
+  // the MMA's A operand: 2 B planes (hi, lo of each decode row) of
+  // mk_plane(a) bf16 each, then 16 zero bytes (the A rows past 2 B)
   L.xw = off;
-  off = al16(off + kpad / 2 * 2 * a.B * 4);
+  off = al16(off + static_cast<size_t>(2 * a.B) * mk_plane(a) * 2 + 16);
   L.wacc = off;
   off = al16(off + static_cast<size_t>(kMkWarps) * a.rows_max * a.B * 4);
   L.gbuf = off;
@@ -228,45 +233,46 @@ namespace {
 // ------------------------------------------------------------------ projections
 // Groups [g0, g1) of 8 weight rows, K columns each: a group's stages are its
 // 1024-column chunks in order.  Warp w multiplies columns [128 w, 128 w + 128)
-// of every stage: per 64-column tile two ldmatrix.x4 (four 8x8 matrices: the
-// B fragments of two k16 steps) and four m16n8k16 MMAs whose A rows are the
-// activations' hi / lo halves (row 2m: hi of decode row m, 2m + 1: lo).  At
-// the group's end the hi and lo rows are added (a shuffle) and the warp's
-// partial sums of the 8 rows go to wacc[warp][row_local][m].  Tiles past K
-// are zero-filled by the copy and meet zero activations.
+// of every stage, 32 columns at a time: one ldmatrix.x4 of the weight tile
+// (the B fragments of two k16 steps), one ldmatrix.x4 of the activation
+// planes (the A fragments of the same two steps: A row p is plane p -- row
+// 2m the hi, 2m + 1 the lo half of decode row m -- and rows past 2 B read
+// zeros), two m16n8k16 MMAs into four independent accumulators.  At the
+// group's end the hi and lo rows are added (a shuffle) and the warp's partial
+// sums of the 8 rows go to wacc[warp][row_local][m].  Tiles past K are
+// zero-filled by the copy and meet zero activations.
 template <int M>
-__device__ __forceinline__ bool gemv_groups(Ring& ring, int K, int g0, int g1, const uint32_t* xw, float* wacc,
+__device__ __forceinline__ bool gemv_groups(Ring& ring, int K, int g0, int g1, uint32_t xa, int plane, float* wacc,
                                             int rows_max, int* status) {
   constexpr int P = 2 * M;
   const int nkc = mk_chunks(K);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane >> 2, t = lane & 3;
   const int lrow = lane & 7, lmat = lane >> 3;
+  // this lane's A row address at column 0 (plane lrow, or the zero block)
+  const uint32_t arow = lrow < P ? xa + static_cast<uint32_t>(lrow * plane * 2 + lmat * 16)
+                                 : xa + static_cast<uint32_t>(P * plane * 2);
+  const uint32_t astep = lrow < P ? 2u : 0u;   // bytes per column (the zero block stays put)
   bool ok = true;
   for (int gi = g0; gi < g1; ++gi) {
-    float d[4][4];   // four independent accumulators (one per 32-column step of a tile pair)
+    float d[4][4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) d[i][0] = d[i][1] = d[i][2] = d[i][3] = 0.f;
     for (int kc = 0; kc < nkc; ++kc) {
       const uint8_t* st = ring_acquire(ring, status, ok);
       if (!ok) return false;
       const uint32_t sb = smem_u32(st) + warp * 2048;
-      const int kw = kc * kMkChunk + warp * 128;
+      const uint32_t ab = arow + astep * static_cast<uint32_t>(kc * kMkChunk + warp * 128);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
-          uint32_t b[4];
+          uint32_t b[4], af[4];
           ldmatrix_x4(b, sb + h * 1024 + lrow * 128 + (((4 * q + lmat) ^ lrow) << 4));
-#pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int kh = (kw + h * 64 + q * 32 + e * 16) >> 1;   // word of the k16 step's first pair
-            uint32_t af[4];
-            af[0] = g < P ? xw[(kh + t) * P + g] : 0u;
-            af[1] = 0u;
-            af[2] = g < P ? xw[(kh + 4 + t) * P + g] : 0u;
-            af[3] = 0u;
-            mma_bf16_16816(d[2 * h + q], af, b[2 * e], b[2 * e + 1]);
-          }
+          ldmatrix_x4(af, ab + astep * static_cast<uint32_t>(h * 64 + q * 32));
+          const uint32_t a0[4] = {af[0], 0u, af[1], 0u};
+          const uint32_t a1[4] = {af[2], 0u, af[3], 0u};
+          mma_bf16_16816(d[2 * h + q], a0, b[0], b[1]);
+          mma_bf16_16816(d[2 * h + q], a1, b[2], b[3]);
         }
       }
       ring_release(ring);
@@ -302,14 +308,14 @@ __device__ __forceinline__ void gemv_finish(float* wacc, int rows_max, int nrows
   cbar();
 }
 
-// The A operand of a projection over K columns: xw[w][2m] and xw[w][2m + 1]
-// hold the hi and lo bf16 pairs of columns (2w, 2w + 1) of row m of src (row
-// stride ld), zero from K to the end of the last 1024-column chunk.
-// `global`: src is in global memory, written by other CTAs in the previous
-// phase (four loads per thread in flight).
+// The A operand of a projection over K columns: plane 2m (hi) and 2m + 1
+// (lo) of row m of src (row stride ld), as bf16 pairs (columns 2w, 2w + 1 in
+// word w of the plane), zero from K to the end of the last 1024-column
+// chunk.  `global`: src is in global memory, written by other CTAs in the
+// previous phase (four loads per thread in flight).
 template <int M>
-__device__ __forceinline__ void mk_pack(uint32_t* xw, const float* src, int K, int ld, bool global) {
-  const int nw = mk_chunks(K) * kMkChunk / 2, kw = K / 2;
+__device__ __forceinline__ void mk_pack(uint32_t* xw, int plane, const float* src, int K, int ld, bool global) {
+  const int nw = mk_chunks(K) * kMkChunk / 2, kw = K / 2, pw = plane / 2;
   for (int w0 = threadIdx.x; w0 < nw; w0 += 4 * kMkCompute) {
     float2 v[4][M];
 #pragma unroll
@@ -332,8 +338,8 @@ __device__ __forceinline__ void mk_pack(uint32_t* xw, const float* src, int K, i
         for (int m = 0; m < M; ++m) {
           uint32_t hi, lo;
           split_bf16x2(v[u][m].x, v[u][m].y, hi, lo);
-          xw[w * 2 * M + 2 * m] = hi;
-          xw[w * 2 * M + 2 * m + 1] = lo;
+          xw[(2 * m) * pw + w] = hi;
+          xw[(2 * m + 1) * pw + w] = lo;
         }
       }
     }
@@ -822,6 +828,8 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
   const int c = blockIdx.x, n = gridDim.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   float* act = reinterpret_cast<float*>(sm + L.act);
   uint32_t* xw = reinterpret_cast<uint32_t*>(sm + L.xw);
+  const int plane = mk_plane(a);
+  const uint32_t xa = smem_u32(xw);
   float* wacc = reinterpret_cast<float*>(sm + L.wacc);
   float* gbuf = reinterpret_cast<float*>(sm + L.gbuf);
   uint8_t* att_sm = sm + L.att;
@@ -878,8 +886,8 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       cur ^= 1;
       mk_rms(a, act, tsum, rstd);
       mk_scale(a, act, rstd, w.g_attn);
-      mk_pack<M>(xw, act, d, d, false);
-      if (!gemv_groups<M>(ring, d, q0, q1, xw, wacc, rows_max, a.status)) {
+      mk_pack<M>(xw, plane, act, d, d, false);
+      if (!gemv_groups<M>(ring, d, q0, q1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
       }
@@ -898,8 +906,8 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       // ---------------- O
       if (!mk_wait(a, bw, flag_s)) return;
       mk_att_combine<HD>(a, act, reinterpret_cast<float*>(att_sm));
-      mk_pack<M>(xw, act, nq, nq, false);
-      if (!gemv_groups<M>(ring, nq, o0, o1, xw, wacc, rows_max, a.status)) {
+      mk_pack<M>(xw, plane, act, nq, nq, false);
+      if (!gemv_groups<M>(ring, nq, o0, o1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
       }
@@ -914,13 +922,13 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       cur ^= 1;
       mk_rms(a, act, tsum, rstd);
       mk_scale(a, act, rstd, w.g_ffn);
-      mk_pack<M>(xw, act, d, d, false);
-      if (!gemv_groups<M>(ring, d, f0, f1, xw, wacc, rows_max, a.status)) {
+      mk_pack<M>(xw, plane, act, d, d, false);
+      if (!gemv_groups<M>(ring, d, f0, f1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
       }
       gemv_finish<M>(wacc, rows_max, (f1 - f0) * kMkGroup, [&](int rl, int m, float v) { gbuf[rl * M + m] = v; });
-      if (!gemv_groups<M>(ring, d, f0, f1, xw, wacc, rows_max, a.status)) {
+      if (!gemv_groups<M>(ring, d, f0, f1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
       }
@@ -932,8 +940,8 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       bw = bn++;
       // ---------------- down
       if (!mk_wait(a, bw, flag_s)) return;
-      mk_pack<M>(xw, a.hbuf, a.F, a.F, true);
-      if (!gemv_groups<M>(ring, a.F, o0, o1, xw, wacc, rows_max, a.status)) {
+      mk_pack<M>(xw, plane, a.hbuf, a.F, a.F, true);
+      if (!gemv_groups<M>(ring, a.F, o0, o1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
       }
@@ -987,8 +995,8 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       mk_signal(a, bn);
       bu_bound = bn++;
     }
-    mk_pack<M>(xw, act, d, d, false);
-    if (!gemv_groups<M>(ring, d, v0, v1, xw, wacc, rows_max, a.status)) {
+    mk_pack<M>(xw, plane, act, d, d, false);
+    if (!gemv_groups<M>(ring, d, v0, v1, xa, plane, wacc, rows_max, a.status)) {
       mk_abort(a);
       return;
     }
@@ -1072,6 +1080,8 @@ __global__ void __launch_bounds__(kMkThreads, 1) mk_kernel(const __grid_constant
   }
   float* wacc = reinterpret_cast<float*>(sm + L.wacc);
   for (int i = tid; i < kMkWarps * a.rows_max * M; i += kMkThreads) wacc[i] = 0.f;
+  // the zero block after the A planes (the A rows past 2 B)
+  if (tid < 4) reinterpret_cast<uint32_t*>(sm + L.xw)[M * mk_plane(a) + tid] = 0u;
   __syncthreads();
   if (tid >= kMkCompute) {
     if (tid == kMkCompute) mk_producer<HD>(a, ring, blockIdx.x, gridDim.x);
