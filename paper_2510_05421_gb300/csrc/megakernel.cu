@@ -570,6 +570,88 @@ __device__ __forceinline__ void mk_scale(const MkArgs& a, float* act, const floa
 namespace dvi {
 namespace {
 
+// The normed input of a projection over d columns in one pass (d <= 4096):
+// x = xa + xb (or the embedding of tok), stored to xr_out by `writer`; the
+// per-128-feature sums of squares (tsum) and 1/rms (rstd); the A planes of
+// x * rstd * g.  Thread tid takes the column pairs tid + 256 e, whose loads
+// (x and gain) are all issued before any is used; a warp's 32 pairs are half
+// a 128-column tile, so the tile sums are two warp sums (hs[m][tile][half]).
+constexpr int kMkPairs = 8;   // column pairs per thread: d <= 512 * kMkPairs
+template <int M>
+__device__ __forceinline__ void mk_norm_pack(const MkArgs& a, const float* __restrict__ xa,
+                                             const float* __restrict__ xb, const int* tok, float* xr_out,
+                                             bool writer, const float* __restrict__ g, uint32_t* xw, int plane,
+                                             float* tsum, float* rstd, float* hs) {
+  const int d = a.d, np = d / 2, nt = d / 128, pw = plane / 2;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  float2 x[M][kMkPairs], gv[kMkPairs];
+#pragma unroll
+  for (int e = 0; e < kMkPairs; ++e) {
+    const int p = tid + e * kMkCompute;
+    gv[e] = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int m = 0; m < M; ++m) x[m][e] = make_float2(0.f, 0.f);
+    if (p < np) {
+      gv[e] = __ldg(reinterpret_cast<const float2*>(g) + p);
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        if (tok) {
+          const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(static_cast<const __nv_bfloat16*>(a.embed) +
+                                                                      static_cast<size_t>(tok[m]) * d) + p);
+          x[m][e] = make_float2(bf16_lo(w), bf16_hi(w));
+        } else {
+          const float2 u = __ldcg(reinterpret_cast<const float2*>(xa + static_cast<size_t>(m) * d) + p);
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(xb + static_cast<size_t>(m) * d) + p);
+          x[m][e] = make_float2(u.x + v.x, u.y + v.y);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < kMkPairs; ++e) {
+    const int p = tid + e * kMkCompute;
+    if (p < np) {
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        if (writer) reinterpret_cast<float2*>(xr_out + static_cast<size_t>(m) * d)[p] = x[m][e];
+        const float sq = warp_sum(fmaf(x[m][e].x, x[m][e].x, x[m][e].y * x[m][e].y));
+        if (lane == 0) hs[(m * nt + (e * kMkCompute + warp * 32) / 64) * 2 + (warp & 1)] = sq;
+      }
+    }
+  }
+  cbar();
+  if (tid < M) {
+    float s = 0.f;
+    for (int t = 0; t < nt; ++t) {
+      const float ts = hs[(tid * nt + t) * 2] + hs[(tid * nt + t) * 2 + 1];
+      tsum[tid * nt + t] = ts;
+      s += ts;
+    }
+    rstd[tid] = rsqrtf(s / static_cast<float>(d) + a.eps);
+  }
+  cbar();
+#pragma unroll
+  for (int e = 0; e < kMkPairs; ++e) {
+    const int p = tid + e * kMkCompute;
+    if (p < np) {
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        const float r = rstd[m];
+        uint32_t hi, lo;
+        split_bf16x2(x[m][e].x * r * gv[e].x, x[m][e].y * r * gv[e].y, hi, lo);
+        xw[(2 * m) * pw + p] = hi;
+        xw[(2 * m + 1) * pw + p] = lo;
+      }
+    }
+  }
+  // zero columns up to the end of the last 1024-column chunk
+  const int nw = mk_chunks(d) * kMkChunk / 2;
+  for (int w = np + tid; w < nw; w += kMkCompute)
+#pragma unroll
+    for (int q = 0; q < 2 * M; ++q) xw[q * pw + w] = 0u;
+  cbar();
+}
+
 // ------------------------------------------------------------------ attention
 // Rows [from, cn) of a K or V chunk stage whose positions were written in
 // this launch (or are the newest one, `fresh`) are copied in from global
@@ -766,11 +848,13 @@ __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& rin
   return true;
 }
 
-// The O phase's input: for every row and query head, the P partials merged
-// (weights exp2(m_p - max) / sum) into act[m][hq * HD + dim].
-template <int HD>
-__device__ __forceinline__ void mk_att_combine(const MkArgs& a, float* act, float* wts) {
-  const int K = a.Hq * HD, P = a.P;
+// The O phase's input: for every row and query head the P partials merged
+// (weights exp2(m_p - max) / sum) and packed straight into the A planes
+// (column pairs of H_q hd; four pairs per thread at a time, all their
+// partials' loads issued together).
+template <int HD, int M>
+__device__ __forceinline__ void mk_att_combine(const MkArgs& a, uint32_t* xw, int plane, float* wts) {
+  const int K = a.Hq * HD, P = a.P, np = K / 2, pw = plane / 2;
   const size_t stride = HD + 2;
   for (int i = threadIdx.x; i < a.B * a.Hq; i += kMkCompute) {
     const float* base = a.att + static_cast<size_t>(i) * P * stride;
@@ -782,31 +866,48 @@ __device__ __forceinline__ void mk_att_combine(const MkArgs& a, float* act, floa
     for (int p = 0; p < P; ++p) wts[i * P + p] = exp2f(__ldcg(base + p * stride) - mx) * inv;
   }
   cbar();
-  // four outputs per thread at a time: their partials' loads go out together
-  for (int m = 0; m < a.B; ++m)
-    for (int e0 = threadIdx.x; e0 < K; e0 += 4 * kMkCompute) {
-      float s[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int q0 = threadIdx.x; q0 < np; q0 += 4 * kMkCompute) {
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      float2 s[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) s[u] = make_float2(0.f, 0.f);
       for (int p = 0; p < P; ++p) {
-        float v[4];
+        float2 v[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const int e = e0 + u * kMkCompute;
-          v[u] = e < K ? __ldcg(a.att + (static_cast<size_t>(m) * a.Hq + e / HD) * P * stride + p * stride + 2 +
-                                e % HD)
-                       : 0.f;
+          const int q = q0 + u * kMkCompute;
+          v[u] = make_float2(0.f, 0.f);
+          if (q < np)
+            v[u] = __ldcg(reinterpret_cast<const float2*>(
+                a.att + ((static_cast<size_t>(m) * a.Hq + (2 * q) / HD) * P + p) * stride + 2 + (2 * q) % HD));
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const int e = e0 + u * kMkCompute;
-          if (e < K) s[u] = fmaf(v[u], wts[(m * a.Hq + e / HD) * P + p], s[u]);
+          const int q = q0 + u * kMkCompute;
+          if (q < np) {
+            const float wgt = wts[(m * a.Hq + (2 * q) / HD) * P + p];
+            s[u].x = fmaf(v[u].x, wgt, s[u].x);
+            s[u].y = fmaf(v[u].y, wgt, s[u].y);
+          }
         }
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const int e = e0 + u * kMkCompute;
-        if (e < K) act[static_cast<size_t>(m) * K + e] = s[u];
+        const int q = q0 + u * kMkCompute;
+        if (q < np) {
+          uint32_t hi, lo;
+          split_bf16x2(s[u].x, s[u].y, hi, lo);
+          xw[(2 * m) * pw + q] = hi;
+          xw[(2 * m + 1) * pw + q] = lo;
+        }
       }
     }
+  }
+  const int nw = mk_chunks(K) * kMkChunk / 2;
+  for (int w = np + threadIdx.x; w < nw; w += kMkCompute)
+#pragma unroll
+    for (int q = 0; q < 2 * M; ++q) xw[q * pw + w] = 0u;
   cbar();
 }
 
@@ -830,9 +931,11 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
   uint32_t* xw = reinterpret_cast<uint32_t*>(sm + L.xw);
   const int plane = mk_plane(a);
   const uint32_t xa = smem_u32(xw);
+  const bool fused = a.d <= 512 * kMkPairs;
   float* wacc = reinterpret_cast<float*>(sm + L.wacc);
   float* gbuf = reinterpret_cast<float*>(sm + L.gbuf);
   uint8_t* att_sm = sm + L.att;
+  float* hs = reinterpret_cast<float*>(att_sm);   // half-tile sums [B][d/128][2] (attention scratch is free then)
   unsigned long long* wkeys = reinterpret_cast<unsigned long long*>(sm + L.misc);   // [8][kMkMaxRows]
   float* rstd = reinterpret_cast<float*>(wkeys + kMkWarps * kMkMaxRows);               // [kMkMaxRows]
   int* tok = reinterpret_cast<int*>(rstd + kMkMaxRows);                                // [kMkMaxRows]
@@ -879,14 +982,18 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
           tok[tid] = t;
         }
         cbar();
-        mk_residual(a, act, nullptr, nullptr, tok, xr[cur ^ 1], c == 0);
+      }
+      if (fused) {
+        mk_norm_pack<M>(a, xr[cur], a.y, l == 0 ? tok : nullptr, xr[cur ^ 1], c == 0, w.g_attn, xw, plane, tsum, rstd,
+                        hs);
       } else {
-        mk_residual(a, act, xr[cur], a.y, nullptr, xr[cur ^ 1], c == 0);
+        if (l == 0) mk_residual(a, act, nullptr, nullptr, tok, xr[cur ^ 1], c == 0);
+        else mk_residual(a, act, xr[cur], a.y, nullptr, xr[cur ^ 1], c == 0);
+        mk_rms(a, act, tsum, rstd);
+        mk_scale(a, act, rstd, w.g_attn);
+        mk_pack<M>(xw, plane, act, d, d, false);
       }
       cur ^= 1;
-      mk_rms(a, act, tsum, rstd);
-      mk_scale(a, act, rstd, w.g_attn);
-      mk_pack<M>(xw, plane, act, d, d, false);
       if (!gemv_groups<M>(ring, d, q0, q1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
@@ -905,8 +1012,7 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       bw = bn++;
       // ---------------- O
       if (!mk_wait(a, bw, flag_s)) return;
-      mk_att_combine<HD>(a, act, reinterpret_cast<float*>(att_sm));
-      mk_pack<M>(xw, plane, act, nq, nq, false);
+      mk_att_combine<HD, M>(a, xw, plane, reinterpret_cast<float*>(att_sm));
       if (!gemv_groups<M>(ring, nq, o0, o1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
@@ -918,11 +1024,15 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       bw = bn++;
       // ---------------- gate / up
       if (!mk_wait(a, bw, flag_s)) return;
-      mk_residual(a, act, xr[cur], a.ao, nullptr, xr[cur ^ 1], c == 0);
+      if (fused) {
+        mk_norm_pack<M>(a, xr[cur], a.ao, nullptr, xr[cur ^ 1], c == 0, w.g_ffn, xw, plane, tsum, rstd, hs);
+      } else {
+        mk_residual(a, act, xr[cur], a.ao, nullptr, xr[cur ^ 1], c == 0);
+        mk_rms(a, act, tsum, rstd);
+        mk_scale(a, act, rstd, w.g_ffn);
+        mk_pack<M>(xw, plane, act, d, d, false);
+      }
       cur ^= 1;
-      mk_rms(a, act, tsum, rstd);
-      mk_scale(a, act, rstd, w.g_ffn);
-      mk_pack<M>(xw, plane, act, d, d, false);
       if (!gemv_groups<M>(ring, d, f0, f1, xa, plane, wacc, rows_max, a.status)) {
         mk_abort(a);
         return;
