@@ -376,12 +376,13 @@ void size_scratch(dvi_ctx* c) {
 
 // The draft-phase megakernel's static arguments and scratch (runtime option
 // megakernel): bf16, at most kMkMaxRows sequences, k <= kMkMaxLayers shallow
-// layers, GQA groups up to kMkMaxGroup, d a multiple of 128, and a ring of at
-// least four 16 KB stages beside the kernel's other shared memory.
+// layers, GQA groups of 1, 2, 4 or 8, d a multiple of 128, d_ffn of 64, and a
+// ring of at least four 16 KB stages beside the kernel's other shared memory.
 void size_mk(dvi_ctx* c) {
   c->mk_sized = false;
   if (!c->tc || !c->rt.megakernel || c->B > kMkMaxRows || c->k > kMkMaxLayers || c->Hq / c->Hkv > kMkMaxGroup ||
-      c->d % 128 || c->F % 64 || (c->hd != 64 && c->hd != 128) || c->B * c->Hkv > c->n_sms)
+      c->d % 128 || c->F % 64 || (c->hd != 64 && c->hd != 128) || c->B * c->Hkv > c->n_sms ||
+      (c->Hq / c->Hkv != 1 && c->Hq / c->Hkv != 2 && c->Hq / c->Hkv != 4 && c->Hq / c->Hkv != 8))
     return;
   MkArgs& a = c->mk;
   a = MkArgs{};

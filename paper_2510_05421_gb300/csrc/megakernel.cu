@@ -48,6 +48,7 @@ constexpr int kMkStageElems = kMkStage / 2;
 constexpr int kMkGroup = 8;          // weight rows per tile (the MMA's N)
 constexpr int kMkChunk = 1024;       // weight columns per stage (16 tiles of 64)
 constexpr int kMkBar = 3;            // named barrier of the compute warps
+constexpr int kMkAttBlock = 8;       // attention key / value chunks per softmax block
 constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ void cbar() { named_bar(kMkBar, kMkCompute); }
@@ -106,11 +107,11 @@ __host__ __device__ inline MkLayout mk_layout(const MkArgs& a, int ns) {
   off = al16(off + static_cast<size_t>(kMkWarps) * a.rows_max * a.B * 4);
   L.gbuf = off;
   off = al16(off + static_cast<size_t>(a.rows_max) * a.B * 4);
-  // attention: q [G][hd], scores [G][CP], part sums [256/hd][G][hd], the new
+  // attention: q [G][hd], scores [G][kMkAttBlock CP], part sums [256/hd][G][hd], the new
   // K and V rows (bf16), running max / sum / correction [G]; the O phase's
   // combine weights [B][H_q][P] reuse it
   const int G = a.Hq / a.Hkv, CP = kMkStageElems / a.hd;
-  size_t att = static_cast<size_t>(G) * a.hd * 4 + static_cast<size_t>(G) * CP * 4 +
+  size_t att = static_cast<size_t>(G) * a.hd * 4 + static_cast<size_t>(G) * kMkAttBlock * CP * 4 +
                static_cast<size_t>(kMkCompute / a.hd) * G * a.hd * 4 + 2 * static_cast<size_t>(a.hd) * 2 +
                3 * static_cast<size_t>(G) * 4;
   const size_t wts = static_cast<size_t>(a.B) * a.Hq * a.P * 4;
@@ -459,12 +460,16 @@ __device__ void mk_producer(const MkArgs& a, Ring& r, int c, int n) {
         ok = group(map, a.d, y);
       }
       if (u.on) {
-        for (int c0 = u.r0; c0 < u.r1 && ok; c0 += CP) {
-          const int cn = min(CP, u.r1 - c0);
-          const uint32_t bytes = static_cast<uint32_t>(att_stable(a, u, c0, cn) * HD * 2);
-          const size_t row = kv_row(a, l, u.b, u.kvh, c0) * HD;
-          ok = kv(static_cast<const __nv_bfloat16*>(a.kc) + row, bytes);
-          if (ok) ok = kv(static_cast<const __nv_bfloat16*>(a.vc) + row, bytes);
+        // per block of kMkAttBlock chunks: its key chunks, then its value chunks
+        for (int b0 = u.r0; b0 < u.r1 && ok; b0 += kMkAttBlock * CP) {
+          const int b1 = min(u.r1, b0 + kMkAttBlock * CP);
+          for (int half = 0; half < 2 && ok; ++half)
+            for (int c0 = b0; c0 < b1 && ok; c0 += CP) {
+              const int cn = min(CP, u.r1 - c0);
+              const uint32_t bytes = static_cast<uint32_t>(att_stable(a, u, c0, cn) * HD * 2);
+              const size_t row = kv_row(a, l, u.b, u.kvh, c0) * HD;
+              ok = kv(static_cast<const __nv_bfloat16*>(half ? a.vc : a.kc) + row, bytes);
+            }
         }
       }
       if (ok) ok = groups(m + 3, a.Hq * HD, o0, o1);
@@ -679,18 +684,21 @@ __device__ __forceinline__ void mk_patch(const MkArgs& a, const void* cache, int
 
 // One attention unit: G query heads of KV head kvh for the decode row of
 // sequence b at position pos, over the unit's range of [0, pos]; writes the
-// partial (running max, sum, o) for the O phase's combine.  Scores use
-// log2-scaled queries (exp2).
-template <int HD>
+// partial (running max, sum, o) for the O phase's combine.  The range is
+// taken in blocks of up to kMkAttBlock chunks of CP positions: the block's
+// key chunks (the scores of all its positions), one online-softmax update,
+// then its value chunks.  Scores use log2-scaled queries (exp2).
+template <int HD, int G>
 __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& ring, uint8_t* att_sm) {
   constexpr int CP = kMkStageElems / HD;   // positions per stage
+  constexpr int BP = kMkAttBlock * CP;     // positions per block
   constexpr int NPART = kMkCompute / HD;   // position interleave of the value loop
+  constexpr int TPP = HD / 32;             // threads per position in the score loop
   constexpr int half = HD / 2;
-  const int G = a.Hq / a.Hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   float* qs = reinterpret_cast<float*>(att_sm);   // [G][HD]
-  float* sc = qs + G * HD;                          // [G][CP]
-  float* osum = sc + G * CP;                        // [NPART][G][HD]
+  float* sc = qs + G * HD;                          // [G][BP]
+  float* osum = sc + G * BP;                        // [NPART][G][HD]
   __nv_bfloat16* kn = reinterpret_cast<__nv_bfloat16*>(osum + NPART * G * HD);   // [HD]
   __nv_bfloat16* vn = kn + HD;
   float* mrun = reinterpret_cast<float*>(vn + HD);  // [G]
@@ -733,67 +741,62 @@ __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& rin
       flag_status(a.status, DVI_DEV_KV_FULL);
     }
   }
-  float o[kMkMaxGroup];
+  float o[G];
 #pragma unroll
-  for (int g = 0; g < kMkMaxGroup; ++g) o[g] = 0.f;
+  for (int g = 0; g < G; ++g) o[g] = 0.f;
   const int part = tid / HD, dim = tid % HD;
+  const int si = tid / TPP, spart = tid % TPP;
   bool ok = true;
-  for (int c0 = u.r0; c0 < u.r1; c0 += CP) {
-    const int cn = min(CP, u.r1 - c0);
-    const int stable = att_stable(a, u, c0, cn);
-    // ---- scores of the chunk's keys
-    uint8_t* st = const_cast<uint8_t*>(ring_acquire(ring, a.status, ok));
-    if (!ok) return false;
-    if (stable < cn) mk_patch<HD>(a, a.kc, l, u, st, c0, stable, cn, kn);
-    {
-      // HD / 32 threads per position, 32 dimensions each (eight 4-element
-      // steps, rotated by the position so the key rows' loads spread over the
-      // banks); the partial dot products meet by shuffles
-      constexpr int TPP = HD / 32;
-      const int i = tid / TPP, part = tid % TPP;
-      float sg[kMkMaxGroup];
+  for (int b0 = u.r0; b0 < u.r1; b0 += BP) {
+    const int bn = min(BP, u.r1 - b0), nch = (bn + CP - 1) / CP;
+    // ---- scores of the block's keys: TPP threads per position, 32
+    // dimensions each (eight 4-element steps, rotated by the position so the
+    // key rows' loads spread over the banks), met by shuffles
+    for (int ch = 0; ch < nch; ++ch) {
+      const int c0 = b0 + ch * CP, cn = min(CP, u.r1 - c0);
+      const int stable = att_stable(a, u, c0, cn);
+      uint8_t* st = const_cast<uint8_t*>(ring_acquire(ring, a.status, ok));
+      if (!ok) return false;
+      if (stable < cn) mk_patch<HD>(a, a.kc, l, u, st, c0, stable, cn, kn);
+      float sg[G];
 #pragma unroll
-      for (int g = 0; g < kMkMaxGroup; ++g) sg[g] = 0.f;
-      if (i < cn) {
-        const __nv_bfloat16* kr = reinterpret_cast<const __nv_bfloat16*>(st) + static_cast<size_t>(i) * HD + part * 32;
+      for (int g = 0; g < G; ++g) sg[g] = 0.f;
+      if (si < cn) {
+        const __nv_bfloat16* kr = reinterpret_cast<const __nv_bfloat16*>(st) + static_cast<size_t>(si) * HD + spart * 32;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const int e2 = (e + i) & 7;
+          const int e2 = (e + si) & 7;
           const uint2 w = *reinterpret_cast<const uint2*>(kr + e2 * 4);
           const float k0 = bf16_lo(w.x), k1 = bf16_hi(w.x), k2 = bf16_lo(w.y), k3 = bf16_hi(w.y);
 #pragma unroll
-          for (int g = 0; g < kMkMaxGroup; ++g) {
-            if (g < G) {
-              const float4 q = *reinterpret_cast<const float4*>(qs + g * HD + part * 32 + e2 * 4);
-              sg[g] = fmaf(q.x, k0, fmaf(q.y, k1, fmaf(q.z, k2, fmaf(q.w, k3, sg[g]))));
-            }
+          for (int g = 0; g < G; ++g) {
+            const float4 q = *reinterpret_cast<const float4*>(qs + g * HD + spart * 32 + e2 * 4);
+            sg[g] = fmaf(q.x, k0, fmaf(q.y, k1, fmaf(q.z, k2, fmaf(q.w, k3, sg[g]))));
           }
         }
       }
 #pragma unroll
-      for (int g = 0; g < kMkMaxGroup; ++g) {
-        if (g < G) {
-          float v = sg[g];
+      for (int g = 0; g < G; ++g) {
+        float v = sg[g];
 #pragma unroll
-          for (int off = 1; off < TPP; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-          if (part == 0 && i < cn) sc[g * CP + i] = v;
-        }
+        for (int off = 1; off < TPP; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if (spart == 0 && si < cn) sc[g * BP + ch * CP + si] = v;
       }
+      ring_release(ring);
     }
-    ring_release(ring);
     cbar();
-    // ---- online softmax over the chunk (one warp per head)
+    // ---- online softmax over the block (one warp per head)
     if (warp < G) {
       const int g = warp;
       float mx = -INFINITY;
-      for (int i = lane; i < cn; i += 32) mx = fmaxf(mx, sc[g * CP + i]);
+      for (int i = lane; i < bn; i += 32) mx = fmaxf(mx, sc[g * BP + i]);
       mx = warp_max(mx);
       const float mo = mrun[g];
       const float mn = fmaxf(mo, mx);
       float sum = 0.f;
-      for (int i = lane; i < cn; i += 32) {
-        const float e = exp2f(sc[g * CP + i] - mn);
-        sc[g * CP + i] = e;
+      for (int i = lane; i < bn; i += 32) {
+        const float e = exp2f(sc[g * BP + i] - mn);
+        sc[g * BP + i] = e;
         sum += e;
       }
       sum = warp_sum(sum);
@@ -806,31 +809,35 @@ __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& rin
     }
     cbar();
     // ---- values
-    st = const_cast<uint8_t*>(ring_acquire(ring, a.status, ok));
-    if (!ok) return false;
-    if (stable < cn) mk_patch<HD>(a, a.vc, l, u, st, c0, stable, cn, vn);
-    const __nv_bfloat16* vs = reinterpret_cast<const __nv_bfloat16*>(st);
 #pragma unroll
-    for (int g = 0; g < kMkMaxGroup; ++g) {
-      if (g < G) {
+    for (int g = 0; g < G; ++g) o[g] *= corr[g];
+    for (int ch = 0; ch < nch; ++ch) {
+      const int c0 = b0 + ch * CP, cn = min(CP, u.r1 - c0);
+      const int stable = att_stable(a, u, c0, cn);
+      uint8_t* st = const_cast<uint8_t*>(ring_acquire(ring, a.status, ok));
+      if (!ok) return false;
+      if (stable < cn) mk_patch<HD>(a, a.vc, l, u, st, c0, stable, cn, vn);
+      const __nv_bfloat16* vs = reinterpret_cast<const __nv_bfloat16*>(st);
+      const float* pb = sc + ch * CP;
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
         // four interleaved partial sums over the chunk's positions
         float t[4] = {0.f, 0.f, 0.f, 0.f};
         int i = part;
         for (; i + 3 * NPART < cn; i += 4 * NPART) {
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            t[q] = fmaf(sc[g * CP + i + q * NPART], __bfloat162float(vs[(i + q * NPART) * HD + dim]), t[q]);
+            t[q] = fmaf(pb[g * BP + i + q * NPART], __bfloat162float(vs[(i + q * NPART) * HD + dim]), t[q]);
         }
-        for (; i < cn; i += NPART) t[0] = fmaf(sc[g * CP + i], __bfloat162float(vs[i * HD + dim]), t[0]);
-        o[g] = fmaf(o[g], corr[g], (t[0] + t[1]) + (t[2] + t[3]));
+        for (; i < cn; i += NPART) t[0] = fmaf(pb[g * BP + i], __bfloat162float(vs[i * HD + dim]), t[0]);
+        o[g] += (t[0] + t[1]) + (t[2] + t[3]);
       }
+      ring_release(ring);
     }
-    ring_release(ring);
-    cbar();
+    cbar();   // the block's scores are read before the next block overwrites them
   }
 #pragma unroll
-  for (int g = 0; g < kMkMaxGroup; ++g)
-    if (g < G) osum[(part * G + g) * HD + dim] = o[g];
+  for (int g = 0; g < G; ++g) osum[(part * G + g) * HD + dim] = o[g];
   cbar();
   const size_t stride = HD + 2;
   for (int i = tid; i < G * HD; i += kMkCompute) {
@@ -846,6 +853,18 @@ __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& rin
     dst[1] = lrun[tid];
   }
   return true;
+}
+
+// The unit's attention for the GQA group size of the model (1, 2, 4 or 8).
+template <int HD>
+__device__ __forceinline__ bool mk_attention_any(const MkArgs& a, int l, const AttUnit& u, Ring& ring,
+                                                 uint8_t* att_sm) {
+  switch (a.Hq / a.Hkv) {
+    case 1: return mk_attention<HD, 1>(a, l, u, ring, att_sm);
+    case 2: return mk_attention<HD, 2>(a, l, u, ring, att_sm);
+    case 4: return mk_attention<HD, 4>(a, l, u, ring, att_sm);
+    default: return mk_attention<HD, 8>(a, l, u, ring, att_sm);
+  }
 }
 
 // The O phase's input: for every row and query head the P partials merged
@@ -1004,7 +1023,7 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       bw = bn++;
       // ---------------- attention
       if (!mk_wait(a, bw, flag_s)) return;
-      if (u.on && !mk_attention<HD>(a, l, u, ring, att_sm)) {
+      if (u.on && !mk_attention_any<HD>(a, l, u, ring, att_sm)) {
         mk_abort(a);
         return;
       }
