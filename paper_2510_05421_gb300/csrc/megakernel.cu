@@ -1131,11 +1131,27 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
     }
     if (r > 0) {
       if (!mk_wait(a, bu_bound, flag_s)) return;
-      for (int q = tid; q < M * r; q += kMkCompute) {
-        const int m = q / r, rr = q % r;
-        float s = 0.f;
-        for (int cc = 0; cc < n; ++cc) s += __ldcg(a.bu_part + (static_cast<size_t>(cc) * M + m) * r + rr);
-        bu[q] = s;
+      // B u = the CTAs' partials summed: 16 lanes per value, each a strided
+      // share of the CTAs (loads in flight together), then a shuffle tree
+      for (int q0 = warp * 2; q0 < M * r; q0 += 2 * kMkWarps) {
+        const int q = q0 + (lane >> 4), sub = lane & 15;
+        float sv = 0.f;
+        if (q < M * r) {
+          const int m = q / r, rr = q % r;
+          float v[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int cc = sub + 16 * i;
+            v[i] = cc < n ? __ldcg(a.bu_part + (static_cast<size_t>(cc) * M + m) * r + rr) : 0.f;
+          }
+          for (int cc = sub + 256; cc < n; cc += 16)
+            v[0] += __ldcg(a.bu_part + (static_cast<size_t>(cc) * M + m) * r + rr);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sv += v[i];
+        }
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, off);
+        if (sub == 0 && q < M * r) bu[q] = sv;
       }
     }
     float* zrow[M];
@@ -1152,7 +1168,27 @@ __device__ void mk_compute(const MkArgs& a, Ring& ring, const MkLayout& L, uint8
       if (r > 0) {
         const float* ar = a.lora_a + static_cast<size_t>(vi) * r;
         float acc = 0.f;
-        for (int q = 0; q < r; ++q) acc = fmaf(ar[q], bu[m * r + q], acc);
+        if ((r & 3) == 0 && (reinterpret_cast<uintptr_t>(a.lora_a) & 15u) == 0) {
+          // the row of A four floats at a time, four loads in flight
+          const int r4 = r >> 2;
+          for (int q0 = 0; q0 < r4; q0 += 4) {
+            float4 av[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if (q0 + q < r4) av[q] = __ldg(reinterpret_cast<const float4*>(ar) + q0 + q);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if (q0 + q < r4) {
+                const float* b4 = bu + m * r + 4 * (q0 + q);
+                acc = fmaf(av[q].x, b4[0], acc);
+                acc = fmaf(av[q].y, b4[1], acc);
+                acc = fmaf(av[q].z, b4[2], acc);
+                acc = fmaf(av[q].w, b4[3], acc);
+              }
+          }
+        } else {
+          for (int q = 0; q < r; ++q) acc = fmaf(ar[q], bu[m * r + q], acc);
+        }
         z = fmaf(a.gamma, acc, z);
       }
       if (zrow[m]) zrow[m][vi] = z;
