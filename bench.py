@@ -324,7 +324,7 @@ def reference_arm(args, w, rank):
     return 0
 
 
-def make_engine(w, dw, max_len, local, persistent=False, megakernel=False):
+def make_engine(w, dw, max_len, local, persistent=False, megakernel=True):
     from paper_2510_05421_gb300 import DVIEngine
     return DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=w.k_spec, split_k=w.split_k,
                      lora_rank=w.lora_rank, lora_gamma=w.lora_gamma, max_seq_len=max_len,
@@ -433,7 +433,7 @@ def extra_workload(name, args, local, dev, pk):
     U, K = w.update_every, w.k_spec
     steps = max(6, args.steps // 2)
     max_len = max(len(p) for p in P) + (args.warmup + steps) * U * K + 2 * K + 64
-    eng = make_engine(w, dw, max_len, local, megakernel=args.megakernel)
+    eng = make_engine(w, dw, max_len, local, megakernel=not args.no_megakernel)
     dP = [torch.from_numpy(p).to(dev) for p in P]
     for b, p in enumerate(dP):
         eng.prefill(b, p)
@@ -463,8 +463,9 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (small profiling cases)")
     ap.add_argument("--prompt", type=int, default=0, help="override the prompt length (small profiling cases)")
-    ap.add_argument("--megakernel", action="store_true",
-                    help="run the draft phase as one persistent launch (runtime option megakernel = 1)")
+    ap.add_argument("--no-megakernel", action="store_true",
+                    help="run the draft phase one kernel per projection, attention and head (runtime option "
+                         "megakernel = 0) instead of one persistent launch")
     ap.add_argument("--persistent", action="store_true",
                     help="run each layer's projections as one persistent launch (runtime option persistent = 1)")
     args = ap.parse_args()
@@ -500,7 +501,7 @@ def main():
     U, K = w.update_every, w.k_spec
     gen_room = max(w.gen_tokens, (args.warmup + args.steps) * U * K)
     max_len = max(len(p) for p in P) + gen_room + 2 * K + 64
-    eng = make_engine(w, dw, max_len, local, args.persistent, args.megakernel)
+    eng = make_engine(w, dw, max_len, local, args.persistent, not args.no_megakernel)
     mk_ctas = eng.stats()["megakernel_ctas"]
     hyper = update_config(w.update)
     # prefill: sequence 0's prompt once to warm up, then every prompt timed
@@ -538,7 +539,7 @@ def main():
     if not args.no_e2e:
         eng.close()
         eng = make_engine(w, dw, max(len(p) for p in P) + w.gen_tokens * K + 64, local, args.persistent,
-                          args.megakernel)
+                          not args.no_megakernel)
         eng.generate(P, 8, update_every=U, hyper=w.update, max_steps=2 * U)
         torch.cuda.synchronize(dev)
         t0 = time.perf_counter()

@@ -213,7 +213,7 @@ class DVIEngine:
                  lora_rank: int, lora_gamma: float = 1.0, max_seq_len: int, log_steps: int,
                  prefill_chunk: int = 0, use_graphs: bool = True, device: int = 0, head_mode: int = 0,
                  bonus: bool = False, persistent: bool = False, chain_counters: bool = False,
-                 megakernel: bool = False):
+                 megakernel: bool = True):
         L = lib()
         self.shape, self.dtype, self.w = shape, dtype, weights
         self.B, self.K = batch, k_spec

@@ -1,4 +1,5 @@
-"""Completion-counter chaining of decode passes (runtime option `chain_counters`).
+"""Completion-counter chaining of decode passes (runtime option `chain_counters`;
+here with the draft phase on the per-kernel path, runtime option megakernel = 0).
 
 With the option, consecutive projection, attention and head launches of a
 bf16 draft pass, verify pass or AR step wait for a per-launch completion
@@ -27,7 +28,7 @@ pytestmark = pytest.mark.gpu
 
 
 def _run(w, W, chain, bonus=False, steps=None):
-    eng, W, dw = engine_for(w, W=W, chain_counters=chain, bonus=bonus)
+    eng, W, dw = engine_for(w, W=W, chain_counters=chain, bonus=bonus, megakernel=False)
     P = make_prompts(w)
     toks, mats, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
     # a last step with logging on and no update after it: the replay buffer
@@ -71,7 +72,7 @@ def test_1b_bit_identical_and_lossless():
     off, _ = _run(w, W, False)
     _same(on, off)
     P = make_prompts(w)
-    eng, _, _ = engine_for(w, W=W, chain_counters=True)
+    eng, _, _ = engine_for(w, W=W, chain_counters=True, megakernel=False)
     ar = eng.generate_ar(P, w.gen_tokens)
     st = eng.stats()
     eng.close()

@@ -5,7 +5,9 @@ step (every draft pass's k layers, the drafter head and its argmax, the
 hand-off of h_k to the verify rows), and the greedy AR step runs its first k
 layers through the same kernel.  Checked through the C-ABI:
 
-* the kernel is in effect (stats: megakernel_ctas > 0) and no wait timed out;
+* the kernel is in effect (stats: megakernel_ctas > 0) and no wait timed out
+  (it is the default for eligible bf16 contexts; the per-kernel draft path,
+  megakernel = 0, is checked the same way on the tiny model);
 * losslessness (Sec. 3.3): the DVI stream equals the GPU's greedy AR stream
   bit for bit with the drafter training online: tiny bf16 (head_dim 128,
   eagerly and with graphs), the bonus row, head_dim 64 with a GQA group of 4,
@@ -31,15 +33,15 @@ from test_gpu_decode import _bf16_case
 pytestmark = pytest.mark.gpu
 
 
-def _lossless(w, W=None, max_seq_len=None, **kw):
+def _lossless(w, W=None, max_seq_len=None, mk=True, **kw):
     P = make_prompts(w)
-    eng, W, _ = engine_for(w, W=W, megakernel=True, max_seq_len=max_seq_len, **kw)
+    eng, W, _ = engine_for(w, W=W, megakernel=mk, max_seq_len=max_seq_len, **kw)
     ar = eng.generate_ar(P, w.gen_tokens)
     st = eng.stats()
     eng.close()
-    assert st["megakernel_ctas"] > 0
+    assert (st["megakernel_ctas"] > 0) == mk
     assert st["device_status"] == 0, st["device_flags"]
-    eng, W, _ = engine_for(w, W=W, megakernel=True, max_seq_len=max_seq_len, **kw)
+    eng, W, _ = engine_for(w, W=W, megakernel=mk, max_seq_len=max_seq_len, **kw)
     toks, mats, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
     st = eng.stats()
     eng.close()
@@ -50,9 +52,9 @@ def _lossless(w, W=None, max_seq_len=None, **kw):
     return W, P, st
 
 
-def _first_step(w, W, P, max_seq_len=None, **kw):
+def _first_step(w, W, P, max_seq_len=None, mk=True, **kw):
     """One logged step of a fresh engine: verify rows, z and u of the buffer."""
-    eng, _, _ = engine_for(w, W=W, megakernel=True, max_seq_len=max_seq_len, **kw)
+    eng, _, _ = engine_for(w, W=W, megakernel=mk, max_seq_len=max_seq_len, **kw)
     toks, _, _, _ = eng.generate(P, 10 ** 6, max_steps=1, log=True)
     eng.sync()
     V = w.shape.vocab
@@ -96,6 +98,13 @@ def test_tiny_bf16_lossless_and_oracle(graphs):
     W, P, st = _lossless(w, use_graphs=graphs)
     assert st["updates"] >= 2
     _check_first_step(w, W, P, use_graphs=graphs)
+
+
+def test_tiny_bf16_per_kernel_draft_path():
+    """The same checks with the draft phase one kernel per projection (megakernel = 0)."""
+    w = _bf16_case()
+    W, P, _ = _lossless(w, mk=False)
+    _check_first_step(w, W, P, mk=False)
 
 
 def test_tiny_bf16_bonus_lossless():

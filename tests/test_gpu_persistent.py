@@ -1,4 +1,5 @@
-"""The persistent projection chain (runtime option `persistent`).
+"""The persistent projection chain (runtime option `persistent`; here with the
+draft phase on the per-kernel path, runtime option megakernel = 0).
 
 With the option, a bf16 decode pass runs each layer's O, gate/up and down
 projections and the next layer's QKV as one persistent launch.  Its CTAs
@@ -34,7 +35,7 @@ def _engine(w, dw, max_seq_len, persistent=True):
     from paper_2510_05421_gb300 import DVIEngine
     return DVIEngine(w.shape, w.dtype, dw, batch=w.batch, k_spec=w.k_spec, split_k=w.split_k,
                      lora_rank=w.lora_rank, lora_gamma=w.lora_gamma, max_seq_len=max_seq_len,
-                     log_steps=w.update_every, persistent=persistent)
+                     log_steps=w.update_every, persistent=persistent, megakernel=False)
 
 
 def _first_step_verify_logits(eng, w, P):
@@ -50,12 +51,12 @@ def _first_step_verify_logits(eng, w, P):
 def test_small_bf16_lossless_and_teacher_forced():
     w = _bf16_case()
     P = make_prompts(w)
-    eng, W, _ = engine_for(w, persistent=True)
+    eng, W, _ = engine_for(w, persistent=True, megakernel=False)
     ar = eng.generate_ar(P, w.gen_tokens)[0]
     st = eng.stats()
     eng.close()
     assert st["persistent_ctas"] > 0
-    eng, W, _ = engine_for(w, W=W, persistent=True)
+    eng, W, _ = engine_for(w, W=W, persistent=True, megakernel=False)
     toks, mats, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
     st = eng.stats()
     eng.close()
@@ -63,7 +64,7 @@ def test_small_bf16_lossless_and_teacher_forced():
     assert st["updates"] >= 2
     assert toks[0] == list(ar)
     assert ((mats >= 0) & (mats <= w.k_spec)).all()
-    eng, _, _ = engine_for(w, W=W, persistent=True)
+    eng, _, _ = engine_for(w, W=W, persistent=True, megakernel=False)
     lg, _ = _first_step_verify_logits(eng, w, P)
     eng.close()
     model = OracleModel(rounded_weights(W), w.shape, w.lora_gamma, kv_dtype="bf16")
@@ -78,10 +79,11 @@ def test_small_bf16_lossless_and_teacher_forced():
 def test_small_bf16_bonus_lossless():
     w = _bf16_case()
     P = make_prompts(w)
-    eng, W, _ = engine_for(w, persistent=True)
+    eng, W, _ = engine_for(w, persistent=True, megakernel=False)
     ar = eng.generate_ar(P, w.gen_tokens)[0]
     eng.close()
-    eng, W, _ = engine_for(w, W=W, bonus=True, persistent=True, max_seq_len=len(P[0]) + 6 * w.gen_tokens + 16)
+    eng, W, _ = engine_for(w, W=W, bonus=True, persistent=True, megakernel=False,
+                           max_seq_len=len(P[0]) + 6 * w.gen_tokens + 16)
     toks, _, _, _ = eng.generate(P, w.gen_tokens, update_every=w.update_every, hyper=w.update)
     st = eng.stats()
     eng.close()
