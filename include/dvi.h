@@ -123,7 +123,8 @@ typedef struct {
                            the same way, so the DVI stream stays bit-identical to AR.  Its
                            projections are row-split GEMVs on f32 activations; its phases
                            meet at completion counters with bounded waits.  Ignored when the
-                           shape or the device does not allow it (stats: megakernel_ctas). */
+                           shape or the device does not allow it, and for max_seq_len above
+                           8192 (stats: megakernel_ctas). */
 } dvi_runtime_config;
 
 typedef struct {

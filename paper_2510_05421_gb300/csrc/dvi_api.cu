@@ -378,11 +378,15 @@ void size_scratch(dvi_ctx* c) {
 // megakernel): bf16, at most kMkMaxRows sequences, k <= kMkMaxLayers shallow
 // layers, GQA groups of 1, 2, 4 or 8, d a multiple of 128, d_ffn of 64, and a
 // ring of at least four 16 KB stages beside the kernel's other shared memory.
+// Its attention runs at most n_sms / (B H_kv) position ranges per KV head, so
+// contexts past kMkMaxContext positions keep the per-kernel draft path, whose
+// decode attention splits every head eight ways (measured faster there).
 void size_mk(dvi_ctx* c) {
   c->mk_sized = false;
   if (!c->tc || !c->rt.megakernel || c->B > kMkMaxRows || c->k > kMkMaxLayers || c->Hq / c->Hkv > kMkMaxGroup ||
       c->d % 128 || c->F % 64 || (c->hd != 64 && c->hd != 128) || c->B * c->Hkv > c->n_sms ||
-      (c->Hq / c->Hkv != 1 && c->Hq / c->Hkv != 2 && c->Hq / c->Hkv != 4 && c->Hq / c->Hkv != 8))
+      (c->Hq / c->Hkv != 1 && c->Hq / c->Hkv != 2 && c->Hq / c->Hkv != 4 && c->Hq / c->Hkv != 8) ||
+      c->max_len > kMkMaxContext)
     return;
   MkArgs& a = c->mk;
   a = MkArgs{};
