@@ -184,8 +184,11 @@ __device__ __forceinline__ bool mk_wait(const MkArgs& a, int i, int* flag_s) {
     const int n = static_cast<int>(gridDim.x);
     volatile int* abort_flag = a.ctr + a.n_bound;
     if (ld_acquire_i32(a.ctr + i) < n) {
+      // the abort flag and the clock only every 64 polls: the counter's
+      // completion is seen one load after it happens
       const uint64_t t0 = global_ns();
-      while (ld_acquire_i32(a.ctr + i) < n) {
+      for (uint32_t it = 1; ld_acquire_i32(a.ctr + i) < n; ++it) {
+        if ((it & 63u) != 0) continue;
         if (*abort_flag) {
           ok = 0;
           break;
