@@ -164,3 +164,38 @@ def test_noalloc_args_rejected_before_any_launch(monkeypatch, case):
     monkeypatch.setattr(D, "lib", no_lib)
     with pytest.raises(ValueError):
         D.linear_noalloc(**_noalloc_args(**over))
+
+
+@pytest.mark.parametrize("name,takes", [("tiny", False), ("1b", True), ("7b", True), ("7b-b8", False),
+                                        ("7b-16k", False)])
+def test_megakernel_workspace(L, name, takes):
+    """The draft-phase megakernel's scratch (residual, projections, attention
+    partials, B u partials, argmax keys, counters, weight descriptors) is
+    reserved exactly for the contexts it takes: bf16, at most 2 sequences,
+    d_ffn a multiple of 64, max_seq_len <= 8192 (tiny: f32; 7b-b8: 8
+    sequences; 7b-16k: a 16K context)."""
+    w = WORKLOADS[name]
+    cfg, rt0 = _cfgs(w, megakernel=0)
+    _, rt1 = _cfgs(w, megakernel=1)
+    if name == "7b-16k":
+        rt0.max_seq_len = rt1.max_seq_len = 16384 + 256
+    n0 = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt0))
+    n1 = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt1))
+    assert n0 > 0 and n1 > 0
+    if not takes:
+        assert n1 == n0
+        return
+    s = w.shape
+    nqkv = (s.n_heads + 2 * s.n_kv_heads) * s.head_dim
+    floats = w.batch * (2 * s.d_model + nqkv + 2 * s.d_model + s.d_ffn)   # xr[2], qkv, ao, y, h
+    assert n0 + 4 * floats < n1 < n0 + (64 << 20)
+
+
+def test_megakernel_bf16_small_ffn_not_taken(L):
+    """d_ffn must be a multiple of 64 (the weight boxes tile K in 64 columns)."""
+    w = WORKLOADS["tiny"].with_(dtype="bf16")
+    cfg, rt0 = _cfgs(w, megakernel=0)
+    _, rt1 = _cfgs(w, megakernel=1)
+    assert w.shape.d_ffn % 64 != 0
+    assert L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt1)) == \
+        L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt0))
