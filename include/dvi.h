@@ -115,16 +115,17 @@ typedef struct {
                            bit-identical results. */
   int megakernel;       /* 0: the draft passes run one kernel per projection, attention and
                            head.  1: bf16 contexts of at most 2 sequences with k <= 16 draft
-                           layers (GQA groups <= 8, head_dim 64 or 128, d a multiple of 128)
+                           layers (GQA groups of 1, 2, 4 or 8 -- 8 at head_dim 64 only --,
+                           head_dim 64 or 128, d a multiple of 128)
                            run the whole draft phase -- every draft pass's k layers, the
                            drafter head with its argmax, the hand-off of h_k to the verify
                            rows -- as one persistent launch of one CTA per SM (Sec. 3.3
                            draft rollout), and the greedy AR step runs its first k layers
                            the same way, so the DVI stream stays bit-identical to AR.  Its
-                           projections are row-split GEMVs on f32 activations; its phases
+                           projections are row-split GEMVs on f32 activations and its
+                           attention runs on warp MMAs (online softmax per warp); its phases
                            meet at completion counters with bounded waits.  Ignored when the
-                           shape or the device does not allow it, and for max_seq_len above
-                           8192 (stats: megakernel_ctas). */
+                           shape or the device does not allow it (stats: megakernel_ctas). */
 } dvi_runtime_config;
 
 typedef struct {

@@ -12,6 +12,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <limits>
 #include <string>
 #include <vector>
 
@@ -281,7 +282,7 @@ size_t layout(dvi_ctx* c, char* base) {
     a.y = reinterpret_cast<float*>(take(sizeof(float) * B * d));
     a.bu_part = reinterpret_cast<float*>(take(sizeof(float) * c->n_sms * B * (r > 0 ? r : 1)));
     c->mk_sync = take(c->mk_sync_bytes);
-    c->mk_maps_dev = reinterpret_cast<CUtensorMap*>(take(sizeof(CUtensorMap) * (7 * c->k + 1)));
+    c->mk_maps_dev = reinterpret_cast<CUtensorMap*>(take(sizeof(CUtensorMap) * (7 * c->k + 3)));
     a.keys = reinterpret_cast<unsigned long long*>(c->mk_sync);
     a.ctr = c->mk_sync ? reinterpret_cast<int*>(static_cast<char*>(c->mk_sync) +
                                                 sizeof(unsigned long long) * c->Kv * B)
@@ -376,17 +377,19 @@ void size_scratch(dvi_ctx* c) {
 
 // The draft-phase megakernel's static arguments and scratch (runtime option
 // megakernel): bf16, at most kMkMaxRows sequences, k <= kMkMaxLayers shallow
-// layers, GQA groups of 1, 2, 4 or 8, d a multiple of 128, d_ffn of 64, and a
-// ring of at least four 16 KB stages beside the kernel's other shared memory.
-// Its attention runs at most n_sms / (B H_kv) position ranges per KV head, so
-// contexts past kMkMaxContext positions keep the per-kernel draft path, whose
-// decode attention splits every head eight ways (measured faster there).
+// layers, GQA groups of 1, 2, 4 or 8 (8 only at head_dim 64), d a multiple of
+// 128, d_ffn of 64, fewer than 2^31 cache rows (its KV boxes take a 32-bit
+// row), and a ring of at least four 16 KB stages beside the kernel's other
+// shared memory.  No context bound: its attention streams each unit's range
+// at the ring's pace (measured ahead of the per-kernel draft path from 1K to
+// 16K positions).
 void size_mk(dvi_ctx* c) {
   c->mk_sized = false;
   if (!c->tc || !c->rt.megakernel || c->B > kMkMaxRows || c->k > kMkMaxLayers || c->Hq / c->Hkv > kMkMaxGroup ||
       c->d % 128 || c->F % 64 || (c->hd != 64 && c->hd != 128) || c->B * c->Hkv > c->n_sms ||
       (c->Hq / c->Hkv != 1 && c->Hq / c->Hkv != 2 && c->Hq / c->Hkv != 4 && c->Hq / c->Hkv != 8) ||
-      c->max_len > kMkMaxContext)
+      (c->hd == 128 && c->Hq / c->Hkv == 8) ||
+      static_cast<long long>(c->L) * c->B * c->Hkv * c->max_len > std::numeric_limits<int>::max())
     return;
   MkArgs& a = c->mk;
   a = MkArgs{};
@@ -1223,8 +1226,9 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
     a.log_step = ctx->log_step;
     a.log_cap_steps = ctx->cap_steps;
     a.status = ctx->status;
-    // weight descriptors (16 tiles of 8 rows x 64 per box): [k][wq, wk, wv, wo, wg, wu, wd], then W^S
-    ctx->mk_maps.assign(7 * ctx->k + 1, CUtensorMap{});
+    // weight descriptors (16 tiles of 8 rows x 64 per box): [k][wq, wk, wv, wo, wg, wu, wd], then W^S,
+    // then the K and V caches (16 KB boxes: hd / 64 tiles of 8192 / hd rows x 64)
+    ctx->mk_maps.assign(7 * ctx->k + 3, CUtensorMap{});
     bool ok = true;
     for (int l = 0; l < ctx->k && ok; ++l) {
       const dvi_layer_weights& lw = ctx->layers[l];
@@ -1238,6 +1242,12 @@ dvi_status dvi_create(const dvi_model_config* cfg, const dvi_runtime_config* rt,
            make_weight_map_kblocks(m + 6, lw.w_down, ctx->d, ctx->F, 8, 16);
     }
     ok = ok && make_weight_map_kblocks(ctx->mk_maps.data() + 7 * ctx->k, weights->draft_head, ctx->V, ctx->d, 8, 16);
+    const int kv_rows = static_cast<int>(static_cast<long long>(ctx->L) * ctx->B * ctx->Hkv * ctx->max_len);
+    const int kv_box = 8192 / ctx->hd;
+    ok = ok && make_weight_map_kblocks(ctx->mk_maps.data() + 7 * ctx->k + 1, ctx->kcache, kv_rows, ctx->hd, kv_box,
+                                       ctx->hd / 64) &&
+         make_weight_map_kblocks(ctx->mk_maps.data() + 7 * ctx->k + 2, ctx->vcache, kv_rows, ctx->hd, kv_box,
+                                 ctx->hd / 64);
     a.wmaps = ctx->mk_maps_dev;   // uploaded after the workspace is cleared (below)
     ctx->mk_on = ok && mk_ctas_per_sm(a) >= 1;
   }

@@ -282,7 +282,6 @@ cudaError_t launch_update_full(const UpdateArgs& a, cudaStream_t s);
 constexpr int kMkMaxLayers = 16;
 constexpr int kMkMaxRows = 2;
 constexpr int kMkMaxGroup = 8;     // query heads per KV head
-constexpr int kMkMaxContext = 8192; // max_seq_len beyond which the per-kernel draft path runs
 enum MkMode : int { MK_DRAFT = 0, MK_AR = 1 };
 struct MkLayerW {
   const void *wq, *wk, *wv, *wo, *wg, *wu, *wd;   // bf16 [out][in]

@@ -48,7 +48,6 @@ constexpr int kMkStageElems = kMkStage / 2;
 constexpr int kMkGroup = 8;          // weight rows per tile (the MMA's N)
 constexpr int kMkChunk = 1024;       // weight columns per stage (16 tiles of 64)
 constexpr int kMkBar = 3;            // named barrier of the compute warps
-constexpr int kMkAttBlock = 8;       // attention key / value chunks per softmax block
 constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ void cbar() { named_bar(kMkBar, kMkCompute); }
@@ -84,6 +83,17 @@ __host__ __device__ __forceinline__ int mk_plane(const MkArgs& a) {
 }
 
 // ------------------------------------------------------------------ layout
+// Bytes of the attention scratch (per unit): the q fragments of the lanes
+// with live A rows [hd / 16][min(32, 8 G)] x 16 B and the new K and V rows
+// (bf16); at the unit's end the warps' partial o [8][G][hd] f32 and (max,
+// sum) [8][G][2] f32 overlay them.
+__host__ __device__ __forceinline__ size_t mk_att_bytes(int G, int hd) {
+  const size_t ql = 8 * G < 32 ? 8 * G : 32;
+  const size_t in = static_cast<size_t>(hd / 16) * ql * 16 + 2 * static_cast<size_t>(hd) * 2;
+  const size_t out = static_cast<size_t>(kMkWarps) * G * hd * 4 + static_cast<size_t>(kMkWarps) * G * 2 * 4;
+  return in > out ? in : out;
+}
+
 struct MkLayout {
   size_t ring, bars, act, xw, wacc, gbuf, att, misc, total;
 };
@@ -107,13 +117,9 @@ __host__ __device__ inline MkLayout mk_layout(const MkArgs& a, int ns) {
   off = al16(off + static_cast<size_t>(kMkWarps) * a.rows_max * a.B * 4);
   L.gbuf = off;
   off = al16(off + static_cast<size_t>(a.rows_max) * a.B * 4);
-  // attention: q [G][hd], scores [G][kMkAttBlock CP], part sums [256/hd][G][hd], the new
-  // K and V rows (bf16), running max / sum / correction [G]; the O phase's
-  // combine weights [B][H_q][P] reuse it
-  const int G = a.Hq / a.Hkv, CP = kMkStageElems / a.hd;
-  size_t att = static_cast<size_t>(G) * a.hd * 4 + static_cast<size_t>(G) * kMkAttBlock * CP * 4 +
-               static_cast<size_t>(kMkCompute / a.hd) * G * a.hd * 4 + 2 * static_cast<size_t>(a.hd) * 2 +
-               3 * static_cast<size_t>(G) * 4;
+  // attention scratch (mk_att_bytes); the O phase's combine weights
+  // [B][H_q][P] reuse it
+  const size_t att = mk_att_bytes(a.Hq / a.Hkv, a.hd);
   const size_t wts = static_cast<size_t>(a.B) * a.Hq * a.P * 4;
   L.att = off;
   off = al16(off + (att > wts ? att : wts));
@@ -432,16 +438,15 @@ __device__ void mk_producer(const MkArgs& a, Ring& r, int c, int n) {
       if (!group(map, K, gi * kMkGroup)) return false;
     return true;
   };
-  // cached K or V rows (a 1D bulk copy; a chunk with nothing stable completes empty)
-  auto kv = [&](const void* src, uint32_t bytes) -> bool {
+  // CP cached K or V rows from `row` on: one box of the cache's 3D map
+  // ([hd / 64][rows][64], 128-byte swizzled tiles of CP rows x 64; rows past
+  // the cache are zero-filled and counted)
+  const uint64_t kv_pol = l2_evict_normal_policy();
+  auto kv = [&](const CUtensorMap* map, int row) -> bool {
     int s;
     if (!take(s)) return false;
-    if (bytes) {
-      mbar_arrive_expect_tx(&r.full[s], bytes);
-      bulk_load(r.base + static_cast<size_t>(s) * kMkStage, src, bytes, &r.full[s]);
-    } else {
-      mbar_arrive(&r.full[s]);
-    }
+    mbar_arrive_expect_tx(&r.full[s], static_cast<uint32_t>(kMkStage));
+    tma_load_3d(r.base + static_cast<size_t>(s) * kMkStage, map, 0, row, 0, &r.full[s], kv_pol);
     ++it;
     return true;
   };
@@ -463,16 +468,10 @@ __device__ void mk_producer(const MkArgs& a, Ring& r, int c, int n) {
         ok = group(map, a.d, y);
       }
       if (u.on) {
-        // per block of kMkAttBlock chunks: its key chunks, then its value chunks
-        for (int b0 = u.r0; b0 < u.r1 && ok; b0 += kMkAttBlock * CP) {
-          const int b1 = min(u.r1, b0 + kMkAttBlock * CP);
-          for (int half = 0; half < 2 && ok; ++half)
-            for (int c0 = b0; c0 < b1 && ok; c0 += CP) {
-              const int cn = min(CP, u.r1 - c0);
-              const uint32_t bytes = static_cast<uint32_t>(att_stable(a, u, c0, cn) * HD * 2);
-              const size_t row = kv_row(a, l, u.b, u.kvh, c0) * HD;
-              ok = kv(static_cast<const __nv_bfloat16*>(half ? a.vc : a.kc) + row, bytes);
-            }
+        // per chunk: its keys, then its values
+        for (int c0 = u.r0; c0 < u.r1 && ok; c0 += CP) {
+          const int row = static_cast<int>(kv_row(a, l, u.b, u.kvh, c0));
+          ok = kv(a.wmaps + a.k * 7 + 1, row) && kv(a.wmaps + a.k * 7 + 2, row);
         }
       }
       if (ok) ok = groups(m + 3, a.Hq * HD, o0, o1);
@@ -661,13 +660,21 @@ __device__ __forceinline__ void mk_norm_pack(const MkArgs& a, const float* __res
 }
 
 // ------------------------------------------------------------------ attention
+// A K or V stage holds CP cache rows as hd / 64 tiles of CP rows x 64
+// (one 3D box, 128-byte swizzled): the 16-byte chunk j of row i.
+template <int HD>
+__device__ __forceinline__ uint32_t kv_off(int i, int j) {
+  constexpr int CP = kMkStageElems / HD;
+  return static_cast<uint32_t>((j >> 3) * CP * 128 + i * 128 + (((j & 7) ^ (i & 7)) << 4));
+}
+
 // Rows [from, cn) of a K or V chunk stage whose positions were written in
 // this launch (or are the newest one, `fresh`) are copied in from global
-// memory, then ordered before the stage's next bulk write.
+// memory, then ordered before the stage's next asynchronous write.
 template <int HD>
 __device__ __forceinline__ void mk_patch(const MkArgs& a, const void* cache, int l, const AttUnit& u, uint8_t* st,
                                          int c0, int from, int cn, const __nv_bfloat16* fresh) {
-  constexpr int V16 = HD / 8;   // 16-byte vectors per row
+  constexpr int V16 = HD / 8;   // 16-byte chunks per row
   for (int e = threadIdx.x; e < (cn - from) * V16; e += kMkCompute) {
     const int i = from + e / V16, q = e % V16;
     const int x = c0 + i;
@@ -679,57 +686,93 @@ __device__ __forceinline__ void mk_patch(const MkArgs& a, const void* cache, int
     else
       v = __ldcg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(cache) +
                                                 kv_row(a, l, u.b, u.kvh, x) * HD) + q);
-    reinterpret_cast<uint4*>(st + static_cast<size_t>(i) * HD * 2)[q] = v;
+    *reinterpret_cast<uint4*>(st + kv_off<HD>(i, q)) = v;
   }
   fence_proxy_async_smem();
   cbar();
 }
 
+// D (16x8 f32) += A (16x8 bf16, row) . B (8x8 bf16, col), one warp.
+__device__ __forceinline__ void mma_bf16_1688(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t b0) {
+  asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, {%0,%1,%2,%3};"
+               : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+               : "r"(a0), "r"(a1), "r"(b0));
+}
+
+// The halves of a bf16 pair at chunk positions p, p + 1 that lie below cn.
+__device__ __forceinline__ uint32_t kv_mask(uint32_t v, int p, int cn) {
+  return (p < cn ? v & 0xffffu : 0u) | (p + 1 < cn ? v & 0xffff0000u : 0u);
+}
+
 // One attention unit: G query heads of KV head kvh for the decode row of
 // sequence b at position pos, over the unit's range of [0, pos]; writes the
-// partial (running max, sum, o) for the O phase's combine.  The range is
-// taken in blocks of up to kMkAttBlock chunks of CP positions: the block's
-// key chunks (the scores of all its positions), one online-softmax update,
-// then its value chunks.  Scores use log2-scaled queries (exp2).
+// partial (running max, sum, o) for the O phase's combine.
+//
+// Both products run on the tensor cores (warp MMA, f32 accumulation) with the
+// stage's CP positions split over the 8 warps, PW each.  Scores: A row 2 h
+// is the bf16 hi part of query head h (pre-scaled by log2(e) / sqrt(hd), so
+// the softmax uses exp2), row 2 h + 1 its lo part (heads 4..7 in rows
+// 8..15); B is the warp's key rows (ldmatrix); a score is its hi row plus its
+// lo row (lanes g and g ^ 1).  Each warp keeps its own online softmax (max,
+// sum and o in registers), updated once per chunk: the chunk's key stage,
+// the update, then its value stage as o^T += V^T p^T with A = the warp's
+// value rows (ldmatrix.trans, 16 dimensions an m-tile) and B = the
+// probabilities, column 2 h the hi part of head h and 2 h + 1 its lo part (a
+// lane's scores are already where the B fragment wants them).  The 8 warps'
+// partials are merged at the end.  Positions past the range get probability 0
+// and their value rows are masked to 0.  The chunk loop is not unrolled
+// (compact code: the phase runs after the projections' code has filled the
+// instruction cache).
 template <int HD, int G>
 __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& ring, uint8_t* att_sm) {
   constexpr int CP = kMkStageElems / HD;   // positions per stage
-  constexpr int BP = kMkAttBlock * CP;     // positions per block
-  constexpr int NPART = kMkCompute / HD;   // position interleave of the value loop
-  constexpr int TPP = HD / 32;             // threads per position in the score loop
+  constexpr int PW = CP / kMkWarps;        // positions per warp and stage
+  constexpr int NT = PW / 8;               // score n-tiles per warp
+  constexpr int KS = HD / 16;              // k16 steps of a score
+  constexpr int MT = HD / 16;              // m-tiles of o^T
+  constexpr int NH = G > 4 ? 2 : 1;        // head tiles (4 heads: hi, lo columns)
   constexpr int half = HD / 2;
+  static_assert(NT == 1 || NT == 2, "8 or 16 positions per warp and stage");
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  float* qs = reinterpret_cast<float*>(att_sm);   // [G][HD]
-  float* sc = qs + G * HD;                          // [G][BP]
-  float* osum = sc + G * BP;                        // [NPART][G][HD]
-  __nv_bfloat16* kn = reinterpret_cast<__nv_bfloat16*>(osum + NPART * G * HD);   // [HD]
+  const int g = lane >> 2, c = lane & 3, lrow = lane & 7, lmat = lane >> 3;
+  constexpr int QL = 8 * G < 32 ? 8 * G : 32;   // lanes with live A rows (g < 2 G)
+  uint4* qf = reinterpret_cast<uint4*>(att_sm);                         // [KS][QL]
+  __nv_bfloat16* kn = reinterpret_cast<__nv_bfloat16*>(qf + KS * QL);   // [HD]
   __nv_bfloat16* vn = kn + HD;
-  float* mrun = reinterpret_cast<float*>(vn + HD);  // [G]
-  float* lrun = mrun + G;
-  float* corr = lrun + G;
 
   const float* qrow = a.qkv + static_cast<size_t>(u.b) * (a.Hq + 2 * a.Hkv) * HD;
   const bool pos_ok = u.pos < a.max_len;
   const int rp = pos_ok ? u.pos : a.max_len - 1;
+  const float2* rope = a.rope + static_cast<size_t>(rp) * half;
   const float qscale = kLog2e * rsqrtf(static_cast<float>(HD));
-  for (int i = tid; i < G * HD; i += kMkCompute) {
-    const int g = i / HD, dim = i % HD;
-    const float* qh = qrow + static_cast<size_t>(u.kvh * G + g) * HD;
-    const float v = __ldcg(qh + dim), vp = __ldcg(qh + (dim < half ? dim + half : dim - half));
-    const float2 cs = a.rope[static_cast<size_t>(rp) * half + dim % half];
-    qs[i] = (dim < half ? v * cs.x - vp * cs.y : v * cs.x + vp * cs.y) * qscale;
+  // dimension dim of head row h of this row's q | k after RoPE
+  auto rot = [&](int h, int dim) {
+    const float* x = qrow + static_cast<size_t>(h) * HD;
+    const float v = __ldcg(x + dim), vp = __ldcg(x + (dim < half ? dim + half : dim - half));
+    const float2 cs = rope[dim % half];
+    return dim < half ? v * cs.x - vp * cs.y : v * cs.x + vp * cs.y;
+  };
+  // the A fragment of lane (gg, cc) for k-step ks: rows gg and gg + 8
+  for (int i = tid; i < KS * QL; i += kMkCompute) {
+    const int ks = i / QL, gg = (i % QL) >> 2, cc = i & 3;
+    uint32_t f[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int row = gg + 8 * r, hq = row >> 1;
+      if (hq < G) {
+        const int h = u.kvh * G + hq, d0 = 16 * ks + 2 * cc;
+        uint32_t hi0, lo0, hi1, lo1;
+        split_bf16x2(rot(h, d0) * qscale, rot(h, d0 + 1) * qscale, hi0, lo0);
+        split_bf16x2(rot(h, d0 + 8) * qscale, rot(h, d0 + 9) * qscale, hi1, lo1);
+        f[r] = row & 1 ? lo0 : hi0;
+        f[2 + r] = row & 1 ? lo1 : hi1;
+      }
+    }
+    qf[i] = make_uint4(f[0], f[1], f[2], f[3]);
   }
   for (int dim = tid; dim < HD; dim += kMkCompute) {
-    const float* kh = qrow + static_cast<size_t>(a.Hq + u.kvh) * HD;
-    const float* vh = qrow + static_cast<size_t>(a.Hq + a.Hkv + u.kvh) * HD;
-    const float v = __ldcg(kh + dim), vp = __ldcg(kh + (dim < half ? dim + half : dim - half));
-    const float2 cs = a.rope[static_cast<size_t>(rp) * half + dim % half];
-    kn[dim] = __float2bfloat16_rn(dim < half ? v * cs.x - vp * cs.y : v * cs.x + vp * cs.y);
-    vn[dim] = __float2bfloat16_rn(__ldcg(vh + dim));
-  }
-  if (tid < G) {
-    mrun[tid] = -INFINITY;
-    lrun[tid] = 0.f;
+    kn[dim] = __float2bfloat16_rn(rot(a.Hq + u.kvh, dim));
+    vn[dim] = __float2bfloat16_rn(__ldcg(qrow + static_cast<size_t>(a.Hq + a.Hkv + u.kvh) * HD + dim));
   }
   cbar();
   // the newest position into the cache (the unit whose range ends at pos)
@@ -744,116 +787,177 @@ __device__ bool mk_attention(const MkArgs& a, int l, const AttUnit& u, Ring& rin
       flag_status(a.status, DVI_DEV_KV_FULL);
     }
   }
-  float o[G];
+  // lane (g, c) tracks heads g / 2 + 4 h (h < NH) for the softmax and holds
+  // o^T of heads c + 4 h at dimensions 16 m + g and 16 m + g + 8
+  float o[MT][NH][4];
 #pragma unroll
-  for (int g = 0; g < G; ++g) o[g] = 0.f;
-  const int part = tid / HD, dim = tid % HD;
-  const int si = tid / TPP, spart = tid % TPP;
+  for (int m = 0; m < MT; ++m)
+#pragma unroll
+    for (int h = 0; h < NH; ++h) o[m][h][0] = o[m][h][1] = o[m][h][2] = o[m][h][3] = 0.f;
+  float mrun[NH], lrun[NH];
+#pragma unroll
+  for (int h = 0; h < NH; ++h) {
+    mrun[h] = -INFINITY;
+    lrun[h] = 0.f;
+  }
+  const int pw0 = warp * PW;   // the warp's first position in a chunk
+  // the lane's q fragments, held for the whole range
+  uint32_t qa[KS][4];
+#pragma unroll
+  for (int ks = 0; ks < KS; ++ks) {
+    const uint4 v = lane < QL ? qf[ks * QL + lane] : make_uint4(0u, 0u, 0u, 0u);
+    qa[ks][0] = v.x;
+    qa[ks][1] = v.y;
+    qa[ks][2] = v.z;
+    qa[ks][3] = v.w;
+  }
   bool ok = true;
-  for (int b0 = u.r0; b0 < u.r1; b0 += BP) {
-    const int bn = min(BP, u.r1 - b0), nch = (bn + CP - 1) / CP;
-    // ---- scores of the block's keys: TPP threads per position, 32
-    // dimensions each (eight 4-element steps, rotated by the position so the
-    // key rows' loads spread over the banks), met by shuffles
-    for (int ch = 0; ch < nch; ++ch) {
-      const int c0 = b0 + ch * CP, cn = min(CP, u.r1 - c0);
-      const int stable = att_stable(a, u, c0, cn);
+#pragma unroll 1
+  for (int c0 = u.r0; c0 < u.r1; c0 += CP) {
+    const int cn = min(CP, u.r1 - c0);
+    const int stable = att_stable(a, u, c0, cn);
+    // ---- scores of the chunk's keys: lane (g, c) gets its heads at the
+    // positions pw0 + 8 t + 2 c + {0, 1} (two accumulators: even and odd k16 steps)
+    float s[NT][NH][2];
+    {
       uint8_t* st = const_cast<uint8_t*>(ring_acquire(ring, a.status, ok));
       if (!ok) return false;
       if (stable < cn) mk_patch<HD>(a, a.kc, l, u, st, c0, stable, cn, kn);
-      float sg[G];
+      const uint32_t sb = smem_u32(st);
 #pragma unroll
-      for (int g = 0; g < G; ++g) sg[g] = 0.f;
-      if (si < cn) {
-        const __nv_bfloat16* kr = reinterpret_cast<const __nv_bfloat16*>(st) + static_cast<size_t>(si) * HD + spart * 32;
+      for (int t = 0; t < NT; ++t) {
+        float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int e2 = (e + si) & 7;
-          const uint2 w = *reinterpret_cast<const uint2*>(kr + e2 * 4);
-          const float k0 = bf16_lo(w.x), k1 = bf16_hi(w.x), k2 = bf16_lo(w.y), k3 = bf16_hi(w.y);
-#pragma unroll
-          for (int g = 0; g < G; ++g) {
-            const float4 q = *reinterpret_cast<const float4*>(qs + g * HD + spart * 32 + e2 * 4);
-            sg[g] = fmaf(q.x, k0, fmaf(q.y, k1, fmaf(q.z, k2, fmaf(q.w, k3, sg[g]))));
-          }
+        for (int kp = 0; kp < KS / 2; ++kp) {
+          uint32_t bk[4];
+          ldmatrix_x4(bk, sb + kv_off<HD>(pw0 + 8 * t + lrow, 4 * kp + lmat));
+          mma_bf16_16816(acc[0], qa[2 * kp], bk[0], bk[1]);
+          mma_bf16_16816(acc[1], qa[2 * kp + 1], bk[2], bk[3]);
         }
-      }
+        const int i0 = pw0 + 8 * t + 2 * c;
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        float v = sg[g];
-#pragma unroll
-        for (int off = 1; off < TPP; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (spart == 0 && si < cn) sc[g * BP + ch * CP + si] = v;
+        for (int h = 0; h < NH; ++h) {
+          const float y0 = acc[0][2 * h] + acc[1][2 * h], y1 = acc[0][2 * h + 1] + acc[1][2 * h + 1];
+          const float x0 = y0 + __shfl_xor_sync(0xffffffffu, y0, 4);
+          const float x1 = y1 + __shfl_xor_sync(0xffffffffu, y1, 4);
+          s[t][h][0] = i0 < cn ? x0 : -INFINITY;
+          s[t][h][1] = i0 + 1 < cn ? x1 : -INFINITY;
+        }
       }
       ring_release(ring);
     }
-    cbar();
-    // ---- online softmax over the block (one warp per head)
-    if (warp < G) {
-      const int g = warp;
+    // ---- the warp's online-softmax update of its heads
+    uint32_t bp[NT][NH];   // the B fragments: hi (g even) or lo (g odd) of the probabilities
+#pragma unroll
+    for (int h = 0; h < NH; ++h) {
       float mx = -INFINITY;
-      for (int i = lane; i < bn; i += 32) mx = fmaxf(mx, sc[g * BP + i]);
-      mx = warp_max(mx);
-      const float mo = mrun[g];
-      const float mn = fmaxf(mo, mx);
-      float sum = 0.f;
-      for (int i = lane; i < bn; i += 32) {
-        const float e = exp2f(sc[g * BP + i] - mn);
-        sc[g * BP + i] = e;
-        sum += e;
-      }
-      sum = warp_sum(sum);
-      if (lane == 0) {
-        const float cr = exp2f(mo - mn);
-        corr[g] = cr;
-        lrun[g] = lrun[g] * cr + sum;
-        mrun[g] = mn;
+#pragma unroll
+      for (int t = 0; t < NT; ++t) mx = fmaxf(mx, fmaxf(s[t][h][0], s[t][h][1]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float mn = fmaxf(mrun[h], mx);
+      const float mu = mn == -INFINITY ? 0.f : mn;   // no position yet: every weight is 0
+      const float cr = exp2f(mrun[h] - mu);
+      mrun[h] = mn;
+      lrun[h] *= cr;
+      // o^T's columns are heads c + 4 h: their factor from lane (2 c, 0)
+      const float co = __shfl_sync(0xffffffffu, cr, 8 * c);
+#pragma unroll
+      for (int m = 0; m < MT; ++m)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) o[m][h][q] *= co;
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+        const float p0 = exp2f(s[t][h][0] - mu), p1 = exp2f(s[t][h][1] - mu);
+        lrun[h] += p0 + p1;
+        uint32_t hi, lo;
+        split_bf16x2(p0, p1, hi, lo);
+        bp[t][h] = g & 1 ? lo : hi;
       }
     }
-    cbar();
-    // ---- values
-#pragma unroll
-    for (int g = 0; g < G; ++g) o[g] *= corr[g];
-    for (int ch = 0; ch < nch; ++ch) {
-      const int c0 = b0 + ch * CP, cn = min(CP, u.r1 - c0);
-      const int stable = att_stable(a, u, c0, cn);
+    // ---- values: o^T += V^T p^T over the warp's positions
+    {
       uint8_t* st = const_cast<uint8_t*>(ring_acquire(ring, a.status, ok));
       if (!ok) return false;
       if (stable < cn) mk_patch<HD>(a, a.vc, l, u, st, c0, stable, cn, vn);
-      const __nv_bfloat16* vs = reinterpret_cast<const __nv_bfloat16*>(st);
-      const float* pb = sc + ch * CP;
+      const uint32_t sb = smem_u32(st);
+      const bool ragged = cn < CP;
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        // four interleaved partial sums over the chunk's positions
-        float t[4] = {0.f, 0.f, 0.f, 0.f};
-        int i = part;
-        for (; i + 3 * NPART < cn; i += 4 * NPART) {
+      for (int q = 0; q < 4; ++q) {
+        uint32_t av[4];
+        if constexpr (NT == 1) {
+          // k8: matrix i is the warp's 8 rows x dimensions 8 (4 q + i), the
+          // A fragments of m-tiles 2 q (i = 0, 1) and 2 q + 1 (i = 2, 3)
+          ldmatrix_x4_trans(av, sb + kv_off<HD>(pw0 + lrow, 4 * q + lmat));
+          if (ragged)
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            t[q] = fmaf(pb[g * BP + i + q * NPART], __bfloat162float(vs[(i + q * NPART) * HD + dim]), t[q]);
+            for (int i = 0; i < 4; ++i) av[i] = kv_mask(av[i], pw0 + 2 * c, cn);
+#pragma unroll
+          for (int h = 0; h < NH; ++h) {
+            mma_bf16_1688(o[2 * q][h], av[0], av[1], bp[0][h]);
+            mma_bf16_1688(o[2 * q + 1][h], av[2], av[3], bp[0][h]);
+          }
+        } else {
+          // k16: matrices (rows 0..7 | 8..15) x (dimensions 16 q + 0..7 | + 8..15)
+          ldmatrix_x4_trans(av, sb + kv_off<HD>(pw0 + 8 * (lmat >> 1) + lrow, 2 * q + (lmat & 1)));
+          if (ragged)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) av[i] = kv_mask(av[i], pw0 + 8 * (i >> 1) + 2 * c, cn);
+#pragma unroll
+          for (int h = 0; h < NH; ++h) mma_bf16_16816(o[q][h], av, bp[0][h], bp[NT - 1][h]);
         }
-        for (; i < cn; i += NPART) t[0] = fmaf(pb[g * BP + i], __bfloat162float(vs[i * HD + dim]), t[0]);
-        o[g] += (t[0] + t[1]) + (t[2] + t[3]);
       }
       ring_release(ring);
     }
-    cbar();   // the block's scores are read before the next block overwrites them
   }
+  // ---- the warp's partials (max, sum, o of each head) overlay the q
+  // fragments and new rows once every warp is done with them; then the 8
+  // are merged (weights exp2(max_w - max))
+  cbar();
+  float* osum = reinterpret_cast<float*>(att_sm);   // [8][G][HD]
+  float* wml = osum + kMkWarps * G * HD;            // [8][G][2]
 #pragma unroll
-  for (int g = 0; g < G; ++g) osum[(part * G + g) * HD + dim] = o[g];
+  for (int h = 0; h < NH; ++h) {
+    lrun[h] += __shfl_xor_sync(0xffffffffu, lrun[h], 1);
+    lrun[h] += __shfl_xor_sync(0xffffffffu, lrun[h], 2);
+    const int ho = c + 4 * h;   // o's head
+    if (ho < G) {
+      float* ow = osum + (warp * G + ho) * HD;
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        ow[16 * m + g] = o[m][h][0] + o[m][h][1];
+        ow[16 * m + g + 8] = o[m][h][2] + o[m][h][3];
+      }
+    }
+    const int hs = (g >> 1) + 4 * h;   // the softmax's head
+    if ((g & 1) == 0 && c == 0 && hs < G) {
+      wml[(warp * G + hs) * 2] = mrun[h];
+      wml[(warp * G + hs) * 2 + 1] = lrun[h];
+    }
+  }
   cbar();
   const size_t stride = HD + 2;
   for (int i = tid; i < G * HD; i += kMkCompute) {
-    const int g = i / HD, dd = i % HD;
-    float s = 0.f;
+    const int gg = i / HD, dd = i % HD;
+    float m = -INFINITY;
 #pragma unroll
-    for (int q = 0; q < NPART; ++q) s += osum[(q * G + g) * HD + dd];
-    a.att[((static_cast<size_t>(u.b) * a.Hq + u.kvh * G + g) * a.P + u.p) * stride + 2 + dd] = s;
-  }
-  if (tid < G) {
-    float* dst = a.att + ((static_cast<size_t>(u.b) * a.Hq + u.kvh * G + tid) * a.P + u.p) * stride;
-    dst[0] = mrun[tid];
-    dst[1] = lrun[tid];
+    for (int w = 0; w < kMkWarps; ++w) m = fmaxf(m, wml[(w * G + gg) * 2]);
+    float v = 0.f, sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kMkWarps; ++w) {
+      const float mw = wml[(w * G + gg) * 2];
+      if (mw != -INFINITY) {
+        const float e = exp2f(mw - m);
+        v = fmaf(e, osum[(w * G + gg) * HD + dd], v);
+        if (dd == 0) sum = fmaf(e, wml[(w * G + gg) * 2 + 1], sum);
+      }
+    }
+    float* dst = a.att + ((static_cast<size_t>(u.b) * a.Hq + u.kvh * G + gg) * a.P + u.p) * stride;
+    dst[2 + dd] = v;
+    if (dd == 0) {
+      dst[0] = m;
+      dst[1] = sum;
+    }
   }
   return true;
 }
@@ -866,7 +970,11 @@ __device__ __forceinline__ bool mk_attention_any(const MkArgs& a, int l, const A
     case 1: return mk_attention<HD, 1>(a, l, u, ring, att_sm);
     case 2: return mk_attention<HD, 2>(a, l, u, ring, att_sm);
     case 4: return mk_attention<HD, 4>(a, l, u, ring, att_sm);
-    default: return mk_attention<HD, 8>(a, l, u, ring, att_sm);
+    default:
+      // a group of 8 at head_dim 128 (o^T in 64 registers a lane) is not
+      // given to this kernel
+      if constexpr (HD == 64) return mk_attention<HD, 8>(a, l, u, ring, att_sm);
+      return false;
   }
 }
 

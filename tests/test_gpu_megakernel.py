@@ -11,7 +11,9 @@ layers through the same kernel.  Checked through the C-ABI:
 * losslessness (Sec. 3.3): the DVI stream equals the GPU's greedy AR stream
   bit for bit with the drafter training online: tiny bf16 (head_dim 128,
   eagerly and with graphs), the bonus row, head_dim 64 with a GQA group of 4,
-  two ragged sequences in one launch, the 1B and 7B workloads at full size;
+  two ragged sequences in one launch, the 1B and 7B workloads at full size,
+  the 7B shape with a 16K-token prompt (64 key / value chunks per attention
+  unit);
 * the verifier logits of the first step's verify rows (whose inputs h_k the
   kernel computed) against the oracle's teacher-forced logits on the
   bf16-rounded weights with a bf16 KV cache, within 3e-2 (every logged row of
@@ -150,3 +152,12 @@ def test_7b_full_size_lossless_and_first_step():
     cap = max(len(p) for p in P) + w.gen_tokens * w.k_spec + 64
     _lossless(w, W=W, max_seq_len=cap)
     _check_first_step(w, W, P, max_seq_len=cap)
+
+
+def test_7b_16k_context_lossless():
+    w = workload("7b-16k").with_(gen_tokens=12)
+    W = make_weights(w)
+    P = make_prompts(w)
+    assert len(P[0]) == 16384
+    cap = len(P[0]) + w.gen_tokens * w.k_spec + 64
+    _lossless(w, W=W, max_seq_len=cap)

@@ -8,7 +8,7 @@ import pytest
 
 from paper_2510_05421_gb300 import build as build_mod
 from paper_2510_05421_gb300 import dvi as D
-from workloads import WORKLOADS
+from workloads import WORKLOADS, tiny_shape
 
 HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "dvi.h")
 
@@ -167,13 +167,13 @@ def test_noalloc_args_rejected_before_any_launch(monkeypatch, case):
 
 
 @pytest.mark.parametrize("name,takes", [("tiny", False), ("1b", True), ("7b", True), ("7b-b8", False),
-                                        ("7b-16k", False)])
+                                        ("7b-16k", True)])
 def test_megakernel_workspace(L, name, takes):
     """The draft-phase megakernel's scratch (residual, projections, attention
-    partials, B u partials, argmax keys, counters, weight descriptors) is
-    reserved exactly for the contexts it takes: bf16, at most 2 sequences,
-    d_ffn a multiple of 64, max_seq_len <= 8192 (tiny: f32; 7b-b8: 8
-    sequences; 7b-16k: a 16K context)."""
+    partials, B u partials, argmax keys, counters, weight and cache
+    descriptors) is reserved exactly for the contexts it takes: bf16, at most
+    2 sequences, d_ffn a multiple of 64, any context length (tiny: f32;
+    7b-b8: 8 sequences; 7b-16k: a 16K context)."""
     w = WORKLOADS[name]
     cfg, rt0 = _cfgs(w, megakernel=0)
     _, rt1 = _cfgs(w, megakernel=1)
@@ -199,3 +199,17 @@ def test_megakernel_bf16_small_ffn_not_taken(L):
     assert w.shape.d_ffn % 64 != 0
     assert L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt1)) == \
         L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt0))
+
+
+@pytest.mark.parametrize("head_dim,takes", [(64, True), (128, False)])
+def test_megakernel_gqa8_only_at_head_dim_64(L, head_dim, takes):
+    """A GQA group of 8 goes to the megakernel at head_dim 64 only (at 128 a
+    lane's o^T tile of 8 heads would take 64 registers)."""
+    shape = tiny_shape(n_layers=4, d_model=16 * head_dim, n_heads=16, n_kv_heads=2, head_dim=head_dim,
+                       d_ffn=1408, vocab=4000)
+    w = WORKLOADS["tiny"].with_(dtype="bf16", shape=shape)
+    cfg, rt0 = _cfgs(w, megakernel=0)
+    _, rt1 = _cfgs(w, megakernel=1)
+    n0 = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt0))
+    n1 = L.dvi_workspace_bytes(ctypes.byref(cfg), ctypes.byref(rt1))
+    assert n0 > 0 and (n1 > n0) == takes and n1 >= n0
