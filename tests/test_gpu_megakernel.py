@@ -10,8 +10,8 @@ layers through the same kernel.  Checked through the C-ABI:
   megakernel = 0, is checked the same way on the tiny model);
 * losslessness (Sec. 3.3): the DVI stream equals the GPU's greedy AR stream
   bit for bit with the drafter training online: tiny bf16 (head_dim 128,
-  eagerly and with graphs), the bonus row, head_dim 64 with a GQA group of 4,
-  two ragged sequences in one launch, the 1B and 7B workloads at full size,
+  eagerly and with graphs), the bonus row, head_dim 64 with GQA groups of 4
+  and 8, two ragged sequences in one launch, the 1B and 7B workloads at full size,
   the 7B shape with a 16K-token prompt (64 key / value chunks per attention
   unit);
 * the verifier logits of the first step's verify rows (whose inputs h_k the
@@ -116,6 +116,15 @@ def test_tiny_bf16_bonus_lossless():
 
 def test_head_dim_64_gqa4_lossless_and_oracle():
     shape = tiny_shape(n_layers=4, d_model=512, n_heads=8, n_kv_heads=2, head_dim=64, d_ffn=1408, vocab=4000)
+    w = _bf16_case().with_(shape=shape)
+    W, P, _ = _lossless(w)
+    _check_first_step(w, W, P)
+
+
+def test_head_dim_64_gqa8_lossless_and_oracle():
+    """A GQA group of 8: the score and value MMAs take two head tiles (query
+    heads 4..7 in A rows 8..15 and in o^T's second column tile)."""
+    shape = tiny_shape(n_layers=4, d_model=1024, n_heads=16, n_kv_heads=2, head_dim=64, d_ffn=1408, vocab=4000)
     w = _bf16_case().with_(shape=shape)
     W, P, _ = _lossless(w)
     _check_first_step(w, W, P)
