@@ -30,10 +30,12 @@
 //
 // The attention of a decode row at position pos splits [0, pos] into P equal
 // ranges (a function of pos only, so a draft pass and a greedy AR step at the
-// same position reduce in the same order).  Cached positions below the
-// sequence's committed length are streamed by the ring; positions written
-// earlier in this launch and the newest one are filled into the stage from
-// global memory and from the pass's own K/V.
+// same position reduce in the same order).  The ring streams a range in
+// chunks of 8192 / hd cached positions, keys then values, each one 16 KB TMA
+// box; positions written earlier in this launch and the newest one are
+// filled into the stage from global memory and from the pass's own K/V.
+// Scores and values run on the warp tensor cores too (each warp owning a
+// slice of a chunk's positions, with its own online softmax).
 #include "common.cuh"
 #include "kernels.h"
 
