@@ -378,8 +378,10 @@ void size_scratch(dvi_ctx* c) {
 // The draft-phase megakernel's static arguments and scratch (runtime option
 // megakernel): bf16, at most kMkMaxRows sequences, k <= kMkMaxLayers shallow
 // layers, GQA groups of 1, 2, 4 or 8 (8 only at head_dim 64), d a multiple of
-// 128, d_ffn of 64, fewer than 2^31 cache rows (its KV boxes take a 32-bit
-// row), and a ring of at least four 16 KB stages beside the kernel's other
+// 128, d_ffn of 64, a cache of fewer than 2^31 - 65536 rows (its KV boxes
+// take a 32-bit row, and a range's last chunk may start past max_seq_len
+// when the cache is full), and a ring of at least four 16 KB stages beside
+// the kernel's other
 // shared memory.  No context bound: its attention streams each unit's range
 // at the ring's pace (measured ahead of the per-kernel draft path from 1K to
 // 16K positions).
@@ -389,7 +391,7 @@ void size_mk(dvi_ctx* c) {
       c->d % 128 || c->F % 64 || (c->hd != 64 && c->hd != 128) || c->B * c->Hkv > c->n_sms ||
       (c->Hq / c->Hkv != 1 && c->Hq / c->Hkv != 2 && c->Hq / c->Hkv != 4 && c->Hq / c->Hkv != 8) ||
       (c->hd == 128 && c->Hq / c->Hkv == 8) ||
-      static_cast<long long>(c->L) * c->B * c->Hkv * c->max_len > std::numeric_limits<int>::max())
+      static_cast<long long>(c->L) * c->B * c->Hkv * c->max_len + 65536 > std::numeric_limits<int>::max())
     return;
   MkArgs& a = c->mk;
   a = MkArgs{};

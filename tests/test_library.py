@@ -215,11 +215,13 @@ def test_megakernel_gqa8_only_at_head_dim_64(L, head_dim, takes):
     assert n0 > 0 and (n1 > n0) == takes and n1 >= n0
 
 
-@pytest.mark.parametrize("max_seq_len,takes", [((1 << 21) - 1, True), (1 << 21, False)])
+@pytest.mark.parametrize("max_seq_len,takes", [(2097087, True), (2097088, False)])
 def test_megakernel_cache_rows_below_2_31(L, max_seq_len, takes):
     """The megakernel's key / value boxes address the cache by a 32-bit row
-    (layers x sequences x KV heads x max_seq_len): the 7B shape (32 x 1 x 32
-    rows per position) is taken up to 2^21 - 1 positions, not at 2^21."""
+    (layers x sequences x KV heads x max_seq_len, plus 65536 rows of margin
+    for a chunk that starts past a full cache): the 7B shape (32 x 1 x 32
+    rows per position) is taken up to (2^31 - 1 - 65536) / 1024 = 2097087
+    positions."""
     w = WORKLOADS["7b"]
     cfg, rt0 = _cfgs(w, megakernel=0)
     _, rt1 = _cfgs(w, megakernel=1)
